@@ -1,0 +1,273 @@
+/*
+ * csr.h -- C ABI of the CSR incremental-prefill attention library (libcsr.so).
+ *
+ * The library keeps one transformer layer's key/value cache for the Cached
+ * State Representation of section III-D of the paper:
+ *
+ *     T_t = (X_static, X_dyn),  X_static = (X_pre, X_chunks),  X_dyn = (X_suff, X_task)
+ *
+ * X_pre is cached once (csr_init_static), state chunks are appended
+ * (csr_append_chunk, Theorem 2 / Eq. incremental_extensibility), the dynamic
+ * suffix is attended and dropped again every task (csr_attend_suffix,
+ * csr_truncate_suffix; Eq. x_dynamic), and old chunks are evicted
+ * (Eq. eviction_operation) with the asynchronous state reconciliation of
+ * Algorithm 1 (csr_evict_and_reconcile, csr_poll_swap).  Every call that adds
+ * tokens rotates them with RoPE at their absolute positions, appends their
+ * keys/values to a paged cache and returns the causal attention of their
+ * queries over the whole cached context (Eq. causal_attention_1..3).
+ *
+ * Conventions shared by every entry point
+ *   - Tensors are bfloat16 in row-major, token-major layout:
+ *       q, out   [n][num_q_heads][head_dim]
+ *       k, v     [n][num_kv_heads][head_dim]
+ *       lse      [num_q_heads][n] float32, natural log of the softmax
+ *                normaliser sum_tau exp(scale * q.k_tau)
+ *     All tensor pointers are DEVICE pointers of the current CUDA device,
+ *     16-byte aligned, owned by the caller, borrowed for the call only (the
+ *     pools and the workspace are borrowed for the context's lifetime).
+ *   - Compute calls are asynchronous: they enqueue kernels on the given
+ *     stream and return.  Inputs must stay valid until that work has run.
+ *   - Foreground calls share one workspace; issue them on one stream, or
+ *     order them yourself.
+ *   - Errors are returned as csr_status; nothing is thrown across the ABI.
+ *     A call that fails with CSR_EINVAL, CSR_ESTATE or CSR_ENOMEM changes
+ *     nothing.  csr_last_error() describes the last failure.
+ *   - Query head h reads key/value head h / (num_q_heads / num_kv_heads).
+ *   - RoPE pairs element i with element i + head_dim/2 (rotate-half) and
+ *     turns the pair by pos * rope_base^(-2i/head_dim).
+ *   - A context is not thread-safe: call it from one host thread at a time.
+ */
+#ifndef CSR_H_
+#define CSR_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Same object as cudaStream_t; NULL is the legacy default stream. */
+typedef struct CUstream_st *csr_stream_t;
+
+typedef struct csr_ctx csr_ctx;
+
+typedef enum csr_status {
+  CSR_OK = 0,
+  CSR_EINVAL = 1,   /* bad argument or configuration */
+  CSR_ENOMEM = 2,   /* the page pool or a version's page table is full */
+  CSR_ESTATE = 3,   /* call not allowed in the current state */
+  CSR_EBUSY = 4,    /* a reconciliation is already running */
+  CSR_ECUDA = 5,    /* a CUDA runtime or driver call failed */
+  CSR_ETIMEOUT = 6, /* a bounded host-side wait ran out */
+  CSR_EDEVICE = 7   /* a kernel reported an error word (see csr_device_status) */
+} csr_status;
+
+/* Bits of the device error word. */
+#define CSR_DEVERR_WAIT_TIMEOUT 0x1u /* a pipeline wait inside a kernel gave up */
+#define CSR_DEVERR_BAD_PAGE 0x2u     /* a page id outside the pool was met */
+#define CSR_DEVERR_ALLOC 0x4u        /* the compaction kernel found too few free pages */
+
+/* csr_config.flags */
+#define CSR_FLAG_PLAN_ONLY 0x1 /* layout planning only: no device memory is touched
+                                  and no kernel runs; compute calls update the page
+                                  tables and lengths but produce no outputs */
+
+typedef struct csr_config {
+  int32_t num_q_heads;    /* H_q */
+  int32_t num_kv_heads;   /* H_kv; H_q / H_kv must be a power of two <= 128 */
+  int32_t head_dim;       /* 64 or 128 */
+  int32_t page_size;      /* tokens per cache page: 16, 32, 64 or 128 */
+  double rope_base;       /* RoPE base (e.g. 1e4, 1e6) */
+  float softmax_scale;    /* 0 selects 1/sqrt(head_dim) (Eq. causal_attention_1) */
+  int32_t max_new_tokens; /* largest n of one call, and of one chunk */
+  int32_t pool_pages;     /* physical pages in each of the K and V pools (<= 65536) */
+  int32_t max_seq_tokens; /* largest length of one cache version */
+  int32_t cap_tokens;     /* tau_mem of Algorithm 1; 0 disables automatic eviction */
+  int32_t evict_tokens;   /* tokens of the oldest chunks dropped by an automatic eviction */
+  int32_t n_catchup;      /* N_catchup of Algorithm 1 */
+  int32_t num_ctas;       /* CTAs of a foreground attention launch; 0 = one per SM */
+  int32_t rebuild_tiles_per_cta; /* key tiles per CTA in rebuild launches; 0 = 64 */
+  int32_t flags;          /* CSR_FLAG_* */
+} csr_config;
+
+/*
+ * Sizes of the caller-allocated device buffers for a configuration.
+ * csr_pool_bytes: bytes of EACH of the K and V pools, laid out
+ *   [pool_pages][num_kv_heads][page_size][head_dim] bfloat16.
+ * csr_workspace_bytes: bytes of the workspace (staging, split partials, page
+ *   tables, error word).  Both return 0 for an invalid configuration.
+ */
+size_t csr_pool_bytes(const csr_config *cfg);
+size_t csr_workspace_bytes(const csr_config *cfg);
+
+/*
+ * Create a context on the current CUDA device.  k_pool, v_pool (csr_pool_bytes
+ * each, 256-byte aligned) and workspace (csr_workspace_bytes, 256-byte aligned)
+ * are borrowed until csr_destroy; create zero-fills them on `stream`.
+ * With CSR_FLAG_PLAN_ONLY the three pointers may be NULL and no CUDA call is
+ * made.  On success *out receives the context.
+ */
+csr_status csr_create(const csr_config *cfg, void *k_pool, void *v_pool,
+                      void *workspace, csr_stream_t stream, csr_ctx **out);
+
+/* Release the context (synchronises its streams first).  NULL is a no-op. */
+void csr_destroy(csr_ctx *ctx);
+
+/*
+ * X_pre (Eq. x_static): cache the static prefix at positions 0..n-1 and write
+ * its causal self-attention to out (and lse when not NULL).  Once per context,
+ * before any other compute call; 1 <= n <= max_new_tokens.  Prefixes longer
+ * than max_new_tokens are built by csr_init_static followed by chunks.
+ */
+csr_status csr_init_static(csr_ctx *ctx, const void *q, const void *k,
+                           const void *v, int32_t n, void *out, float *lse,
+                           csr_stream_t stream);
+
+/*
+ * Increment of Algorithm 1: append the state chunk x_t at positions
+ * len..len+n-1 of the active version, attend its queries over the whole cache,
+ * and return its id in *chunk_id (may be NULL).  While a reconciliation runs
+ * the chunk is also reserved in the version being rebuilt and buffered for its
+ * catch-up.  If a reconciler is set, cap_tokens > 0 and the length reaches
+ * cap_tokens, an eviction of evict_tokens starts (Algorithm 1, Increment); if
+ * it cannot start, the chunk stays appended and its error code is returned.
+ * CSR_ESTATE while a suffix is live.
+ */
+csr_status csr_append_chunk(csr_ctx *ctx, const void *q, const void *k,
+                            const void *v, int32_t n, void *out, float *lse,
+                            csr_stream_t stream, int64_t *chunk_id);
+
+/*
+ * X_dyn = (X_suff, X_task) (Eq. x_dynamic, i* = |X_static| + 1 of
+ * Eq. csr_i_star): append the transient suffix at positions len..len+n-1 and
+ * attend it causally over the cache.  At most one suffix is live: CSR_ESTATE
+ * otherwise.
+ */
+csr_status csr_attend_suffix(csr_ctx *ctx, const void *q, const void *k,
+                             const void *v, int32_t n, void *out, float *lse,
+                             csr_stream_t stream);
+
+/*
+ * Drop the live suffix: the length returns to |X_static| and the pages that
+ * hold only suffix slots go back to the pool.  Host-only (no kernel).
+ * CSR_ESTATE when no suffix is live.
+ */
+csr_status csr_truncate_suffix(csr_ctx *ctx);
+
+/*
+ * Source of a chunk's layer inputs for the rebuild (the "LLM(X_eps)" of
+ * Algorithm 1 recomputes a retained chunk in its new context).  The callback
+ * is called on the thread that drives the context, with the chunk's id and
+ * length, and must set *q, *k, *v to device pointers holding that chunk's
+ * pre-RoPE queries/keys/values in the layouts above, valid until the
+ * reconciliation that asked for them has swapped or failed.  It may set *out
+ * to a device buffer [n][num_q_heads][head_dim] that receives the chunk's
+ * rebuilt attention output, or leave it NULL.  Returns 0 on success; any other
+ * value aborts the reconciliation (the active version stays as it is).
+ */
+typedef int (*csr_qkv_provider)(void *user, int64_t chunk_id, int32_t n_tokens,
+                                const void **q, const void **k, const void **v,
+                                void **out);
+
+/*
+ * Register the rebuild source and the low-priority stream on which the
+ * rebuild runs (the secondary resource R_2 of Algorithm 1 becomes a stream of
+ * the same GPU).  Create lo_stream with a lower priority than the foreground
+ * stream.  CSR_EBUSY while a reconciliation runs.
+ */
+csr_status csr_set_reconciler(csr_ctx *ctx, csr_qkv_provider provider,
+                              void *user, csr_stream_t lo_stream);
+
+/*
+ * Eviction + asynchronous reconciliation (Eq. eviction_operation, Algorithm 1
+ * Reconcile, App. D steps 1-3): drop the oldest whole chunks until at least
+ * evict_tokens tokens are gone, reserve a second cache version that shares the
+ * prefix's full pages, and enqueue on the low-priority stream the compaction
+ * kernel (new page table, copy of a partly filled prefix page) and a fresh
+ * causal prefill of every retained chunk at its renumbered position.  Work
+ * already enqueued on fg_stream is ordered before the rebuild.  Returns at
+ * once; the active version keeps serving foreground calls.
+ * CSR_EBUSY if a reconciliation runs, CSR_ESTATE without a reconciler, with a
+ * live suffix or with no chunk to evict, CSR_ENOMEM if the pool cannot hold
+ * the second version.
+ */
+csr_status csr_evict_and_reconcile(csr_ctx *ctx, int32_t evict_tokens,
+                                   csr_stream_t fg_stream);
+
+/* Values of *state from csr_poll_swap / csr_wait_reconcile. */
+#define CSR_RECON_IDLE 0    /* no reconciliation */
+#define CSR_RECON_RUNNING 1 /* rebuild or catch-up still running (or swap deferred) */
+#define CSR_RECON_SWAPPED 2 /* this call swapped the versions */
+
+/*
+ * Non-blocking step of Algorithm 1's catch-up loop.  When the rebuild's last
+ * launch has finished: while more than n_catchup chunks are buffered, enqueue
+ * their catch-up on the low-priority stream; otherwise compute the remaining
+ * buffered chunks on fg_stream ("computed at next task inference") and swap
+ * the active version atomically (App. D step 5).  The old version's own pages
+ * return to the pool.  The swap waits while a suffix is live.
+ */
+csr_status csr_poll_swap(csr_ctx *ctx, csr_stream_t fg_stream, int *state);
+
+/*
+ * Blocking form of csr_poll_swap: polls until the swap happens or timeout_us
+ * microseconds pass (CSR_ETIMEOUT; the reconciliation keeps running).
+ */
+csr_status csr_wait_reconcile(csr_ctx *ctx, csr_stream_t fg_stream,
+                              int64_t timeout_us, int *state);
+
+/* Which version an inspection call reads. */
+#define CSR_VERSION_ACTIVE 0
+#define CSR_VERSION_PENDING 1
+
+/*
+ * Host view of a version's layout: its page table (logical page i holds
+ * positions i*page_size .. i*page_size+page_size-1 in physical page
+ * page_table[i]; the slot of position p is page_table[p/P]*P + p%P), its page
+ * count and length.  page_table may be NULL to query the count; capacity is
+ * its length in entries.  CSR_ESTATE for PENDING without a reconciliation.
+ */
+csr_status csr_get_layout(csr_ctx *ctx, int which, int32_t *page_table,
+                          int32_t capacity, int32_t *n_pages, int64_t *length);
+
+/* Ascending ids of the free physical pages (ids may be NULL to count). */
+csr_status csr_get_free_pages(csr_ctx *ctx, int32_t *ids, int32_t capacity,
+                              int32_t *count);
+
+/*
+ * Chunk ids and lengths of a version in order (X_chunks), and its prefix
+ * length.  Arrays may be NULL to count.
+ */
+csr_status csr_get_chunks(csr_ctx *ctx, int which, int64_t *ids, int32_t *lens,
+                          int32_t capacity, int32_t *count, int64_t *prefix_len);
+
+/* Device pointer of a version's page table (int32, n_pages entries). */
+csr_status csr_device_page_table(csr_ctx *ctx, int which, const int32_t **ptr);
+
+/*
+ * Gather the cached (rotated) keys and the values of positions pos0..pos0+n-1
+ * of a version into k_out, v_out [n][num_kv_heads][head_dim] (device), on
+ * stream.  For inspection and tests.
+ */
+csr_status csr_gather_kv(csr_ctx *ctx, int which, int64_t pos0, int32_t n,
+                         void *k_out, void *v_out, csr_stream_t stream);
+
+/*
+ * Wait for all of the context's device work (device-wide synchronise), then
+ * return and clear the device error word (CSR_DEVERR_* bits) in *flags.
+ * Returns CSR_EDEVICE when a bit was set.
+ */
+csr_status csr_device_status(csr_ctx *ctx, uint32_t *flags);
+
+/* Number of kernels the context has launched since creation. */
+int64_t csr_kernel_launches(const csr_ctx *ctx);
+
+/* Text of the last failure on this context (never NULL). */
+const char *csr_last_error(const csr_ctx *ctx);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* CSR_H_ */

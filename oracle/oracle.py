@@ -208,6 +208,7 @@ class OracleCSR:
         self.prefix_len = 0
         self.has_static = False
         self.threads = threads
+        self.attend = True   # False: cache bookkeeping only (fill phases)
 
     # ---- helpers ---------------------------------------------------------
     @property
@@ -226,14 +227,17 @@ class OracleCSR:
         return attention(q_rot, qpos, k, v, kpos, self.scale, self.threads)
 
     def _add(self, ver: Version, kind: str, ident: int, q, k, v):
-        """Rotate the block at positions len..len+n-1, cache it, attend it."""
+        """Rotate the block at positions len..len+n-1, cache it, attend it
+        (the attention is skipped while ``self.attend`` is False)."""
         n = q.shape[0]
         L = ver.length
         pos = np.arange(L, L + n, dtype=np.int64)
         self._grow(ver, L + n)
-        q_rot = rope(q, pos, self.base)
         k_rot = rope(k, pos, self.base)
         ver.segments.append(Segment(kind, ident, pos, k_rot, np.array(v, np.float64)))
+        if not self.attend:
+            return None, None
+        q_rot = rope(q, pos, self.base)
         return self._attend_new(ver, q_rot, pos)
 
     # ---- operations --------------------------------------------------------
@@ -255,6 +259,8 @@ class OracleCSR:
                              np.array(v, np.float64))
         was_reconciling = self.is_reconciling
         out = self._add(self.active, "chunk", cid, q, k, v)
+        if not self.attend:
+            self.sources.pop(cid, None)   # fill-phase chunks are never rebuilt
         if was_reconciling:
             # reserve the rebuilt version's pages now (reading R4), buffer the chunk
             start = self.pending.length
@@ -327,6 +333,8 @@ class OracleCSR:
         """Re-prefill one chunk of ``ver`` at its renumbered position (R5)."""
         idx = [i for i, s in enumerate(ver.segments) if s.kind == "chunk" and s.ident == cid][0]
         pos = ver.segments[idx].pos
+        if cid not in self.sources:      # bookkeeping-only session (attend False)
+            return None, None
         q, k, v = self.sources[cid]
         q_rot = rope(q, pos, self.base)
         k_rot = rope(k, pos, self.base)

@@ -1,0 +1,877 @@
+// csr_api.cpp -- host side of libcsr: the C ABI of include/csr.h.
+//
+// Owns the cache bookkeeping of section III-D (X_pre, the ordered X_chunks,
+// the transient X_dyn suffix), the physical page pool (smallest free id
+// first), two cache versions (the active one and the one a reconciliation
+// rebuilds, Algorithm 1 / App. D), and the launch of the kernels:
+//   K1 rope_append  -> K2 attention (stream-K split) -> K3 merge   per block
+//   K4 evict_compact                                                per eviction
+// The foreground runs on the caller's stream; the rebuild and its catch-up
+// run on the low-priority stream registered with csr_set_reconciler.
+#include <algorithm>
+#include <atomic>
+#include <chrono>
+#include <cmath>
+#include <cstring>
+#include <string>
+#include <thread>
+#include <vector>
+
+#include <cuda.h>
+#include <cudaTypedefs.h>
+#include <cuda_runtime.h>
+
+#include "../../include/csr.h"
+#include "internal.h"
+
+using namespace csr;
+
+namespace {
+
+constexpr int kFgGridDefaultCap = 304;   // 2 x 152 SMs
+constexpr int kRebuildGridFactor = 8;    // rebuild CTAs per foreground CTA, at most
+constexpr int kDefaultRebuildTiles = 64;
+constexpr size_t kAlign = 256;
+
+size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+int64_t ceil_div(int64_t a, int64_t b) { return (a + b - 1) / b; }
+bool is_pow2(int64_t x) { return x > 0 && (x & (x - 1)) == 0; }
+
+// Physical page pool: bit set = free; each request takes the smallest free id.
+struct PagePool {
+  int32_t n = 0;
+  int32_t n_free = 0;
+  std::vector<uint32_t> free_bits;
+  std::vector<uint16_t> refs;
+
+  void init(int32_t pages) {
+    n = pages;
+    n_free = pages;
+    free_bits.assign(static_cast<size_t>(ceil_div(pages, 32)), 0u);
+    for (int32_t i = 0; i < pages; ++i) free_bits[i >> 5] |= 1u << (i & 31);
+    refs.assign(static_cast<size_t>(pages), 0);
+  }
+  int32_t take() {
+    for (size_t w = 0; w < free_bits.size(); ++w) {
+      if (free_bits[w]) {
+        const int b = __builtin_ctz(free_bits[w]);
+        free_bits[w] &= ~(1u << b);
+        const int32_t id = static_cast<int32_t>(w * 32 + b);
+        refs[id] = 1;
+        --n_free;
+        return id;
+      }
+    }
+    return -1;
+  }
+  void share(int32_t id) { ++refs[id]; }
+  void release(int32_t id) {
+    if (--refs[id] == 0) {
+      free_bits[id >> 5] |= 1u << (id & 31);
+      ++n_free;
+    }
+  }
+};
+
+struct ChunkRec {
+  int64_t id;
+  int32_t len;
+};
+
+struct Version {
+  std::vector<int32_t> pages;  // logical page -> physical page
+  int64_t prefix_len = 0;
+  std::vector<ChunkRec> chunks;
+  int32_t suffix_len = 0;
+  int64_t length() const {
+    int64_t L = prefix_len + suffix_len;
+    for (const auto &c : chunks) L += c.len;
+    return L;
+  }
+  void clear() {
+    pages.clear();
+    prefix_len = 0;
+    chunks.clear();
+    suffix_len = 0;
+  }
+};
+
+PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (!fn) {
+    void *p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  }
+  return fn;
+}
+
+// 2-D bf16 tensor map: rows x d elements, boxes of 64 columns x box_rows rows,
+// 128-byte swizzle (the layout the MMA descriptors describe).
+bool encode_rows(CUtensorMap *m, void *base, uint64_t rows, uint64_t d, uint32_t box_rows) {
+  auto fn = tensor_map_encoder();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {d, rows};
+  cuuint64_t strides[1] = {d * 2};
+  cuuint32_t box[2] = {64, box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, base, dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+struct Layout {  // workspace carve-out (byte offsets)
+  size_t qpack[2], rb_out, part_o[2], part_lse[2], pt[2], ids_out, err, total;
+  int32_t rows_cap, fg_cap, rb_cap, max_pages;
+};
+
+bool valid_config(const csr_config *c, std::string *why) {
+  auto bad = [&](const char *m) {
+    if (why) *why = m;
+    return false;
+  };
+  if (!c) return bad("config is NULL");
+  if (c->num_q_heads <= 0 || c->num_kv_heads <= 0 || c->num_q_heads % c->num_kv_heads)
+    return bad("num_q_heads must be a positive multiple of num_kv_heads");
+  const int g = c->num_q_heads / c->num_kv_heads;
+  if (!is_pow2(g) || g > kBM) return bad("num_q_heads/num_kv_heads must be a power of two <= 128");
+  if (c->head_dim != 64 && c->head_dim != 128) return bad("head_dim must be 64 or 128");
+  if (c->page_size != 16 && c->page_size != 32 && c->page_size != 64 && c->page_size != 128)
+    return bad("page_size must be 16, 32, 64 or 128");
+  if (!(c->rope_base > 1.0)) return bad("rope_base must be > 1");
+  if (c->softmax_scale < 0.f) return bad("softmax_scale must be >= 0");
+  if (c->max_new_tokens < 1) return bad("max_new_tokens must be >= 1");
+  if (c->max_new_tokens / c->page_size + 2 > kMaxIdsPerCall)
+    return bad("max_new_tokens / page_size too large for one launch");
+  if (c->pool_pages < 1 || c->pool_pages > 32 * kMaxPoolWords)
+    return bad("pool_pages must be in [1, 65536]");
+  if (c->max_seq_tokens < 1) return bad("max_seq_tokens must be >= 1");
+  if (static_cast<int64_t>(c->pool_pages) * c->num_kv_heads * c->page_size >= (1ll << 31))
+    return bad("pool rows exceed the 32-bit TMA coordinate range");
+  if (c->cap_tokens < 0 || c->evict_tokens < 0 || c->n_catchup < 0 || c->num_ctas < 0 ||
+      c->rebuild_tiles_per_cta < 0)
+    return bad("negative cap_tokens/evict_tokens/n_catchup/num_ctas/rebuild_tiles_per_cta");
+  if (c->cap_tokens > 0 && c->evict_tokens <= 0) return bad("cap_tokens needs evict_tokens > 0");
+  return true;
+}
+
+Layout make_layout(const csr_config *c) {
+  Layout L{};
+  const int g = c->num_q_heads / c->num_kv_heads;
+  L.rows_cap = static_cast<int32_t>(align_up(static_cast<size_t>(c->max_new_tokens) * g, kBM));
+  L.fg_cap = c->num_ctas > 0 ? c->num_ctas : kFgGridDefaultCap;
+  L.rb_cap = kRebuildGridFactor * (c->num_ctas > 0 ? c->num_ctas : 152);
+  L.max_pages = static_cast<int32_t>(ceil_div(c->max_seq_tokens, c->page_size) + 1);
+  const size_t d = static_cast<size_t>(c->head_dim);
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    const size_t o = off;
+    off = align_up(off + bytes, kAlign);
+    return o;
+  };
+  for (int i = 0; i < 2; ++i) L.qpack[i] = take(static_cast<size_t>(c->num_kv_heads) * L.rows_cap * d * 2);
+  L.rb_out = take(static_cast<size_t>(c->max_new_tokens) * c->num_q_heads * d * 2);
+  const int caps[2] = {L.fg_cap, L.rb_cap};
+  for (int i = 0; i < 2; ++i) {
+    L.part_o[i] = take(static_cast<size_t>(caps[i]) * 2 * kBM * d * 4);
+    L.part_lse[i] = take(static_cast<size_t>(caps[i]) * 2 * kBM * 4);
+  }
+  for (int i = 0; i < 2; ++i) L.pt[i] = take(static_cast<size_t>(L.max_pages) * 4);
+  L.ids_out = take(static_cast<size_t>(L.max_pages) * 4);
+  L.err = take(256);
+  L.total = off;
+  return L;
+}
+
+}  // namespace
+
+struct csr_ctx {
+  csr_config cfg{};
+  bool plan_only = false;
+  int device = 0, num_sms = 0, group = 1, fg_grid = 1;
+  Layout lay{};
+  uint16_t *k_pool = nullptr, *v_pool = nullptr;
+  uint8_t *ws = nullptr;
+  CUtensorMap tm_q[2]{}, tm_k{}, tm_v{};
+  double inv_turns[kMaxHalfDim]{};
+  float scale_log2 = 0.f;
+  PagePool pool;
+  Version ver[2];
+  std::atomic<int> active{0};
+  bool has_static = false;
+  int64_t next_chunk_id = 0;
+  // Algorithm 1 state
+  bool reconciling = false;
+  std::vector<ChunkRec> buffer;      // Delta X_buffer
+  int64_t rebuilt_len = 0;           // length of the pending version computed so far
+  std::vector<int32_t> reserved_ids; // fresh ids the compaction kernel must produce
+  bool ids_checked = false;
+  csr_qkv_provider provider = nullptr;
+  void *user = nullptr;
+  cudaStream_t lo = nullptr;
+  cudaEvent_t ev_fg = nullptr, ev_rb = nullptr;
+  int64_t launches = 0;
+  std::string err = "no error";
+
+  template <class T> T *wsp(size_t off) { return reinterpret_cast<T *>(ws + off); }
+  Version &act() { return ver[active.load()]; }
+  Version &pend() { return ver[1 - active.load()]; }
+  int32_t *d_pt(int slot) { return wsp<int32_t>(lay.pt[slot]); }
+};
+
+namespace {
+
+csr_status fail(csr_ctx *c, csr_status s, const std::string &msg) {
+  if (c) c->err = msg;
+  return s;
+}
+
+csr_status cuda_fail(csr_ctx *c, cudaError_t e, const char *where) {
+  return fail(c, CSR_ECUDA, std::string(where) + ": " + cudaGetErrorString(e));
+}
+
+int64_t pages_for(const csr_ctx *c, int64_t len) { return ceil_div(len, c->cfg.page_size); }
+
+// K1 -> K2 -> K3 for n tokens at positions L.. of version `slot`.
+// ws: 0 = foreground staging, 1 = rebuild staging.  ids/n_ids name the physical
+// pages of logical pages first_lp.. (written into the device table by K1);
+// n_ids == 0 reads the device table instead.
+csr_status run_block(csr_ctx *c, int slot, int ws, const void *q, const void *k, const void *v,
+                     int32_t n, int64_t L, const int32_t *ids, int32_t n_ids, int32_t first_lp,
+                     void *out, float *lse, cudaStream_t s) {
+  const csr_config &cf = c->cfg;
+  RopeAppendParams rp{};
+  rp.q = static_cast<const uint16_t *>(q);
+  rp.k = static_cast<const uint16_t *>(k);
+  rp.v = static_cast<const uint16_t *>(v);
+  rp.k_pool = c->k_pool;
+  rp.v_pool = c->v_pool;
+  rp.q_pack = c->wsp<uint16_t>(c->lay.qpack[ws]);
+  rp.page_table = c->d_pt(slot);
+  rp.err = c->wsp<uint32_t>(c->lay.err);
+  rp.pos0 = L;
+  rp.n = n;
+  rp.hq = cf.num_q_heads;
+  rp.hkv = cf.num_kv_heads;
+  rp.d = cf.head_dim;
+  rp.page_size = cf.page_size;
+  rp.group = c->group;
+  rp.rows_cap = c->lay.rows_cap;
+  rp.pool_pages = cf.pool_pages;
+  rp.first_lp = first_lp;
+  rp.n_ids = n_ids;
+  std::memcpy(rp.inv_turns, c->inv_turns, sizeof(rp.inv_turns));
+  for (int i = 0; i < n_ids; ++i) rp.ids[i] = ids[i];
+  cudaError_t e = launch_rope_append(rp, s);
+  if (e != cudaSuccess) return cuda_fail(c, e, "rope_append launch");
+  ++c->launches;
+
+  AttnParams ap{};
+  ap.tm_q = c->tm_q[ws];
+  ap.tm_k = c->tm_k;
+  ap.tm_v = c->tm_v;
+  ap.page_table = c->d_pt(slot);
+  ap.out = static_cast<uint16_t *>(out);
+  ap.lse = lse;
+  ap.part_o = c->wsp<float>(c->lay.part_o[ws]);
+  ap.part_lse = c->wsp<float>(c->lay.part_lse[ws]);
+  ap.err = rp.err;
+  ap.L = L;
+  ap.n = n;
+  ap.hq = cf.num_q_heads;
+  ap.hkv = cf.num_kv_heads;
+  ap.group = c->group;
+  ap.page_size = cf.page_size;
+  ap.rows_cap = c->lay.rows_cap;
+  ap.n_tiles = static_cast<int32_t>(ceil_div(static_cast<int64_t>(n) * c->group, kBM));
+  ap.n_pages_valid = static_cast<int32_t>(pages_for(c, L + n));
+  ap.pool_pages = cf.pool_pages;
+  const int T = kBM / c->group;
+  int64_t iph = 0;
+  for (int t = 0; t < ap.n_tiles; ++t) iph += unit_iters(L, n, T, t);
+  ap.iters_per_head = iph;
+  ap.total_iters = iph * cf.num_kv_heads;
+  int64_t grid;
+  if (ws == 0) {
+    grid = std::min<int64_t>(c->fg_grid, ap.total_iters);
+  } else {
+    const int tpc = cf.rebuild_tiles_per_cta > 0 ? cf.rebuild_tiles_per_cta : kDefaultRebuildTiles;
+    grid = std::max<int64_t>(std::min<int64_t>(c->num_sms, ap.total_iters),
+                             ceil_div(ap.total_iters, tpc));
+    grid = std::min<int64_t>(grid, c->lay.rb_cap);
+  }
+  ap.grid = static_cast<int32_t>(grid);
+  ap.scale_log2 = c->scale_log2;
+  e = launch_attention(ap, cf.head_dim, s);
+  if (e != cudaSuccess) return cuda_fail(c, e, "attention launch");
+  ++c->launches;
+  if (ap.grid > 1) {
+    MergeParams mp{};
+    mp.part_o = ap.part_o;
+    mp.part_lse = ap.part_lse;
+    mp.out = ap.out;
+    mp.lse = lse;
+    mp.L = L;
+    mp.total_iters = ap.total_iters;
+    mp.iters_per_head = iph;
+    mp.n = n;
+    mp.hq = ap.hq;
+    mp.hkv = ap.hkv;
+    mp.group = ap.group;
+    mp.n_tiles = ap.n_tiles;
+    mp.grid = ap.grid;
+    mp.d = cf.head_dim;
+    e = launch_merge(mp, s);
+    if (e != cudaSuccess) return cuda_fail(c, e, "merge launch");
+    ++c->launches;
+  }
+  return CSR_OK;
+}
+
+enum class Kind { Prefix, Chunk, Suffix };
+
+csr_status add_block(csr_ctx *c, Kind kind, const void *q, const void *k, const void *v,
+                     int32_t n, void *out, float *lse, cudaStream_t s, int64_t *chunk_id) {
+  if (n < 1 || n > c->cfg.max_new_tokens)
+    return fail(c, CSR_EINVAL, "n must be in [1, max_new_tokens]");
+  if (!c->plan_only && (!q || !k || !v || !out))
+    return fail(c, CSR_EINVAL, "q, k, v and out must be device pointers");
+  if (!c->plan_only) {
+    for (const void *ptr : {q, k, v, static_cast<const void *>(out)})
+      if (reinterpret_cast<uintptr_t>(ptr) % 16)
+        return fail(c, CSR_EINVAL, "tensor pointers must be 16-byte aligned");
+  }
+  Version &A = c->act();
+  const int64_t L = A.length();
+  const int64_t new_len = L + n;
+  if (new_len > c->cfg.max_seq_tokens) return fail(c, CSR_ENOMEM, "max_seq_tokens exceeded");
+  const int64_t needA = pages_for(c, new_len) - static_cast<int64_t>(A.pages.size());
+  const bool fork = kind == Kind::Chunk && c->reconciling;
+  int64_t needB = 0;
+  if (fork) {
+    Version &B = c->pend();
+    if (B.length() + n > c->cfg.max_seq_tokens)
+      return fail(c, CSR_ENOMEM, "max_seq_tokens exceeded in the rebuilt version");
+    needB = pages_for(c, B.length() + n) - static_cast<int64_t>(B.pages.size());
+  }
+  if (needA + needB > c->pool.n_free) return fail(c, CSR_ENOMEM, "page pool exhausted");
+  for (int64_t i = 0; i < needA; ++i) A.pages.push_back(c->pool.take());
+  const int32_t first_lp = static_cast<int32_t>(L / c->cfg.page_size);
+  const int32_t n_ids = static_cast<int32_t>(pages_for(c, new_len)) - first_lp;
+  int64_t id = -1;
+  if (kind == Kind::Chunk) id = c->next_chunk_id++;
+  if (!c->plan_only) {
+    const int slot = c->active.load();
+    csr_status st = run_block(c, slot, 0, q, k, v, n, L, A.pages.data() + first_lp, n_ids,
+                              first_lp, out, lse, s);
+    if (st != CSR_OK) return st;
+  }
+  switch (kind) {
+    case Kind::Prefix: A.prefix_len = n; break;
+    case Kind::Chunk: A.chunks.push_back({id, n}); break;
+    case Kind::Suffix: A.suffix_len = n; break;
+  }
+  if (fork) {
+    // Algorithm 1, Increment: fork the chunk into the buffer of the rebuild;
+    // its pages in the rebuilt version are reserved now (after the active ones).
+    Version &B = c->pend();
+    for (int64_t i = 0; i < needB; ++i) B.pages.push_back(c->pool.take());
+    B.chunks.push_back({id, n});
+    c->buffer.push_back({id, n});
+  }
+  if (chunk_id) *chunk_id = id;
+  return CSR_OK;
+}
+
+// Release every page reference of a version and forget it.
+void drop_version(csr_ctx *c, Version &V) {
+  for (int32_t p : V.pages) c->pool.release(p);
+  V.clear();
+}
+
+// Abort a reconciliation: wait for its device work, give its pages back.
+void abort_reconcile(csr_ctx *c) {
+  if (!c->plan_only && c->lo) cudaStreamSynchronize(c->lo);
+  drop_version(c, c->pend());
+  c->reconciling = false;
+  c->buffer.clear();
+  c->reserved_ids.clear();
+}
+
+// Recompute `chunks` of the pending version on stream s, starting at position
+// c->rebuilt_len (the catch-up of Algorithm 1, or the remainder at the swap).
+csr_status materialise(csr_ctx *c, const std::vector<ChunkRec> &chunks, int ws, cudaStream_t s) {
+  const int slot = 1 - c->active.load();
+  Version &B = c->pend();
+  for (const ChunkRec &ch : chunks) {
+    const void *q = nullptr, *k = nullptr, *v = nullptr;
+    void *out = nullptr;
+    if (c->provider(c->user, ch.id, ch.len, &q, &k, &v, &out) != 0 || !q || !k || !v)
+      return fail(c, CSR_ESTATE, "qkv provider failed for chunk " + std::to_string(ch.id));
+    const int64_t L = c->rebuilt_len;
+    const int32_t first_lp = static_cast<int32_t>(L / c->cfg.page_size);
+    const int32_t n_ids = static_cast<int32_t>(pages_for(c, L + ch.len)) - first_lp;
+    csr_status st = run_block(c, slot, ws, q, k, v, ch.len, L, B.pages.data() + first_lp, n_ids,
+                              first_lp, out ? out : c->wsp<void>(c->lay.rb_out), nullptr, s);
+    if (st != CSR_OK) return st;
+    c->rebuilt_len += ch.len;
+  }
+  return CSR_OK;
+}
+
+}  // namespace
+
+// ============================================================== C ABI
+extern "C" {
+
+size_t csr_pool_bytes(const csr_config *cfg) {
+  if (!valid_config(cfg, nullptr)) return 0;
+  return static_cast<size_t>(cfg->pool_pages) * cfg->num_kv_heads * cfg->page_size *
+         cfg->head_dim * 2;
+}
+
+size_t csr_workspace_bytes(const csr_config *cfg) {
+  if (!valid_config(cfg, nullptr)) return 0;
+  return make_layout(cfg).total;
+}
+
+csr_status csr_create(const csr_config *cfg, void *k_pool, void *v_pool, void *workspace,
+                      csr_stream_t stream, csr_ctx **out) {
+  static thread_local std::string create_err;
+  if (!out) return CSR_EINVAL;
+  *out = nullptr;
+  std::string why;
+  if (!valid_config(cfg, &why)) return CSR_EINVAL;
+  csr_ctx *c = new csr_ctx();
+  c->cfg = *cfg;
+  c->plan_only = (cfg->flags & CSR_FLAG_PLAN_ONLY) != 0;
+  c->group = cfg->num_q_heads / cfg->num_kv_heads;
+  c->lay = make_layout(cfg);
+  const double scale = cfg->softmax_scale > 0.f ? static_cast<double>(cfg->softmax_scale)
+                                                : 1.0 / std::sqrt(static_cast<double>(cfg->head_dim));
+  c->scale_log2 = static_cast<float>(scale * 1.4426950408889634);  // log2(e)
+  const double two_pi = 6.283185307179586476925286766559;
+  for (int i = 0; i < cfg->head_dim / 2; ++i)
+    c->inv_turns[i] = std::pow(cfg->rope_base, -2.0 * i / cfg->head_dim) / two_pi;
+  c->pool.init(cfg->pool_pages);
+  if (!c->plan_only) {
+    const uintptr_t a = reinterpret_cast<uintptr_t>(k_pool) | reinterpret_cast<uintptr_t>(v_pool) |
+                        reinterpret_cast<uintptr_t>(workspace);
+    if (!k_pool || !v_pool || !workspace || (a % kAlign)) {
+      delete c;
+      return CSR_EINVAL;
+    }
+    c->k_pool = static_cast<uint16_t *>(k_pool);
+    c->v_pool = static_cast<uint16_t *>(v_pool);
+    c->ws = static_cast<uint8_t *>(workspace);
+    cudaError_t e = cudaGetDevice(&c->device);
+    if (e == cudaSuccess)
+      e = cudaDeviceGetAttribute(&c->num_sms, cudaDevAttrMultiProcessorCount, c->device);
+    if (e == cudaSuccess) e = attn_configure(cfg->head_dim);
+    if (e != cudaSuccess) {
+      delete c;
+      return CSR_ECUDA;
+    }
+    c->fg_grid = cfg->num_ctas > 0 ? cfg->num_ctas : std::min(c->num_sms, c->lay.fg_cap);
+    const uint64_t pool_rows = static_cast<uint64_t>(cfg->pool_pages) * cfg->num_kv_heads * cfg->page_size;
+    bool ok = encode_rows(&c->tm_k, k_pool, pool_rows, cfg->head_dim, cfg->page_size) &&
+              encode_rows(&c->tm_v, v_pool, pool_rows, cfg->head_dim, cfg->page_size);
+    for (int i = 0; i < 2 && ok; ++i)
+      ok = encode_rows(&c->tm_q[i], c->ws + c->lay.qpack[i],
+                       static_cast<uint64_t>(cfg->num_kv_heads) * c->lay.rows_cap, cfg->head_dim, kBM);
+    if (!ok) {
+      delete c;
+      return CSR_ECUDA;
+    }
+    const cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    const size_t pool_bytes = csr_pool_bytes(cfg);
+    e = cudaMemsetAsync(k_pool, 0, pool_bytes, s);
+    if (e == cudaSuccess) e = cudaMemsetAsync(v_pool, 0, pool_bytes, s);
+    if (e == cudaSuccess) e = cudaMemsetAsync(workspace, 0, c->lay.total, s);
+    if (e == cudaSuccess) e = cudaEventCreateWithFlags(&c->ev_fg, cudaEventDisableTiming);
+    if (e == cudaSuccess) e = cudaEventCreateWithFlags(&c->ev_rb, cudaEventDisableTiming);
+    if (e != cudaSuccess) {
+      if (c->ev_fg) cudaEventDestroy(c->ev_fg);
+      if (c->ev_rb) cudaEventDestroy(c->ev_rb);
+      delete c;
+      return CSR_ECUDA;
+    }
+  }
+  *out = c;
+  return CSR_OK;
+}
+
+void csr_destroy(csr_ctx *c) {
+  if (!c) return;
+  if (!c->plan_only) {
+    if (c->lo) cudaStreamSynchronize(c->lo);
+    cudaDeviceSynchronize();
+    if (c->ev_fg) cudaEventDestroy(c->ev_fg);
+    if (c->ev_rb) cudaEventDestroy(c->ev_rb);
+  }
+  delete c;
+}
+
+csr_status csr_init_static(csr_ctx *c, const void *q, const void *k, const void *v, int32_t n,
+                           void *out, float *lse, csr_stream_t stream) {
+  if (!c) return CSR_EINVAL;
+  if (c->has_static) return fail(c, CSR_ESTATE, "static prefix already initialised");
+  csr_status st = add_block(c, Kind::Prefix, q, k, v, n, out, lse,
+                            reinterpret_cast<cudaStream_t>(stream), nullptr);
+  if (st == CSR_OK) c->has_static = true;
+  return st;
+}
+
+csr_status csr_append_chunk(csr_ctx *c, const void *q, const void *k, const void *v, int32_t n,
+                            void *out, float *lse, csr_stream_t stream, int64_t *chunk_id) {
+  if (!c) return CSR_EINVAL;
+  if (!c->has_static) return fail(c, CSR_ESTATE, "csr_init_static must come first");
+  if (c->act().suffix_len > 0) return fail(c, CSR_ESTATE, "a suffix is live: truncate it first");
+  csr_status st = add_block(c, Kind::Chunk, q, k, v, n, out, lse,
+                            reinterpret_cast<cudaStream_t>(stream), chunk_id);
+  if (st != CSR_OK) return st;
+  // Algorithm 1, Increment: trigger the eviction at tau_mem.
+  if (c->provider && c->cfg.cap_tokens > 0 && !c->reconciling &&
+      c->act().length() >= c->cfg.cap_tokens)
+    return csr_evict_and_reconcile(c, c->cfg.evict_tokens, stream);
+  return CSR_OK;
+}
+
+csr_status csr_attend_suffix(csr_ctx *c, const void *q, const void *k, const void *v, int32_t n,
+                             void *out, float *lse, csr_stream_t stream) {
+  if (!c) return CSR_EINVAL;
+  if (!c->has_static) return fail(c, CSR_ESTATE, "csr_init_static must come first");
+  if (c->act().suffix_len > 0) return fail(c, CSR_ESTATE, "a suffix is already live");
+  return add_block(c, Kind::Suffix, q, k, v, n, out, lse, reinterpret_cast<cudaStream_t>(stream),
+                   nullptr);
+}
+
+csr_status csr_truncate_suffix(csr_ctx *c) {
+  if (!c) return CSR_EINVAL;
+  Version &A = c->act();
+  if (A.suffix_len == 0) return fail(c, CSR_ESTATE, "no live suffix");
+  A.suffix_len = 0;
+  const int64_t keep = pages_for(c, A.length());
+  while (static_cast<int64_t>(A.pages.size()) > keep) {
+    c->pool.release(A.pages.back());
+    A.pages.pop_back();
+  }
+  return CSR_OK;
+}
+
+csr_status csr_set_reconciler(csr_ctx *c, csr_qkv_provider provider, void *user,
+                              csr_stream_t lo_stream) {
+  if (!c) return CSR_EINVAL;
+  if (c->reconciling) return fail(c, CSR_EBUSY, "a reconciliation is running");
+  c->provider = provider;
+  c->user = user;
+  c->lo = reinterpret_cast<cudaStream_t>(lo_stream);
+  return CSR_OK;
+}
+
+csr_status csr_evict_and_reconcile(csr_ctx *c, int32_t evict_tokens, csr_stream_t fg_stream) {
+  if (!c) return CSR_EINVAL;
+  if (c->reconciling) return fail(c, CSR_EBUSY, "a reconciliation is already running");
+  if (!c->provider) return fail(c, CSR_ESTATE, "no reconciler registered");
+  if (evict_tokens < 1) return fail(c, CSR_EINVAL, "evict_tokens must be >= 1");
+  Version &A = c->act();
+  if (A.suffix_len > 0) return fail(c, CSR_ESTATE, "a suffix is live");
+  if (A.chunks.empty()) return fail(c, CSR_ESTATE, "no chunk to evict");
+  // Eq. eviction_operation: drop the oldest whole chunks until >= evict_tokens are gone.
+  size_t k = 0;
+  int64_t dropped = 0;
+  while (k < A.chunks.size() && dropped < evict_tokens) dropped += A.chunks[k++].len;
+  std::vector<ChunkRec> retained(A.chunks.begin() + k, A.chunks.end());
+  int64_t new_len = A.prefix_len;
+  for (const auto &ch : retained) new_len += ch.len;
+  const int P = c->cfg.page_size;
+  const int32_t full = static_cast<int32_t>(A.prefix_len / P);
+  const int32_t tail = static_cast<int32_t>(A.prefix_len % P);
+  const int64_t fresh = pages_for(c, new_len) - full;
+  if (new_len > c->cfg.max_seq_tokens) return fail(c, CSR_ENOMEM, "max_seq_tokens exceeded");
+  if (fresh > c->pool.n_free) return fail(c, CSR_ENOMEM, "page pool cannot hold the rebuilt version");
+  EvictParams *ep = nullptr;
+  if (!c->plan_only) {
+    ep = new EvictParams();
+    ep->n_words = static_cast<int32_t>(c->pool.free_bits.size());
+    std::memcpy(ep->free_words, c->pool.free_bits.data(), c->pool.free_bits.size() * 4);
+  }
+  // Reserve the rebuilt version: shared full prefix pages, then the smallest free ids.
+  const int act_slot = c->active.load();
+  Version &B = c->ver[1 - act_slot];
+  B.clear();
+  B.prefix_len = A.prefix_len;
+  for (int32_t i = 0; i < full; ++i) {
+    c->pool.share(A.pages[i]);
+    B.pages.push_back(A.pages[i]);
+  }
+  c->reserved_ids.clear();
+  for (int64_t i = 0; i < fresh; ++i) {
+    const int32_t id = c->pool.take();
+    B.pages.push_back(id);
+    c->reserved_ids.push_back(id);
+  }
+  B.chunks = retained;
+  c->reconciling = true;
+  c->buffer.clear();
+  c->ids_checked = c->plan_only;
+  c->rebuilt_len = A.prefix_len;
+  if (c->plan_only) {
+    for (const auto &ch : retained) c->rebuilt_len += ch.len;
+    return CSR_OK;
+  }
+  const cudaStream_t fg = reinterpret_cast<cudaStream_t>(fg_stream);
+  cudaError_t e = cudaEventRecord(c->ev_fg, fg);
+  if (e == cudaSuccess) e = cudaStreamWaitEvent(c->lo, c->ev_fg, 0);
+  if (e != cudaSuccess) {
+    delete ep;
+    abort_reconcile(c);
+    return cuda_fail(c, e, "ordering the rebuild after the foreground");
+  }
+  ep->old_pt = c->d_pt(act_slot);
+  ep->new_pt = c->d_pt(1 - act_slot);
+  ep->ids_out = c->wsp<int32_t>(c->lay.ids_out);
+  ep->k_pool = c->k_pool;
+  ep->v_pool = c->v_pool;
+  ep->err = c->wsp<uint32_t>(c->lay.err);
+  ep->full_prefix_pages = full;
+  ep->prefix_tail = tail;
+  ep->n_new = static_cast<int32_t>(fresh);
+  ep->hkv = c->cfg.num_kv_heads;
+  ep->page_size = P;
+  ep->d = c->cfg.head_dim;
+  ep->pool_pages = c->cfg.pool_pages;
+  e = launch_evict(*ep, c->lo);
+  delete ep;
+  if (e != cudaSuccess) {
+    abort_reconcile(c);
+    return cuda_fail(c, e, "evict_compact launch");
+  }
+  ++c->launches;
+  // Warm-up (LLM(X_eps) on the secondary resource): a fresh causal prefill of
+  // every retained chunk at its renumbered position, reading the page table
+  // the compaction kernel wrote.
+  const int slot = 1 - act_slot;
+  for (const ChunkRec &ch : retained) {
+    const void *q = nullptr, *k2 = nullptr, *v = nullptr;
+    void *out = nullptr;
+    if (c->provider(c->user, ch.id, ch.len, &q, &k2, &v, &out) != 0 || !q || !k2 || !v) {
+      abort_reconcile(c);
+      return fail(c, CSR_ESTATE, "qkv provider failed for chunk " + std::to_string(ch.id));
+    }
+    csr_status st = run_block(c, slot, 1, q, k2, v, ch.len, c->rebuilt_len, nullptr, 0, 0,
+                              out ? out : c->wsp<void>(c->lay.rb_out), nullptr, c->lo);
+    if (st != CSR_OK) {
+      abort_reconcile(c);
+      return st;
+    }
+    c->rebuilt_len += ch.len;
+  }
+  e = cudaEventRecord(c->ev_rb, c->lo);
+  if (e != cudaSuccess) {
+    abort_reconcile(c);
+    return cuda_fail(c, e, "recording the rebuild event");
+  }
+  return CSR_OK;
+}
+
+csr_status csr_poll_swap(csr_ctx *c, csr_stream_t fg_stream, int *state) {
+  if (!c || !state) return CSR_EINVAL;
+  if (!c->reconciling) {
+    *state = CSR_RECON_IDLE;
+    return CSR_OK;
+  }
+  *state = CSR_RECON_RUNNING;
+  if (!c->plan_only) {
+    const cudaError_t q = cudaEventQuery(c->ev_rb);
+    if (q == cudaErrorNotReady) return CSR_OK;
+    if (q != cudaSuccess) return cuda_fail(c, q, "rebuild event");
+    if (!c->ids_checked) {
+      // The compaction kernel's page choice must equal the host's reservation.
+      const size_t cnt = c->reserved_ids.size();
+      std::vector<int32_t> got(cnt);
+      cudaError_t e = cnt ? cudaMemcpyAsync(got.data(), c->wsp<int32_t>(c->lay.ids_out), cnt * 4,
+                                            cudaMemcpyDeviceToHost, c->lo)
+                          : cudaSuccess;
+      if (e == cudaSuccess) e = cudaStreamSynchronize(c->lo);
+      if (e != cudaSuccess) return cuda_fail(c, e, "reading the compaction result");
+      if (got != c->reserved_ids) {
+        abort_reconcile(c);
+        return fail(c, CSR_EDEVICE, "compaction kernel page ids differ from the host allocator");
+      }
+      c->ids_checked = true;
+    }
+  }
+  // Algorithm 1: while |buffer| > N_catchup, catch up on the secondary resource.
+  if (static_cast<int64_t>(c->buffer.size()) > c->cfg.n_catchup) {
+    std::vector<ChunkRec> batch;
+    batch.swap(c->buffer);
+    if (!c->plan_only) {
+      csr_status st = materialise(c, batch, 1, c->lo);
+      if (st != CSR_OK) {
+        abort_reconcile(c);
+        return st;
+      }
+      const cudaError_t e = cudaEventRecord(c->ev_rb, c->lo);
+      if (e != cudaSuccess) return cuda_fail(c, e, "recording the catch-up event");
+    } else {
+      for (const auto &ch : batch) c->rebuilt_len += ch.len;
+    }
+    return CSR_OK;
+  }
+  if (c->act().suffix_len > 0) return CSR_OK;  // swap only between tasks
+  // The remainder (<= N_catchup chunks) is computed now, on the foreground.
+  if (!c->buffer.empty()) {
+    std::vector<ChunkRec> rest;
+    rest.swap(c->buffer);
+    if (!c->plan_only) {
+      csr_status st = materialise(c, rest, 0, reinterpret_cast<cudaStream_t>(fg_stream));
+      if (st != CSR_OK) {
+        abort_reconcile(c);
+        return st;
+      }
+    } else {
+      for (const auto &ch : rest) c->rebuilt_len += ch.len;
+    }
+  }
+  // Atomic swap of the active version (App. D step 5); the old version's own
+  // pages return to the pool (the shared prefix pages stay referenced).
+  const int old = c->active.load();
+  c->active.store(1 - old);
+  drop_version(c, c->ver[old]);
+  c->reconciling = false;
+  c->reserved_ids.clear();
+  *state = CSR_RECON_SWAPPED;
+  return CSR_OK;
+}
+
+csr_status csr_wait_reconcile(csr_ctx *c, csr_stream_t fg_stream, int64_t timeout_us, int *state) {
+  if (!c || !state) return CSR_EINVAL;
+  const auto t0 = std::chrono::steady_clock::now();
+  while (true) {
+    csr_status st = csr_poll_swap(c, fg_stream, state);
+    if (st != CSR_OK || *state != CSR_RECON_RUNNING) return st;
+    if (c->act().suffix_len > 0 && c->buffer.empty())
+      return fail(c, CSR_ESTATE, "swap waits for the live suffix to be truncated");
+    const auto us = std::chrono::duration_cast<std::chrono::microseconds>(
+                        std::chrono::steady_clock::now() - t0)
+                        .count();
+    if (us > timeout_us) return fail(c, CSR_ETIMEOUT, "reconciliation still running");
+    std::this_thread::sleep_for(std::chrono::microseconds(50));
+  }
+}
+
+csr_status csr_get_layout(csr_ctx *c, int which, int32_t *page_table, int32_t capacity,
+                          int32_t *n_pages, int64_t *length) {
+  if (!c) return CSR_EINVAL;
+  if (which != CSR_VERSION_ACTIVE && which != CSR_VERSION_PENDING)
+    return fail(c, CSR_EINVAL, "which must be ACTIVE or PENDING");
+  if (which == CSR_VERSION_PENDING && !c->reconciling)
+    return fail(c, CSR_ESTATE, "no reconciliation running");
+  const Version &V = which == CSR_VERSION_ACTIVE ? c->act() : c->pend();
+  const int32_t np = static_cast<int32_t>(V.pages.size());
+  if (n_pages) *n_pages = np;
+  if (length) *length = V.length();
+  if (page_table) {
+    if (capacity < np) return fail(c, CSR_EINVAL, "page_table capacity too small");
+    std::copy(V.pages.begin(), V.pages.end(), page_table);
+  }
+  return CSR_OK;
+}
+
+csr_status csr_get_free_pages(csr_ctx *c, int32_t *ids, int32_t capacity, int32_t *count) {
+  if (!c) return CSR_EINVAL;
+  if (count) *count = c->pool.n_free;
+  if (ids) {
+    if (capacity < c->pool.n_free) return fail(c, CSR_EINVAL, "capacity too small");
+    int32_t k = 0;
+    for (int32_t i = 0; i < c->pool.n; ++i)
+      if (c->pool.free_bits[i >> 5] & (1u << (i & 31))) ids[k++] = i;
+  }
+  return CSR_OK;
+}
+
+csr_status csr_get_chunks(csr_ctx *c, int which, int64_t *ids, int32_t *lens, int32_t capacity,
+                          int32_t *count, int64_t *prefix_len) {
+  if (!c) return CSR_EINVAL;
+  if (which != CSR_VERSION_ACTIVE && which != CSR_VERSION_PENDING)
+    return fail(c, CSR_EINVAL, "which must be ACTIVE or PENDING");
+  if (which == CSR_VERSION_PENDING && !c->reconciling)
+    return fail(c, CSR_ESTATE, "no reconciliation running");
+  const Version &V = which == CSR_VERSION_ACTIVE ? c->act() : c->pend();
+  const int32_t n = static_cast<int32_t>(V.chunks.size());
+  if (count) *count = n;
+  if (prefix_len) *prefix_len = V.prefix_len;
+  if (ids || lens) {
+    if (capacity < n) return fail(c, CSR_EINVAL, "capacity too small");
+    for (int32_t i = 0; i < n; ++i) {
+      if (ids) ids[i] = V.chunks[i].id;
+      if (lens) lens[i] = V.chunks[i].len;
+    }
+  }
+  return CSR_OK;
+}
+
+csr_status csr_device_page_table(csr_ctx *c, int which, const int32_t **ptr) {
+  if (!c || !ptr) return CSR_EINVAL;
+  if (c->plan_only) return fail(c, CSR_ESTATE, "plan-only context has no device memory");
+  if (which == CSR_VERSION_PENDING && !c->reconciling)
+    return fail(c, CSR_ESTATE, "no reconciliation running");
+  const int slot = which == CSR_VERSION_ACTIVE ? c->active.load() : 1 - c->active.load();
+  *ptr = c->d_pt(slot);
+  return CSR_OK;
+}
+
+csr_status csr_gather_kv(csr_ctx *c, int which, int64_t pos0, int32_t n, void *k_out,
+                         void *v_out, csr_stream_t stream) {
+  if (!c) return CSR_EINVAL;
+  if (c->plan_only) return fail(c, CSR_ESTATE, "plan-only context has no device memory");
+  if (which != CSR_VERSION_ACTIVE && which != CSR_VERSION_PENDING)
+    return fail(c, CSR_EINVAL, "which must be ACTIVE or PENDING");
+  if (which == CSR_VERSION_PENDING && !c->reconciling)
+    return fail(c, CSR_ESTATE, "no reconciliation running");
+  const Version &V = which == CSR_VERSION_ACTIVE ? c->act() : c->pend();
+  if (n < 1 || pos0 < 0 || pos0 + n > V.length() || !k_out || !v_out)
+    return fail(c, CSR_EINVAL, "position range outside the version, or NULL output");
+  GatherParams gp{};
+  gp.k_pool = c->k_pool;
+  gp.v_pool = c->v_pool;
+  gp.page_table = c->d_pt(which == CSR_VERSION_ACTIVE ? c->active.load() : 1 - c->active.load());
+  gp.k_out = static_cast<uint16_t *>(k_out);
+  gp.v_out = static_cast<uint16_t *>(v_out);
+  gp.err = c->wsp<uint32_t>(c->lay.err);
+  gp.pos0 = pos0;
+  gp.n = n;
+  gp.hkv = c->cfg.num_kv_heads;
+  gp.d = c->cfg.head_dim;
+  gp.page_size = c->cfg.page_size;
+  gp.pool_pages = c->cfg.pool_pages;
+  const cudaError_t e = launch_gather(gp, reinterpret_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(c, e, "gather launch");
+  ++c->launches;
+  return CSR_OK;
+}
+
+csr_status csr_device_status(csr_ctx *c, uint32_t *flags) {
+  if (!c) return CSR_EINVAL;
+  if (flags) *flags = 0;
+  if (c->plan_only) return CSR_OK;
+  cudaError_t e = cudaDeviceSynchronize();
+  if (e != cudaSuccess) return cuda_fail(c, e, "device synchronise");
+  uint32_t word = 0;
+  e = cudaMemcpy(&word, c->wsp<uint32_t>(c->lay.err), 4, cudaMemcpyDeviceToHost);
+  if (e == cudaSuccess) e = cudaMemset(c->wsp<uint32_t>(c->lay.err), 0, 4);
+  if (e != cudaSuccess) return cuda_fail(c, e, "reading the error word");
+  if (flags) *flags = word;
+  if (word) return fail(c, CSR_EDEVICE, "a kernel reported device error bits");
+  return CSR_OK;
+}
+
+int64_t csr_kernel_launches(const csr_ctx *c) { return c ? c->launches : 0; }
+
+const char *csr_last_error(const csr_ctx *c) { return c ? c->err.c_str() : "NULL context"; }
+
+}  // extern "C"

@@ -48,8 +48,14 @@ class Block:
 
 def block(seed: int, n: int, hq: int, hkv: int, d: int, kind: str = "normal") -> Block:
     """Draw one block.  ``kind``: "normal" (N(0,1)), "ones_v" (V = 1),
-    "zero_k" (K = 0), "const_q" (every query row equal)."""
+    "zero_k" (K = 0), "const_q" (every query row equal), "kv_only" (K then V
+    are drawn from the seed and Q is all zero: fill-phase chunks of long
+    caches whose outputs are not compared)."""
     rng = np.random.default_rng(seed)
+    if kind == "kv_only":
+        k = rng.standard_normal((n, hkv, d), dtype=np.float32)
+        v = rng.standard_normal((n, hkv, d), dtype=np.float32)
+        return Block(np.zeros((n, hq, d), np.uint16), bf16_bits(k), bf16_bits(v))
     q = rng.standard_normal((n, hq, d), dtype=np.float32)
     k = rng.standard_normal((n, hkv, d), dtype=np.float32)
     v = rng.standard_normal((n, hkv, d), dtype=np.float32)

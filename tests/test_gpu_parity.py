@@ -1,0 +1,137 @@
+"""GPU path (through the C-ABI) against the fp64 oracle, element by element.
+
+Covers the tiny correctness configuration in full, the 64/4/128 head shape
+with ragged sizes, split-KV partial merging under forced CTA counts, edge
+cases (one token, n = max_new_tokens, special inputs) and run-to-run bitwise
+determinism.
+"""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+from gpu_util import C1, C2, Pair, assert_close, bits_of, to_f64
+
+pytestmark = pytest.mark.gpu
+
+
+def test_tiny_config_full_session(libcsr):
+    """8 q heads / 2 kv heads, d=64, page 16, base 1e4: 256-token prefix,
+    3 chunks of 256, a 32-token suffix, truncate, one more chunk, suffix again."""
+    p = Pair(C1, pool_pages=256, max_seq=4096, max_new=512)
+    p.init_static(p.blk(0, 256))
+    for i in range(3):
+        p.append(p.blk(1 + i, 256))
+    p.check_layout()
+    p.suffix(p.blk(1_000_000, 32))
+    p.check_layout()
+    p.truncate()
+    p.check_layout()
+    p.append(p.blk(4, 256))
+    p.suffix(p.blk(1_000_001, 32))
+    p.check_layout()
+    p.check_cache()
+    p.truncate()
+    p.check_layout()
+    p.device_clean()
+
+
+def test_single_token_prefix_returns_v(libcsr):
+    """L=0, n=1: the only visible key is the token itself, so out = V exactly."""
+    p = Pair(C2, pool_pages=16, max_seq=1024, max_new=256)
+    b = p.blk(5, 1)
+    out, lse = p.init_static(b)
+    v = b.f64()[2]                                    # [1][hkv][d]
+    expect = np.repeat(v, p.hq // p.hkv, axis=1)
+    assert np.array_equal(to_f64(out), expect)
+    p.device_clean()
+
+
+@pytest.mark.parametrize("shape", [C1, C2], ids=["d64_p16_g4", "d128_p64_g16"])
+def test_ragged_sizes(libcsr, shape):
+    p = Pair(shape, pool_pages=128, max_seq=4096, max_new=512)
+    p.init_static(p.blk(10, 37))
+    for i, n in enumerate([1, 129, 64, 300, 17]):
+        p.append(p.blk(11 + i, n))
+    p.suffix(p.blk(20, 7))
+    p.check_layout()
+    p.truncate()
+    p.append(p.blk(21, 5))
+    p.suffix(p.blk(22, 250))
+    p.check_layout()
+    p.check_cache()
+    p.device_clean()
+
+
+@pytest.mark.parametrize("num_ctas", [1, 2, 3, 7, 19, 64])
+def test_split_kv_partials_any_grid(libcsr, num_ctas):
+    """Forced CTA counts cut units at arbitrary key tiles: every split must
+    merge back to the oracle."""
+    p = Pair(C2, pool_pages=256, max_seq=8192, max_new=1024, num_ctas=num_ctas)
+    p.init_static(p.blk(30, 700))
+    p.append(p.blk(31, 1000))
+    p.append(p.blk(32, 33))
+    p.suffix(p.blk(33, 200))
+    p.truncate()
+    p.device_clean()
+
+
+def test_max_new_tokens_call(libcsr):
+    p = Pair(C2, pool_pages=128, max_seq=8192, max_new=1024)
+    p.init_static(p.blk(40, 1024))
+    p.append(p.blk(41, 1024))
+    p.check_layout()
+    p.device_clean()
+
+
+def test_special_inputs(libcsr):
+    """V = 1 gives outputs of 1 (the weights sum to one); K = 0 gives the
+    causal mean of V (within the bf16 rounding of the weights)."""
+    p = Pair(C2, pool_pages=64, max_seq=4096, max_new=512)
+    out, _ = p.init_static(p.blk(50, 300, "ones_v"))
+    got = to_f64(out)
+    assert np.max(np.abs(got - 1.0)) <= 2e-2
+    p2 = Pair(C1, pool_pages=64, max_seq=4096, max_new=512)
+    p2.init_static(p2.blk(51, 200, "zero_k"))
+    p2.append(p2.blk(52, 100, "zero_k"))
+    p.device_clean()
+    p2.device_clean()
+
+
+def test_bitwise_deterministic(libcsr):
+    outs = []
+    for _ in range(2):
+        p = Pair(C2, pool_pages=128, max_seq=8192, max_new=1024)
+        p.init_static(p.blk(60, 500), compare=False)
+        o1, _, _ = p.append(p.blk(61, 700), compare=False)
+        o2, _ = p.suffix(p.blk(62, 100), compare=False)
+        torch.cuda.synchronize()
+        outs.append((bits_of(o1), bits_of(o2)))
+    assert np.array_equal(outs[0][0], outs[1][0]) and np.array_equal(outs[0][1], outs[1][1])
+
+
+def test_8k_context_step(libcsr):
+    """64 q heads / 4 kv heads, d=128, page 64, base 1e6: 2048-token prefix plus
+    48 chunks of 128 (8192 cached); a step appends a 128-token chunk, attends a
+    64-token suffix over the whole cache, then truncates."""
+    p = Pair(C2, pool_pages=512, max_seq=16384, max_new=2048)
+    p.init_static(p.blk(100, 2048), compare=False)
+    for i in range(48):
+        p.append(p.blk(101 + i, 128, "kv_only"), compare=False)
+    assert p.orc.length() == 8192
+    for step in range(2):
+        p.append(p.blk(200 + step, 128))
+        p.suffix(p.blk(1_000_000 + step, 64))
+        p.check_layout()
+        p.truncate()
+    p.check_layout()
+    p.check_cache(positions=np.arange(0, p.orc.length(), 7))
+    p.device_clean()
+
+
+def test_launch_count_reported(libcsr):
+    p = Pair(C1, pool_pages=64, max_seq=2048, max_new=256)
+    before = p.ctx.kernel_launches()
+    p.init_static(p.blk(70, 100))
+    assert p.ctx.kernel_launches() - before >= 2   # K1 + K2 (+ K3)
