@@ -1,0 +1,403 @@
+#!/usr/bin/env python
+"""Benchmark: incremental-prefill attention at 120K cached tokens, one layer.
+
+Workload (the 120K-context step): 64 query heads, 4 KV heads, head_dim 128,
+bf16, RoPE base 1e6, page size 64.  The cache holds a 4,096-token static
+prefix plus 256-token chunks; the first timed step starts at 122,880 cached
+tokens.  A step appends a 256-token state chunk, attends a 512-token task
+suffix over the whole cache and truncates the suffix (section III-D), through
+the C-ABI library.  Inputs are seeded synthetic N(0,1) bf16 tensors already
+resident in HBM; the KV cache (about 252 MB) is larger than the 129 MB L2, so
+no flush is needed between steps.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+Prints one JSON line (rank 0).  `value` is the device-timed microseconds per
+layer-step (lower is better), `e2e` the same through the public API with the
+step's inputs copied from pinned host memory and its outputs copied back
+inside the timed region.  `roofline` is the attention kernel's achieved
+TFLOP/s (algorithmic FLOPs / its CUDA-event time) against the measured bf16
+peak; `cpu_baseline` times the fp64 CPU oracle on a bounded sample of the
+same step.  With N > 1 (torchrun) every rank runs an independent replica
+(the path does not shard: one layer's cache lives on one GPU); the slowest
+rank's time is reported.  `--impl reference` times the fp64 oracle alone.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "µs/layer and % roofline, incremental-prefill attention at 120K cached tokens"
+UNIT = "us/layer"
+HQ, HKV, D, P, BASE = 64, 4, 128, 64, 1e6
+PREFIX, CHUNK, SUFFIX, L0 = 4096, 256, 512, 122880
+LAYERS_PROXY = 94
+WORKLOAD_NAME = ("120K-context step: append 256-token chunk + attend 512-token suffix + truncate, "
+                 "122,880 cached tokens, 64 q / 4 kv heads, head_dim 128, page 64, bf16, 1 layer")
+TRAFFIC_FILE = os.path.join(ROOT, "profiles", "attention_120k_traffic.txt")
+ATTN_SRC = os.path.join(ROOT, "paper_2605_07325_gb300", "csrc", "kernels_attn.cu")
+
+
+def _peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            m = json.load(f)
+        return float(m["hbm_gbs"]), float(m["bf16_tflops"]), float(m["bf16_tflops_sustained"]), "measured"
+    except (OSError, KeyError, ValueError):
+        return 6800.0, 1900.0, 1700.0, "fallback"
+
+
+def _attention_source_hash() -> str:
+    with open(ATTN_SRC, "rb") as f:
+        return hashlib.sha256(f.read()).hexdigest()[:16]
+
+
+def _traffic_per_launch_step():
+    """DRAM bytes per step of the attention kernel from the committed ncu
+    summary, if it was taken on the current kernel source; else None."""
+    try:
+        with open(TRAFFIC_FILE) as f:
+            kv = dict(line.strip().split("=", 1) for line in f if "=" in line)
+        if kv.get("kernel_source_sha256_16") != _attention_source_hash():
+            return None
+        return float(kv["dram_bytes_per_step"])
+    except (OSError, KeyError, ValueError):
+        return None
+
+
+# --------------------------------------------------------------------- clocks
+class ClockSampler:
+    FIELDS = ("timestamp,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_id: str):
+        self.proc = None
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={gpu_id}", f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+
+    def stop(self, t0: float, t1: float):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=10)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        rows = []
+        for line in out.splitlines():
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                ts = time.mktime(time.strptime(parts[0].split(".")[0], "%Y/%m/%d %H:%M:%S"))
+                rows.append((ts, float(parts[1]), float(parts[2]), parts[5:9]))
+            except ValueError:
+                continue
+        if not rows:
+            return None
+        inside = [r for r in rows if t0 - 1 <= r[0] <= t1 + 1] or rows
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in inside for i, v in enumerate(r[3]) if v == "Active"})
+        return {"sm_mhz": statistics.median(r[1] for r in inside),
+                "sm_max_mhz": max(r[2] for r in inside), "reasons": reasons,
+                "samples": len(inside)}
+
+
+# ------------------------------------------------------------------ oracle leg
+def _oracle_cache(seed: int = 7):
+    """Rotated keys and values of a 122,880-token cache for the oracle."""
+    import numpy as np
+    from oracle import oracle as orc
+    from paper_2605_07325_gb300 import synth
+    rng = np.random.default_rng(seed)
+    k = synth.bf16_to_f64(synth.bf16_bits(rng.standard_normal((L0, HKV, D), dtype=np.float32)))
+    v = synth.bf16_to_f64(synth.bf16_bits(rng.standard_normal((L0, HKV, D), dtype=np.float32)))
+    k = orc.rope(k, np.arange(L0), BASE)
+    return k, v
+
+
+def _oracle_step_sample(k_cache, v_cache, n_chunk: int, n_suffix: int, seed: int):
+    """Time the oracle on n_chunk tokens of the chunk and n_suffix tokens of
+    the suffix (all 64 query heads), and return (seconds, sampled pairs,
+    full-step pairs) so the time can be scaled to the whole step."""
+    import numpy as np
+    from oracle import oracle as orc
+    from paper_2605_07325_gb300 import costmodel, synth
+    rng = np.random.default_rng(seed)
+    new = CHUNK + SUFFIX
+    q = synth.bf16_to_f64(synth.bf16_bits(rng.standard_normal((new, HQ, D), dtype=np.float32)))
+    kn = synth.bf16_to_f64(synth.bf16_bits(rng.standard_normal((new, HKV, D), dtype=np.float32)))
+    vn = synth.bf16_to_f64(synth.bf16_bits(rng.standard_normal((new, HKV, D), dtype=np.float32)))
+    pos_new = np.arange(L0, L0 + new)
+    sel = np.concatenate([np.arange(n_chunk), CHUNK + np.arange(n_suffix)])
+    t0 = time.perf_counter()
+    kn_rot = orc.rope(kn, pos_new, BASE)                         # all new keys
+    q_rot = orc.rope(q[sel], pos_new[sel], BASE)                 # sampled queries
+    k_all = np.concatenate([k_cache, kn_rot])
+    v_all = np.concatenate([v_cache, vn])
+    kpos = np.arange(L0 + new)
+    orc.attention(q_rot, pos_new[sel], k_all, v_all, kpos, 1.0 / math.sqrt(D))
+    secs = time.perf_counter() - t0
+    sampled = int(sum(L0 + int(s) + 1 for s in sel))
+    full = costmodel.query_key_pairs(L0, new)
+    return secs, sampled, full
+
+
+def cpu_baseline(target_s: float = 15.0):
+    """The oracle as it stands, on this host's cores, on a bounded sample of
+    the step, scaled by query-key pairs to microseconds per layer-step."""
+    from oracle import oracle as orc
+    k, v = _oracle_cache()
+    s1, p1, full = _oracle_step_sample(k, v, 1, 1, seed=11)       # calibration
+    per_pair = s1 / p1
+    tokens = max(2, min(CHUNK + SUFFIX, int(target_s / (per_pair * (L0 + 300)))))
+    n_c = min(CHUNK, tokens // 2)
+    n_s = min(SUFFIX, tokens - n_c)
+    secs, pairs, full = _oracle_step_sample(k, v, n_c, n_s, seed=12)
+    us = secs * full / pairs * 1e6
+    return {"value": us, "unit": UNIT, "cores": orc.default_threads(), "kind": "oracle",
+            "sample": (f"fp64 C oracle: RoPE of the step's 768 new keys + attention of {n_c} chunk "
+                       f"and {n_s} suffix query tokens (all 64 heads) over 122,880+ keys, "
+                       f"{secs:.1f} s, scaled by query-key pairs to the full step")}
+
+
+def run_reference(args):
+    """--impl reference: the fp64 oracle timed alone on the host cores."""
+    from oracle import oracle as orc
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return 0
+    k, v = _oracle_cache()
+    s1, p1, _ = _oracle_step_sample(k, v, 1, 1, seed=11)
+    budget = 150.0 / max(1, args.steps + args.warmup)              # seconds per step
+    tokens = max(2, int(budget / (s1 / p1 * (L0 + 300))))
+    n_c, n_s = tokens // 2, tokens - tokens // 2
+    vals = []
+    for i in range(args.warmup + args.steps):
+        secs, pairs, full = _oracle_step_sample(k, v, n_c, n_s, seed=100 + i)
+        if i >= args.warmup:
+            vals.append(secs * full / pairs * 1e6)
+    value = statistics.mean(vals)
+    cores = orc.default_threads()
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT,
+            "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": value / 1e3, "higher_is_better": False, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": WORKLOAD_NAME},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+                             "sample": f"per step: {n_c} chunk + {n_s} suffix query tokens, "
+                                       "scaled by query-key pairs"},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+# -------------------------------------------------------------------- GPU leg
+def run_ours(args):
+    import torch
+    import torch.distributed as dist
+    from paper_2605_07325_gb300 import costmodel, csr
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=dev)
+
+    K, W = args.steps, args.warmup
+    fill_chunks = (L0 - PREFIX) // CHUNK - W          # W warm-up steps bring L to L0
+    max_tokens = L0 + CHUNK * (K + 2) + SUFFIX
+    pool_pages = math.ceil(max_tokens / P) + 16
+    cfg = csr.make_config(HQ, HKV, D, P, BASE, max_new_tokens=PREFIX, pool_pages=pool_pages,
+                          max_seq_tokens=max_tokens + P)
+    stream = torch.cuda.Stream(device=dev, priority=-1)
+    gen = torch.Generator(device=dev).manual_seed(1234 + rank)
+
+    def rnd(n, h):
+        return torch.randn((n, h, D), generator=gen, device=dev, dtype=torch.float32).to(torch.bfloat16)
+
+    with torch.cuda.stream(stream):
+        ctx = csr.Context(cfg, device=str(dev), stream=stream)
+        pq, pk, pv = rnd(PREFIX, HQ), rnd(PREFIX, HKV), rnd(PREFIX, HKV)
+        ctx.init_static(pq, pk, pv, stream=stream)
+        fq = rnd(CHUNK, HQ)
+        fout = torch.empty((CHUNK, HQ, D), dtype=torch.bfloat16, device=dev)
+        for _ in range(fill_chunks):
+            ctx.append_chunk(fq, rnd(CHUNK, HKV), rnd(CHUNK, HKV), out=fout, stream=stream)
+        sets = []
+        for _ in range(4):
+            sets.append(dict(cq=rnd(CHUNK, HQ), ck=rnd(CHUNK, HKV), cv=rnd(CHUNK, HKV),
+                             sq=rnd(SUFFIX, HQ), sk=rnd(SUFFIX, HKV), sv=rnd(SUFFIX, HKV),
+                             co=torch.empty((CHUNK, HQ, D), dtype=torch.bfloat16, device=dev),
+                             so=torch.empty((SUFFIX, HQ, D), dtype=torch.bfloat16, device=dev)))
+    stream.synchronize()
+    assert ctx.layout()[1] == L0 - CHUNK * W, ctx.layout()[1]
+
+    def step(i):
+        s = sets[i % len(sets)]
+        ctx.append_chunk(s["cq"], s["ck"], s["cv"], out=s["co"], stream=stream)
+        ctx.attend_suffix(s["sq"], s["sk"], s["sv"], out=s["so"], stream=stream)
+        ctx.truncate_suffix()
+
+    for i in range(W):
+        step(i)
+    stream.synchronize()
+    assert ctx.layout()[1] == L0
+
+    # ------------------------------------------------ device-timed region
+    props = torch.cuda.get_device_properties(dev)
+    uuid = getattr(props, "uuid", None)
+    gpu_id = f"GPU-{uuid}" if uuid is not None else os.environ.get("CUDA_VISIBLE_DEVICES", "0").split(",")[local]
+    sampler = ClockSampler(gpu_id)
+    ctx.set_timing(True)
+    launches0 = ctx.kernel_launches()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize(dev)
+    t_wall0 = time.time()
+    e0.record(stream)
+    for i in range(K):
+        step(i)
+    e1.record(stream)
+    torch.cuda.synchronize(dev)
+    t_wall1 = time.time()
+    if world > 1:
+        dist.barrier()
+    ms_total = e0.elapsed_time(e1)
+    launches = ctx.kernel_launches() - launches0
+    ktimes = ctx.get_timing()
+    ctx.set_timing(False)
+    clocks = sampler.stop(t_wall0, t_wall1)
+
+    # ------------------------------------------------ end to end, host buffers
+    host = []
+    for s in sets:
+        host.append({k: v.cpu().pin_memory() for k, v in s.items() if k[1] in "qkv"})
+        host[-1]["co"] = torch.empty((CHUNK, HQ, D), dtype=torch.bfloat16).pin_memory()
+        host[-1]["so"] = torch.empty((SUFFIX, HQ, D), dtype=torch.bfloat16).pin_memory()
+    stage = {k: torch.empty_like(v) for k, v in sets[0].items()}
+    h2d = sum(v.numel() * 2 for k, v in sets[0].items() if k[1] in "qkv")
+    d2h = (CHUNK + SUFFIX) * HQ * D * 2
+
+    def step_e2e(i):
+        h = host[i % len(host)]
+        with torch.cuda.stream(stream):
+            for k in ("cq", "ck", "cv", "sq", "sk", "sv"):
+                stage[k].copy_(h[k], non_blocking=True)
+            ctx.append_chunk(stage["cq"], stage["ck"], stage["cv"], out=stage["co"], stream=stream)
+            ctx.attend_suffix(stage["sq"], stage["sk"], stage["sv"], out=stage["so"], stream=stream)
+            ctx.truncate_suffix()
+            h["co"].copy_(stage["co"], non_blocking=True)
+            h["so"].copy_(stage["so"], non_blocking=True)
+
+    for i in range(W):
+        step_e2e(i)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize(dev)
+    e2, e3 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e2.record(stream)
+    for i in range(K):
+        step_e2e(i)
+    e3.record(stream)
+    torch.cuda.synchronize(dev)
+    if world > 1:
+        dist.barrier()
+    ms_e2e = e2.elapsed_time(e3)
+    flags = ctx.device_status()
+
+    if world > 1:
+        t = torch.tensor([ms_total, ms_e2e], device=dev, dtype=torch.float64)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms_total, ms_e2e = float(t[0]), float(t[1])
+
+    # ------------------------------------------------ roofline of the attention kernel
+    hbm, peak_burst, peak_sust, peak_kind = _peaks()
+    # the timed steps covered L = L0 + 256 i for the chunk and + 256 for the suffix
+    flops = sum(costmodel.attention_flops(HQ, D, L0 + CHUNK * i, CHUNK) +
+                costmodel.attention_flops(HQ, D, L0 + CHUNK * (i + 1), SUFFIX) for i in range(K))
+    att_ms, att_n = ktimes["attention"]
+    achieved = flops / (att_ms * 1e-3) / 1e12 if att_ms > 0 else None
+    traffic_step = _traffic_per_launch_step()
+    step_floor = statistics.mean(
+        costmodel.floor_seconds(costmodel.attention_flops(HQ, D, L0 + CHUNK * i, CHUNK),
+                                costmodel.call_bytes(HQ, HKV, D, L0 + CHUNK * i, CHUNK), peak_burst, hbm) +
+        costmodel.floor_seconds(costmodel.attention_flops(HQ, D, L0 + CHUNK * (i + 1), SUFFIX),
+                                costmodel.call_bytes(HQ, HKV, D, L0 + CHUNK * (i + 1), SUFFIX), peak_burst, hbm)
+        for i in range(K)) * 1e6
+    us_step = ms_total / K * 1e3
+    line = {
+        "metric": METRIC, "value": us_step, "unit": UNIT, "n_gpus": world, "steps": K,
+        "warmup": W, "ms_per_step": ms_total / K, "higher_is_better": False, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic: seeded N(0,1) bf16 Q/K/V (torch CUDA generator), resident in HBM",
+        "config": {"workload": WORKLOAD_NAME, "cached_tokens_first_step": L0,
+                   "cached_tokens_last_step": L0 + CHUNK * (K - 1),
+                   "l2": "inputs larger than L2: the 252 MB KV cache is streamed every step",
+                   "replicas": world, "foreground_ctas": ctx.cfg.num_ctas or props.multi_processor_count},
+        "roofline": {"bound": "tensor", "achieved": achieved, "peak": peak_burst, "unit": "TFLOP/s",
+                     "frac": (achieved / peak_burst) if achieved else None,
+                     "traffic": (traffic_step / 2) if traffic_step else None,
+                     "kernel": "attn_kernel<128> (tcgen05 QK^T and PV, TMA paged K/V)",
+                     "launches": att_n, "avg_launch_us": att_ms / max(1, att_n) * 1e3,
+                     "peak_source": f"bf16_tflops ({peak_kind}, burst)",
+                     "frac_of_sustained": (achieved / peak_sust) if achieved else None},
+        "step_roofline": {"floor_us": step_floor, "frac": step_floor / us_step,
+                          "note": "max(FLOPs / bf16 peak, bytes / HBM peak) per call, summed over the step"},
+        "ttft_proxy_94_layers_ms": us_step * LAYERS_PROXY / 1e3,
+        "kernels": {k: {"ms_total": v[0], "launches": v[1]} for k, v in ktimes.items() if v[1]},
+        "e2e": {"value": ms_e2e / K * 1e3, "unit": UNIT, "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": d2h},
+        "gpu_launches": launches,
+        "clocks": clocks,
+        "device_error_flags": flags,
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline()
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    ctx.close()
+    if world > 1:
+        dist.destroy_process_group()
+    return 0
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args(argv)
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_ours(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -263,6 +263,27 @@ csr_status csr_device_status(csr_ctx *ctx, uint32_t *flags);
 /* Number of kernels the context has launched since creation. */
 int64_t csr_kernel_launches(const csr_ctx *ctx);
 
+/* Kernel kinds of csr_timing. */
+#define CSR_KERNEL_ROPE_APPEND 0
+#define CSR_KERNEL_ATTENTION 1
+#define CSR_KERNEL_MERGE 2
+#define CSR_KERNEL_EVICT 3
+#define CSR_KERNEL_KINDS 4
+
+typedef struct csr_timing {
+  double ms[CSR_KERNEL_KINDS];        /* summed device time per kernel kind */
+  int64_t launches[CSR_KERNEL_KINDS]; /* timed launches per kernel kind */
+} csr_timing;
+
+/*
+ * Per-kernel timing of the foreground path: while enabled, every kernel a
+ * foreground call launches is bracketed by two CUDA events on the call's
+ * stream.  csr_get_timing waits for those events, sums their elapsed times
+ * per kernel kind into *out and forgets them.  Disabling drops pending events.
+ */
+csr_status csr_set_timing(csr_ctx *ctx, int enable);
+csr_status csr_get_timing(csr_ctx *ctx, csr_timing *out);
+
 /* Text of the last failure on this context (never NULL). */
 const char *csr_last_error(const csr_ctx *ctx);
 

@@ -53,6 +53,13 @@ class Config(ctypes.Structure):
     ]
 
 
+KERNEL_KINDS = ("rope_append", "attention", "merge", "evict_compact")
+
+
+class Timing(ctypes.Structure):
+    _fields_ = [("ms", ctypes.c_double * 4), ("launches", ctypes.c_int64 * 4)]
+
+
 PROVIDER = ctypes.CFUNCTYPE(ctypes.c_int, ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32,
                             ctypes.POINTER(ctypes.c_void_p), ctypes.POINTER(ctypes.c_void_p),
                             ctypes.POINTER(ctypes.c_void_p), ctypes.POINTER(ctypes.c_void_p))
@@ -81,6 +88,8 @@ _SIGS = {
     "csr_device_status": ([_vp, _Pu32], ctypes.c_int),
     "csr_kernel_launches": ([_vp], ctypes.c_int64),
     "csr_last_error": ([_vp], ctypes.c_char_p),
+    "csr_set_timing": ([_vp, ctypes.c_int], ctypes.c_int),
+    "csr_get_timing": ([_vp, ctypes.POINTER(Timing)], ctypes.c_int),
 }
 for _name, (_args, _res) in _SIGS.items():
     _fn = getattr(_lib, _name)
@@ -300,6 +309,15 @@ class Context:
     def kernel_launches(self) -> int:
         return int(_lib.csr_kernel_launches(self._h))
 
+    def set_timing(self, enable: bool) -> None:
+        self._check(_lib.csr_set_timing(self._h, 1 if enable else 0))
+
+    def get_timing(self) -> Dict[str, Tuple[float, int]]:
+        """{kernel: (summed ms, launches)} of the foreground launches timed so far."""
+        t = Timing()
+        self._check(_lib.csr_get_timing(self._h, ctypes.byref(t)))
+        return {k: (t.ms[i], int(t.launches[i])) for i, k in enumerate(KERNEL_KINDS)}
+
     def last_error(self) -> str:
         return _lib.csr_last_error(self._h).decode()
 
@@ -312,6 +330,6 @@ def _alias_int32(ptr: int, n: int, device) -> torch.Tensor:
     """An int32 CUDA tensor viewing n entries of raw device memory (no ownership)."""
 
     class _Holder:
-        __cuda_array_interface__ = {"shape": (n,), "typestr": "<i4", "data": (ptr, True),
+        __cuda_array_interface__ = {"shape": (n,), "typestr": "<i4", "data": (ptr, False),
                                     "version": 3, "strides": None}
     return torch.as_tensor(_Holder(), device=device)

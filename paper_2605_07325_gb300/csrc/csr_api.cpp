@@ -215,6 +215,14 @@ struct csr_ctx {
   cudaEvent_t ev_fg = nullptr, ev_rb = nullptr;
   int64_t launches = 0;
   std::string err = "no error";
+  // per-kernel event timing of foreground launches
+  struct Timed {
+    int kind;
+    cudaEvent_t a, b;
+  };
+  bool timing = false;
+  std::vector<Timed> timed;
+  std::vector<cudaEvent_t> spare_events;
 
   template <class T> T *wsp(size_t off) { return reinterpret_cast<T *>(ws + off); }
   Version &act() { return ver[active.load()]; }
@@ -234,6 +242,32 @@ csr_status cuda_fail(csr_ctx *c, cudaError_t e, const char *where) {
 }
 
 int64_t pages_for(const csr_ctx *c, int64_t len) { return ceil_div(len, c->cfg.page_size); }
+
+cudaEvent_t take_event(csr_ctx *c) {
+  if (!c->spare_events.empty()) {
+    cudaEvent_t e = c->spare_events.back();
+    c->spare_events.pop_back();
+    return e;
+  }
+  cudaEvent_t e = nullptr;
+  cudaEventCreate(&e);
+  return e;
+}
+
+// Launch through `fn` (returns cudaError_t); bracket it with timing events on
+// foreground launches while timing is enabled.
+template <class F>
+cudaError_t timed_launch(csr_ctx *c, int kind, bool foreground, cudaStream_t s, F fn) {
+  if (!(c->timing && foreground)) return fn();
+  cudaEvent_t a = take_event(c), b = take_event(c);
+  if (!a || !b) return cudaErrorMemoryAllocation;
+  cudaError_t e = cudaEventRecord(a, s);
+  if (e == cudaSuccess) e = fn();
+  if (e == cudaSuccess) e = cudaEventRecord(b, s);
+  if (e != cudaSuccess) return e;
+  c->timed.push_back({kind, a, b});
+  return cudaSuccess;
+}
 
 // K1 -> K2 -> K3 for n tokens at positions L.. of version `slot`.
 // ws: 0 = foreground staging, 1 = rebuild staging.  ids/n_ids name the physical
@@ -265,7 +299,8 @@ csr_status run_block(csr_ctx *c, int slot, int ws, const void *q, const void *k,
   rp.n_ids = n_ids;
   std::memcpy(rp.inv_turns, c->inv_turns, sizeof(rp.inv_turns));
   for (int i = 0; i < n_ids; ++i) rp.ids[i] = ids[i];
-  cudaError_t e = launch_rope_append(rp, s);
+  const bool fg = ws == 0;
+  cudaError_t e = timed_launch(c, CSR_KERNEL_ROPE_APPEND, fg, s, [&] { return launch_rope_append(rp, s); });
   if (e != cudaSuccess) return cuda_fail(c, e, "rope_append launch");
   ++c->launches;
 
@@ -305,7 +340,7 @@ csr_status run_block(csr_ctx *c, int slot, int ws, const void *q, const void *k,
   }
   ap.grid = static_cast<int32_t>(grid);
   ap.scale_log2 = c->scale_log2;
-  e = launch_attention(ap, cf.head_dim, s);
+  e = timed_launch(c, CSR_KERNEL_ATTENTION, fg, s, [&] { return launch_attention(ap, cf.head_dim, s); });
   if (e != cudaSuccess) return cuda_fail(c, e, "attention launch");
   ++c->launches;
   if (ap.grid > 1) {
@@ -324,7 +359,7 @@ csr_status run_block(csr_ctx *c, int slot, int ws, const void *q, const void *k,
     mp.n_tiles = ap.n_tiles;
     mp.grid = ap.grid;
     mp.d = cf.head_dim;
-    e = launch_merge(mp, s);
+    e = timed_launch(c, CSR_KERNEL_MERGE, fg, s, [&] { return launch_merge(mp, s); });
     if (e != cudaSuccess) return cuda_fail(c, e, "merge launch");
     ++c->launches;
   }
@@ -511,6 +546,11 @@ void csr_destroy(csr_ctx *c) {
     cudaDeviceSynchronize();
     if (c->ev_fg) cudaEventDestroy(c->ev_fg);
     if (c->ev_rb) cudaEventDestroy(c->ev_rb);
+    for (auto &t : c->timed) {
+      cudaEventDestroy(t.a);
+      cudaEventDestroy(t.b);
+    }
+    for (cudaEvent_t e : c->spare_events) cudaEventDestroy(e);
   }
   delete c;
 }
@@ -871,6 +911,38 @@ csr_status csr_device_status(csr_ctx *c, uint32_t *flags) {
 }
 
 int64_t csr_kernel_launches(const csr_ctx *c) { return c ? c->launches : 0; }
+
+csr_status csr_set_timing(csr_ctx *c, int enable) {
+  if (!c) return CSR_EINVAL;
+  if (c->plan_only) return fail(c, CSR_ESTATE, "plan-only context launches no kernels");
+  if (!enable) {
+    for (auto &t : c->timed) {
+      cudaEventSynchronize(t.b);
+      c->spare_events.push_back(t.a);
+      c->spare_events.push_back(t.b);
+    }
+    c->timed.clear();
+  }
+  c->timing = enable != 0;
+  return CSR_OK;
+}
+
+csr_status csr_get_timing(csr_ctx *c, csr_timing *out) {
+  if (!c || !out) return CSR_EINVAL;
+  std::memset(out, 0, sizeof(*out));
+  for (auto &t : c->timed) {
+    float ms = 0.f;
+    cudaError_t e = cudaEventSynchronize(t.b);
+    if (e == cudaSuccess) e = cudaEventElapsedTime(&ms, t.a, t.b);
+    if (e != cudaSuccess) return cuda_fail(c, e, "reading kernel timing events");
+    out->ms[t.kind] += ms;
+    out->launches[t.kind] += 1;
+    c->spare_events.push_back(t.a);
+    c->spare_events.push_back(t.b);
+  }
+  c->timed.clear();
+  return CSR_OK;
+}
 
 const char *csr_last_error(const csr_ctx *c) { return c ? c->err.c_str() : "NULL context"; }
 
