@@ -156,6 +156,17 @@ csr_status csr_attend_suffix(csr_ctx *ctx, const void *q, const void *k,
 csr_status csr_truncate_suffix(csr_ctx *ctx);
 
 /*
+ * Invalidate the cache after its first `length` tokens (section III-B: a
+ * cache stays valid up to the first differing token i*, Eq.
+ * first_differing_token, so a task that differs from position length+1 on
+ * reuses exactly this much).  `length` must be the end of the static prefix or
+ * of a chunk of the active version; the later chunks are dropped and their
+ * pages return to the pool.  Host-only (no kernel).  CSR_ESTATE while a suffix
+ * is live or a reconciliation runs, CSR_EINVAL if length is not a boundary.
+ */
+csr_status csr_rewind(csr_ctx *ctx, int64_t length);
+
+/*
  * Source of a chunk's layer inputs for the rebuild (the "LLM(X_eps)" of
  * Algorithm 1 recomputes a retained chunk in its new context).  The callback
  * is called on the thread that drives the context, with the chunk's id and

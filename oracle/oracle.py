@@ -289,6 +289,22 @@ class OracleCSR:
         while len(ver.pages) > keep:
             self.alloc.release(ver.pages.pop())
 
+    def rewind(self, length: int) -> None:
+        """Keep the first `length` tokens: the cache is valid up to the first
+        differing token (Eq. first_differing_token); later chunks are dropped."""
+        ver = self.active
+        if self._live_suffix(ver) or self.is_reconciling:
+            raise ValueError("suffix live or reconciling")
+        at, keep = 0, 0
+        while at < length and keep < len(ver.segments):
+            at += len(ver.segments[keep].pos)
+            keep += 1
+        if at != length:
+            raise ValueError("not a segment boundary")
+        ver.segments = ver.segments[:keep]
+        while len(ver.pages) > self._pages_for(length):
+            self.alloc.release(ver.pages.pop())
+
     def chunk_ids(self) -> List[int]:
         return [s.ident for s in self.active.segments if s.kind == "chunk"]
 

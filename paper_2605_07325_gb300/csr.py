@@ -76,6 +76,7 @@ _SIGS = {
     "csr_append_chunk": ([_vp, _vp, _vp, _vp, _i32, _vp, _vp, _vp, _P64], ctypes.c_int),
     "csr_attend_suffix": ([_vp, _vp, _vp, _vp, _i32, _vp, _vp, _vp], ctypes.c_int),
     "csr_truncate_suffix": ([_vp], ctypes.c_int),
+    "csr_rewind": ([_vp, _i64], ctypes.c_int),
     "csr_set_reconciler": ([_vp, PROVIDER, _vp, _vp], ctypes.c_int),
     "csr_evict_and_reconcile": ([_vp, _i32, _vp], ctypes.c_int),
     "csr_poll_swap": ([_vp, _vp, ctypes.POINTER(ctypes.c_int)], ctypes.c_int),
@@ -213,6 +214,10 @@ class Context:
 
     def truncate_suffix(self) -> None:
         self._check(_lib.csr_truncate_suffix(self._h))
+
+    def rewind(self, length: int) -> None:
+        """Keep the first `length` tokens (a prefix or chunk boundary)."""
+        self._check(_lib.csr_rewind(self._h, int(length)))
 
     # -------------------------------------------------------- reconciliation
     def set_reconciler(self, provider: Callable[[int, int], tuple], lo_stream=None) -> None:

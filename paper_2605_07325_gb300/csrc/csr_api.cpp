@@ -602,6 +602,25 @@ csr_status csr_truncate_suffix(csr_ctx *c) {
   return CSR_OK;
 }
 
+csr_status csr_rewind(csr_ctx *c, int64_t length) {
+  if (!c) return CSR_EINVAL;
+  Version &A = c->act();
+  if (A.suffix_len > 0) return fail(c, CSR_ESTATE, "a suffix is live");
+  if (c->reconciling) return fail(c, CSR_ESTATE, "a reconciliation is running");
+  if (!c->has_static) return fail(c, CSR_ESTATE, "csr_init_static must come first");
+  int64_t at = A.prefix_len;
+  size_t keep = 0;
+  while (at < length && keep < A.chunks.size()) at += A.chunks[keep++].len;
+  if (at != length) return fail(c, CSR_EINVAL, "length is not the end of the prefix or of a chunk");
+  A.chunks.resize(keep);
+  const int64_t pages = pages_for(c, length);
+  while (static_cast<int64_t>(A.pages.size()) > pages) {
+    c->pool.release(A.pages.back());
+    A.pages.pop_back();
+  }
+  return CSR_OK;
+}
+
 csr_status csr_set_reconciler(csr_ctx *c, csr_qkv_provider provider, void *user,
                               csr_stream_t lo_stream) {
   if (!c) return CSR_EINVAL;

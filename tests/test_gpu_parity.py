@@ -135,3 +135,24 @@ def test_launch_count_reported(libcsr):
     before = p.ctx.kernel_launches()
     p.init_static(p.blk(70, 100))
     assert p.ctx.kernel_launches() - before >= 2   # K1 + K2 (+ K3)
+
+
+def test_rewind_then_append_matches_never_appended(libcsr):
+    """Cache invalidation after a chunk boundary (Eq. first_differing_token):
+    the next chunk's output and layout equal a run that never had the dropped
+    chunk, bit for bit."""
+    a = Pair(C2, pool_pages=128, max_seq=8192, max_new=512)
+    b = Pair(C2, pool_pages=128, max_seq=8192, max_new=512)
+    for p in (a, b):
+        p.init_static(p.blk(80, 300), compare=False)
+        p.append(p.blk(81, 100), compare=False)
+    a.append(a.blk(82, 200), compare=False)
+    a.ctx.rewind(400)
+    a.orc.rewind(400)
+    oa, _, _ = a.append(a.blk(83, 150))
+    ob, _, _ = b.append(b.blk(83, 150))
+    torch.cuda.synchronize()
+    assert np.array_equal(bits_of(oa), bits_of(ob))
+    assert a.ctx.layout() == b.ctx.layout()
+    a.check_layout()
+    a.device_clean()

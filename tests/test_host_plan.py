@@ -181,3 +181,26 @@ def test_invalid_configs_rejected(libcsr, bad):
     with pytest.raises(libcsr.CsrError) as e:
         libcsr.Context(cfg)
     assert e.value.status == libcsr.EINVAL
+
+
+def test_rewind_matches_oracle(libcsr):
+    ctx, m = _plan(libcsr), _Model(64)
+    ctx.init_static(None, None, None, n=40)
+    m.o.init_static(*m.blk(40))
+    for n in (10, 30, 7):
+        ctx.append_chunk(None, None, None, n=n)
+        m.o.append_chunk(*m.blk(n))
+    for bad in (41, 45, 200, 39):
+        _err(libcsr, lambda: ctx.rewind(bad), libcsr.EINVAL)
+    ctx.rewind(80)
+    m.o.rewind(80)
+    _same(ctx, m, libcsr)
+    ctx.rewind(40)
+    m.o.rewind(40)
+    _same(ctx, m, libcsr)
+    assert ctx.chunks()[0] == []
+    ctx.append_chunk(None, None, None, n=25)
+    m.o.append_chunk(*m.blk(25))
+    _same(ctx, m, libcsr)
+    ctx.attend_suffix(None, None, None, n=3)
+    _err(libcsr, lambda: ctx.rewind(40), libcsr.ESTATE)

@@ -162,3 +162,19 @@ def test_reconcile_page_reservation_order(oracle_mod):
     s.reconcile()
     assert s.page_table() == [0, 1, 6, 7, 9]
     assert s.free_ids()[:5] == [2, 3, 4, 5, 8]
+
+
+def test_rewind_then_append_equals_never_appended(oracle_mod):
+    """Eq. first_differing_token: after invalidating the cache past a chunk
+    boundary, the next chunk sees exactly the cache it would have seen."""
+    orc = oracle_mod
+    a, b = _session(orc), _session(orc)
+    for s in (a, b):
+        s.init_static(*_blk(0, 33))
+        s.append_chunk(*_blk(1, 16))
+    a.append_chunk(*_blk(2, 40))
+    a.rewind(49)
+    oa = a.append_chunk(*_blk(3, 21))
+    ob = b.append_chunk(*_blk(3, 21))
+    assert np.array_equal(oa[0], ob[0]) and a.page_table() == b.page_table()
+    assert a.free_ids() == b.free_ids()
