@@ -227,7 +227,8 @@ def run_ours(args):
         dist.init_process_group("nccl", device_id=dev)
 
     K, W = args.steps, args.warmup
-    fill_chunks = (L0 - PREFIX) // CHUNK
+    fill = args.fill_chunk
+    fill_chunks = (L0 - PREFIX) // fill
     max_tokens = L0 + CHUNK + SUFFIX
     pool_pages = math.ceil(max_tokens / P) + 16
     cfg = csr.make_config(HQ, HKV, D, P, BASE, max_new_tokens=PREFIX, pool_pages=pool_pages,
@@ -242,10 +243,10 @@ def run_ours(args):
         ctx = csr.Context(cfg, device=str(dev), stream=stream)
         pq, pk, pv = rnd(PREFIX, HQ), rnd(PREFIX, HKV), rnd(PREFIX, HKV)
         ctx.init_static(pq, pk, pv, stream=stream)
-        fq = rnd(CHUNK, HQ)
-        fout = torch.empty((CHUNK, HQ, D), dtype=torch.bfloat16, device=dev)
+        fq = rnd(fill, HQ)
+        fout = torch.empty((fill, HQ, D), dtype=torch.bfloat16, device=dev)
         for _ in range(fill_chunks):
-            ctx.append_chunk(fq, rnd(CHUNK, HKV), rnd(CHUNK, HKV), out=fout, stream=stream)
+            ctx.append_chunk(fq, rnd(fill, HKV), rnd(fill, HKV), out=fout, stream=stream)
         sets = []
         for _ in range(4):
             sets.append(dict(cq=rnd(CHUNK, HQ), ck=rnd(CHUNK, HKV), cv=rnd(CHUNK, HKV),
@@ -397,6 +398,9 @@ def main(argv=None):
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--fill-chunk", type=int, default=CHUNK, choices=[256, 512, 1024, 2048, 4096],
+                    help="chunk size used to fill the cache before timing (fewer launches "
+                         "for profiler captures); the timed steps are unchanged")
     args = ap.parse_args(argv)
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
