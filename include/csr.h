@@ -87,8 +87,10 @@ typedef struct csr_config {
   int32_t evict_tokens;   /* tokens of the oldest chunks dropped by an automatic eviction */
   int32_t n_catchup;      /* N_catchup of Algorithm 1 */
   int32_t num_ctas;       /* CTAs of a foreground attention launch; 0 = one per SM */
-  int32_t rebuild_tiles_per_cta; /* key tiles per CTA in rebuild launches; 0 = 64 */
+  int32_t rebuild_tiles_per_cta; /* key tiles (128 keys) per CTA in rebuild launches; 0 = 64 */
   int32_t flags;          /* CSR_FLAG_* */
+  int32_t fg_chunk_tiles; /* key tiles per split-KV item of a foreground launch; 0 = chosen
+                             per launch from its shape */
 } csr_config;
 
 /*

@@ -50,6 +50,7 @@ class Config(ctypes.Structure):
         ("num_ctas", ctypes.c_int32),
         ("rebuild_tiles_per_cta", ctypes.c_int32),
         ("flags", ctypes.c_int32),
+        ("fg_chunk_tiles", ctypes.c_int32),
     ]
 
 
@@ -106,10 +107,11 @@ class CsrError(RuntimeError):
 
 def make_config(num_q_heads, num_kv_heads, head_dim, page_size, rope_base, max_new_tokens,
                 pool_pages, max_seq_tokens, softmax_scale=0.0, cap_tokens=0, evict_tokens=0,
-                n_catchup=0, num_ctas=0, rebuild_tiles_per_cta=0, flags=0) -> Config:
+                n_catchup=0, num_ctas=0, rebuild_tiles_per_cta=0, flags=0,
+                fg_chunk_tiles=0) -> Config:
     return Config(num_q_heads, num_kv_heads, head_dim, page_size, float(rope_base),
                   float(softmax_scale), max_new_tokens, pool_pages, max_seq_tokens, cap_tokens,
-                  evict_tokens, n_catchup, num_ctas, rebuild_tiles_per_cta, flags)
+                  evict_tokens, n_catchup, num_ctas, rebuild_tiles_per_cta, flags, fg_chunk_tiles)
 
 
 def pool_bytes(cfg: Config) -> int:

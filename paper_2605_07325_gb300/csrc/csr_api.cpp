@@ -29,7 +29,7 @@ using namespace csr;
 namespace {
 
 constexpr int kFgGridDefaultCap = 304;   // 2 x 152 SMs
-constexpr int kRebuildGridFactor = 8;    // rebuild CTAs per foreground CTA, at most
+constexpr int kPartialItems = 4096;      // split partials a launch may write (per staging)
 constexpr int kDefaultRebuildTiles = 64;
 constexpr size_t kAlign = 256;
 
@@ -125,7 +125,7 @@ bool encode_rows(CUtensorMap *m, void *base, uint64_t rows, uint64_t d, uint32_t
 
 struct Layout {  // workspace carve-out (byte offsets)
   size_t qpack[2], rb_out, part_o[2], part_lse[2], pt[2], ids_out, err, total;
-  int32_t rows_cap, fg_cap, rb_cap, max_pages;
+  int32_t rows_cap, fg_cap, max_pages;
 };
 
 bool valid_config(const csr_config *c, std::string *why) {
@@ -152,8 +152,8 @@ bool valid_config(const csr_config *c, std::string *why) {
   if (static_cast<int64_t>(c->pool_pages) * c->num_kv_heads * c->page_size >= (1ll << 31))
     return bad("pool rows exceed the 32-bit TMA coordinate range");
   if (c->cap_tokens < 0 || c->evict_tokens < 0 || c->n_catchup < 0 || c->num_ctas < 0 ||
-      c->rebuild_tiles_per_cta < 0)
-    return bad("negative cap_tokens/evict_tokens/n_catchup/num_ctas/rebuild_tiles_per_cta");
+      c->rebuild_tiles_per_cta < 0 || c->fg_chunk_tiles < 0)
+    return bad("negative cap_tokens/evict_tokens/n_catchup/num_ctas/chunk tiles");
   if (c->cap_tokens > 0 && c->evict_tokens <= 0) return bad("cap_tokens needs evict_tokens > 0");
   return true;
 }
@@ -163,7 +163,6 @@ Layout make_layout(const csr_config *c) {
   const int g = c->num_q_heads / c->num_kv_heads;
   L.rows_cap = static_cast<int32_t>(align_up(static_cast<size_t>(c->max_new_tokens) * g, kBM));
   L.fg_cap = c->num_ctas > 0 ? c->num_ctas : kFgGridDefaultCap;
-  L.rb_cap = kRebuildGridFactor * (c->num_ctas > 0 ? c->num_ctas : 152);
   L.max_pages = static_cast<int32_t>(ceil_div(c->max_seq_tokens, c->page_size) + 1);
   const size_t d = static_cast<size_t>(c->head_dim);
   size_t off = 0;
@@ -174,10 +173,9 @@ Layout make_layout(const csr_config *c) {
   };
   for (int i = 0; i < 2; ++i) L.qpack[i] = take(static_cast<size_t>(c->num_kv_heads) * L.rows_cap * d * 2);
   L.rb_out = take(static_cast<size_t>(c->max_new_tokens) * c->num_q_heads * d * 2);
-  const int caps[2] = {L.fg_cap, L.rb_cap};
   for (int i = 0; i < 2; ++i) {
-    L.part_o[i] = take(static_cast<size_t>(caps[i]) * 2 * kBM * d * 4);
-    L.part_lse[i] = take(static_cast<size_t>(caps[i]) * 2 * kBM * 4);
+    L.part_o[i] = take(static_cast<size_t>(kPartialItems) * kBM * d * 4);
+    L.part_lse[i] = take(static_cast<size_t>(kPartialItems) * kBM * 4);
   }
   for (int i = 0; i < 2; ++i) L.pt[i] = take(static_cast<size_t>(L.max_pages) * 4);
   L.ids_out = take(static_cast<size_t>(L.max_pages) * 4);
@@ -242,6 +240,38 @@ csr_status cuda_fail(csr_ctx *c, cudaError_t e, const char *where) {
 }
 
 int64_t pages_for(const csr_ctx *c, int64_t len) { return ceil_div(len, c->cfg.page_size); }
+
+// Key chunks per unit for a launch of `units` query tiles whose longest key
+// range is kv_max tiles.  Foreground: minimise a time estimate over the
+// persistent grid: waves x (tiles per item x t_tile + per-item cost) plus the
+// split partials' write + merge read.  Rebuild (max_tiles > 0): the fewest
+// chunks of at most max_tiles tiles, so each CTA is short and a foreground
+// launch waits at most one item for an SM.  Never more than kPartialItems
+// items when split.
+int32_t choose_chunk_tiles(int64_t units, int64_t kv_max, int64_t grid, int max_tiles,
+                           int head_dim) {
+  const double t_tile = 0.75, t_item = 2.0, t_part = head_dim == 128 ? 0.02 : 0.01;  // us
+  int64_t best_c = kv_max;
+  double best_t = 1e300;
+  for (int64_t S = 1; S <= std::min<int64_t>(kv_max, 256); ++S) {
+    const int64_t C = ceil_div(kv_max, S);
+    const int64_t Se = ceil_div(kv_max, C);
+    const int64_t items = units * Se;
+    if (Se > 1 && items > kPartialItems) break;
+    if (max_tiles > 0) {
+      if (C <= max_tiles) return static_cast<int32_t>(C);
+      best_c = C;  // the smallest chunk that still fits the partial buffer
+      continue;
+    }
+    const int64_t waves = ceil_div(items, grid);
+    const double t = waves * (C * t_tile + t_item) + (Se > 1 ? items * t_part : 0.0);
+    if (t < best_t - 1e-9) {
+      best_t = t;
+      best_c = C;
+    }
+  }
+  return static_cast<int32_t>(best_c);
+}
 
 cudaEvent_t take_event(csr_ctx *c) {
   if (!c->spare_events.empty()) {
@@ -325,39 +355,37 @@ csr_status run_block(csr_ctx *c, int slot, int ws, const void *q, const void *k,
   ap.n_pages_valid = static_cast<int32_t>(pages_for(c, L + n));
   ap.pool_pages = cf.pool_pages;
   const int T = kBM / c->group;
-  int64_t iph = 0;
-  for (int t = 0; t < ap.n_tiles; ++t) iph += unit_iters(L, n, T, t);
-  ap.iters_per_head = iph;
-  ap.total_iters = iph * cf.num_kv_heads;
-  int64_t grid;
-  if (ws == 0) {
-    grid = std::min<int64_t>(c->fg_grid, ap.total_iters);
+  const int64_t units = static_cast<int64_t>(ap.n_tiles) * cf.num_kv_heads;
+  const int64_t kv_max = unit_iters(L, n, T, ap.n_tiles - 1);
+  const int tpc = cf.rebuild_tiles_per_cta > 0 ? cf.rebuild_tiles_per_cta : kDefaultRebuildTiles;
+  if (ws == 0 && cf.fg_chunk_tiles > 0) {
+    // fixed chunk length, but never more split items than the partial buffer holds
+    const int64_t min_c = ceil_div(kv_max, std::max<int64_t>(1, kPartialItems / units));
+    ap.chunk_tiles = static_cast<int32_t>(std::max<int64_t>(cf.fg_chunk_tiles, min_c));
   } else {
-    const int tpc = cf.rebuild_tiles_per_cta > 0 ? cf.rebuild_tiles_per_cta : kDefaultRebuildTiles;
-    grid = std::max<int64_t>(std::min<int64_t>(c->num_sms, ap.total_iters),
-                             ceil_div(ap.total_iters, tpc));
-    grid = std::min<int64_t>(grid, c->lay.rb_cap);
+    ap.chunk_tiles = choose_chunk_tiles(units, kv_max, c->fg_grid, ws == 0 ? 0 : tpc, cf.head_dim);
   }
-  ap.grid = static_cast<int32_t>(grid);
+  const int64_t n_chunks = ceil_div(kv_max, ap.chunk_tiles);
+  ap.n_items = static_cast<int32_t>(n_chunks * units);
+  // foreground: persistent CTAs over the items; rebuild: one item per CTA
+  ap.grid = ws == 0 ? static_cast<int32_t>(std::min<int64_t>(c->fg_grid, ap.n_items)) : ap.n_items;
   ap.scale_log2 = c->scale_log2;
   e = timed_launch(c, CSR_KERNEL_ATTENTION, fg, s, [&] { return launch_attention(ap, cf.head_dim, s); });
   if (e != cudaSuccess) return cuda_fail(c, e, "attention launch");
   ++c->launches;
-  if (ap.grid > 1) {
+  if (n_chunks > 1) {
     MergeParams mp{};
     mp.part_o = ap.part_o;
     mp.part_lse = ap.part_lse;
     mp.out = ap.out;
     mp.lse = lse;
     mp.L = L;
-    mp.total_iters = ap.total_iters;
-    mp.iters_per_head = iph;
     mp.n = n;
     mp.hq = ap.hq;
     mp.hkv = ap.hkv;
     mp.group = ap.group;
     mp.n_tiles = ap.n_tiles;
-    mp.grid = ap.grid;
+    mp.chunk_tiles = ap.chunk_tiles;
     mp.d = cf.head_dim;
     e = timed_launch(c, CSR_KERNEL_MERGE, fg, s, [&] { return launch_merge(mp, s); });
     if (e != cudaSuccess) return cuda_fail(c, e, "merge launch");

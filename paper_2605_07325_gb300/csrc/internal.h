@@ -43,14 +43,14 @@ struct AttnParams {
   const int32_t *page_table;
   uint16_t *out;           // [n][hq][d] bf16
   float *lse;              // [hq][n] natural log, or null
-  float *part_o;           // [grid][2][kBM][d] fp32 (normalised partial outputs)
-  float *part_lse;         // [grid][2][kBM] fp32 (log2 domain)
+  float *part_o;           // [n_items][kBM][d] fp32 (normalised partial outputs)
+  float *part_lse;         // [n_items][kBM] fp32 (log2 domain)
   uint32_t *err;
   int64_t L;               // cached tokens before this call
-  int64_t total_iters;     // sum over units of key tiles
-  int64_t iters_per_head;
   int32_t n, hq, hkv, group, page_size, rows_cap, n_tiles, n_pages_valid, pool_pages;
-  int32_t grid;
+  int32_t chunk_tiles;     // key tiles per item
+  int32_t n_items;         // n_chunks * hkv * n_tiles, numbered (chunk, head, tile)
+  int32_t grid;            // CTAs; CTA c runs items c, c + grid, ...
   float scale_log2;        // softmax_scale * log2(e)
 };
 
@@ -60,8 +60,8 @@ struct MergeParams {
   const float *part_lse;
   uint16_t *out;
   float *lse;
-  int64_t L, total_iters, iters_per_head;
-  int32_t n, hq, hkv, group, n_tiles, grid, d;
+  int64_t L;
+  int32_t n, hq, hkv, group, n_tiles, chunk_tiles, d;
 };
 
 // K4: eviction / compaction: new version's page table from the free bitmap.

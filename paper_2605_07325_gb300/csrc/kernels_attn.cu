@@ -5,11 +5,14 @@
 // Work decomposition.  The rotated queries of one KV head are packed as rows
 // t*G + g (token t, group member g), so one 128-row tile holds 128/G tokens of
 // all G query heads that read the same keys.  A unit is one (kv head, query
-// tile); its key range is [0, L + last token of the tile], walked in tiles of
-// 128 keys.  The (unit, key tile) iteration space is cut into `grid` equal
-// contiguous ranges, one per CTA (stream-K): a CTA that holds a whole unit
-// writes its output directly, the pieces of a unit split between CTAs are
-// written as normalised partials with their log-sum-exp and merged by K3.
+// tile); its key range [0, L + last token of the tile] is cut into n_chunks
+// chunks of chunk_tiles 128-key tiles.  An item is one (key chunk, unit);
+// items are numbered chunk-major, (chunk, head, tile), and CTA c takes items
+// c, c + grid, c + 2 grid, ...  The CTAs running at the same time therefore
+// work on the same key chunk and read it through L2 instead of each
+// streaming the whole cache from HBM.  A unit that fits in one chunk is
+// written directly; otherwise each item writes a normalised partial output
+// with its log-sum-exp and K3 merges them.
 //
 // CTA roles (192 threads):
 //   warp 4 lane 0  TMA producer: the Q tile, then K and V tiles page by page
@@ -55,44 +58,43 @@ struct Bars {
   uint64_t o_done, o_final, o_free, drain;
   uint32_t tmem_base;
   int abort;
-  int32_t start_head, start_tile;
-  int64_t start_j;
 };
 
 size_t attn_smem_bytes(int head_dim) {
   return head_dim == 64 ? AttnCfg<64>::kSmem : AttnCfg<128>::kSmem;
 }
 
-// One contiguous run of key tiles of one unit inside a CTA's range.
+// One item: a run of key tiles [j0, j1) of one unit.
 struct Seg {
-  int32_t head, tile;
+  int32_t head, tile, item;
   int64_t j0, j1;
-  bool complete, first;
+  bool complete;
 };
 
-struct SegWalker {
-  int32_t head, tile;
-  int64_t j, g, g0, g1;
+// Walks the CTA's items (c, c + grid, ...); every role walks the same list.
+struct ItemWalker {
+  int32_t item;
   __device__ bool next(const AttnParams &p, int T, Seg &s) {
-    if (g >= g1) return false;
-    const int64_t it = unit_iters(p.L, p.n, T, tile);
-    const int64_t take = min(it - j, g1 - g);
-    s.head = head;
-    s.tile = tile;
-    s.j0 = j;
-    s.j1 = j + take;
-    s.complete = (j == 0 && take == it);
-    s.first = (g == g0);
-    g += take;
-    j += take;
-    if (j == it) {
-      j = 0;
-      if (++tile == p.n_tiles) {
-        tile = 0;
-        ++head;
-      }
+    const int32_t units = p.hkv * p.n_tiles;
+    while (item < p.n_items) {
+      const int32_t it = item;
+      item += p.grid;
+      const int32_t k = it / units;
+      const int32_t rem = it - k * units;
+      const int32_t head = rem / p.n_tiles;
+      const int32_t tile = rem - head * p.n_tiles;
+      const int64_t kv = unit_iters(p.L, p.n, T, tile);
+      const int64_t j0 = static_cast<int64_t>(k) * p.chunk_tiles;
+      if (j0 >= kv) continue;  // this unit has fewer chunks
+      s.head = head;
+      s.tile = tile;
+      s.item = it;
+      s.j0 = j0;
+      s.j1 = min(j0 + p.chunk_tiles, kv);
+      s.complete = kv <= p.chunk_tiles;
+      return true;
     }
-    return true;
+    return false;
   }
 };
 
@@ -107,6 +109,25 @@ __device__ __forceinline__ void drain_wait(uint64_t *bar, uint32_t parity) {
   while (!mbar_try_wait(bar, parity)) {
     if (globaltimer_ns() - t0 > 100ull * 1000ull * 1000ull) return;
   }
+}
+
+// O row *= alpha in place (one TMEM load and store of the thread's lane).
+template <int HD>
+__device__ __forceinline__ void rescale_o(uint32_t taddr, float alpha) {
+  uint32_t o[HD];
+  if constexpr (HD == 128) tmem_ld128_wait(taddr, o);
+  else tmem_ld64_wait(taddr, o);
+#pragma unroll
+  for (int c = 0; c < HD; ++c) o[c] = __float_as_uint(__uint_as_float(o[c]) * alpha);
+  if constexpr (HD == 128) tmem_st128(taddr, o);
+  else tmem_st64(taddr, o);
+  tmem_st_wait();
+}
+
+template <int HD>
+__device__ __forceinline__ void load_o(uint32_t taddr, uint32_t (&o)[HD]) {
+  if constexpr (HD == 128) tmem_ld128_wait(taddr, o);
+  else tmem_ld64_wait(taddr, o);
 }
 
 template <int HD>
@@ -139,9 +160,6 @@ __global__ void __launch_bounds__(192, 1) attn_kernel(const __grid_constant__ At
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   const int T = kBM / p.group;
-  const int64_t g0 = static_cast<int64_t>(blockIdx.x) * p.total_iters / p.grid;
-  const int64_t g1 = static_cast<int64_t>(blockIdx.x + 1) * p.total_iters / p.grid;
-
   if (threadIdx.x == 0) {
     mbar_init(&bars->q_full, 1);
     mbar_init(&bars->q_empty, 1);
@@ -163,42 +181,10 @@ __global__ void __launch_bounds__(192, 1) attn_kernel(const __grid_constant__ At
     bars->abort = 0;
     fence_barrier_init();
   }
-  if (warp == 4) {
-    // Locate the CTA's first iteration: head, query tile and key tile.
-    const int64_t head = g0 / p.iters_per_head;
-    const int64_t rem = g0 - head * p.iters_per_head;
-    const int per = (p.n_tiles + 31) / 32;
-    const int t_begin = min(lane * per, p.n_tiles);
-    const int t_end = min(t_begin + per, p.n_tiles);
-    int64_t mine = 0;
-    for (int t = t_begin; t < t_end; ++t) mine += unit_iters(p.L, p.n, T, t);
-    int64_t incl = mine;
-#pragma unroll
-    for (int off = 1; off < 32; off <<= 1) {
-      const int64_t y = __shfl_up_sync(0xffffffffu, incl, off);
-      if (lane >= off) incl += y;
-    }
-    const int64_t excl = incl - mine;
-    const unsigned owner_mask = __ballot_sync(0xffffffffu, excl <= rem && rem < incl);
-    const int owner = __ffs(owner_mask) - 1;
-    if (lane == owner) {
-      int64_t c = excl;
-      for (int t = t_begin; t < t_end; ++t) {
-        const int64_t it = unit_iters(p.L, p.n, T, t);
-        if (rem < c + it) {
-          bars->start_head = static_cast<int32_t>(head);
-          bars->start_tile = t;
-          bars->start_j = rem - c;
-          break;
-        }
-        c += it;
-      }
-    }
-    if (lane == 0) {
-      tma_prefetch_desc(&p.tm_q);
-      tma_prefetch_desc(&p.tm_k);
-      tma_prefetch_desc(&p.tm_v);
-    }
+  if (warp == 4 && lane == 0) {
+    tma_prefetch_desc(&p.tm_q);
+    tma_prefetch_desc(&p.tm_k);
+    tma_prefetch_desc(&p.tm_v);
   }
   if (warp == 5) {
     tmem_alloc(&bars->tmem_base, C::kTmemCols);
@@ -209,7 +195,7 @@ __global__ void __launch_bounds__(192, 1) attn_kernel(const __grid_constant__ At
   tc_fence_after();
   const uint32_t tmem = bars->tmem_base;
   volatile int *abort = &bars->abort;
-  SegWalker walk{bars->start_head, bars->start_tile, bars->start_j, g0, g0, g1};
+  ItemWalker walk{static_cast<int32_t>(blockIdx.x)};
   Seg seg;
 
   if (warp == 4) {
@@ -370,10 +356,7 @@ __global__ void __launch_bounds__(192, 1) attn_kernel(const __grid_constant__ At
         }
         tc_fence_after();
         uint32_t sr[kBN];
-#pragma unroll
-        for (int q4 = 0; q4 < kBN / 32; ++q4)
-          tmem_ld32_wait(tmem + lane_base + sb * kBN + q4 * 32,
-                         *reinterpret_cast<uint32_t(*)[32]>(&sr[q4 * 32]));
+        tmem_ld128_wait(tmem + lane_base + sb * kBN, sr);  // the whole score row, one wait
         float s[kBN];
 #pragma unroll
         for (int c = 0; c < kBN; ++c) s[c] = __uint_as_float(sr[c]);
@@ -383,15 +366,37 @@ __global__ void __launch_bounds__(192, 1) attn_kernel(const __grid_constant__ At
           for (int c = 0; c < kBN; ++c)
             if (key0 + c > limit) s[c] = -CUDART_INF_F;
         }
-        float mx = -CUDART_INF_F;
+        // row max as a tree over 8 independent partial maxima (no 128-long chain)
+        float mp[8];
 #pragma unroll
-        for (int c = 0; c < kBN; ++c) mx = fmaxf(mx, s[c]);
+        for (int e = 0; e < 8; ++e) mp[e] = s[e];
+#pragma unroll
+        for (int c = 8; c < kBN; ++c) mp[c & 7] = fmaxf(mp[c & 7], s[c]);
+        const float mx = fmaxf(fmaxf(fmaxf(mp[0], mp[1]), fmaxf(mp[2], mp[3])),
+                               fmaxf(fmaxf(mp[4], mp[5]), fmaxf(mp[6], mp[7])));
         const float mx_s = mx * p.scale_log2;
         const bool need = mx_s > m_ref + 8.0f;
         const float m_new = need ? mx_s : m_ref;
         const float alpha = need ? ex2_approx(m_ref - m_new) : 1.0f;
-        if (i > 0 && __any_sync(0xffffffffu, need && l > 0.f)) {
-          // O holds the sum up to the previous tile: rescale it once that PV landed.
+        const bool had_mass = l > 0.f;
+        l *= alpha;
+        m_ref = m_new;
+        const float m_use = (m_ref == -CUDART_INF_F) ? 0.f : m_ref;
+        float rp[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) rp[e] = 0.f;
+        uint32_t pk[kBN / 2];
+#pragma unroll
+        for (int c = 0; c < kBN; c += 2) {
+          const float p0 = ex2_approx(fmaf(s[c], p.scale_log2, -m_use));
+          const float p1 = ex2_approx(fmaf(s[c + 1], p.scale_log2, -m_use));
+          rp[(c >> 1) & 7] += p0 + p1;
+          pk[c / 2] = pack_bf16x2(p0, p1);
+        }
+        l += ((rp[0] + rp[1]) + (rp[2] + rp[3])) + ((rp[4] + rp[5]) + (rp[6] + rp[7]));
+        if (i > 0 && __any_sync(0xffffffffu, need && had_mass)) {
+          // O holds the sum up to the previous tile: rescale it once that PV
+          // landed, before this tile's P is published.
           const bool got_o = mbar_wait(&bars->o_done, (s_it - 1) & 1, abort, p.err,
                                        CSR_DEVERR_WAIT_TIMEOUT);
           if (!__all_sync(0xffffffffu, got_o)) {
@@ -399,31 +404,9 @@ __global__ void __launch_bounds__(192, 1) attn_kernel(const __grid_constant__ At
             break;
           }
           tc_fence_after();
-#pragma unroll
-          for (int q4 = 0; q4 < HD / 32; ++q4) {
-            uint32_t o[32];
-            tmem_ld32_wait(tmem + lane_base + C::kOCol + q4 * 32, o);
-#pragma unroll
-            for (int c = 0; c < 32; ++c) o[c] = __float_as_uint(__uint_as_float(o[c]) * alpha);
-            tmem_st32(tmem + lane_base + C::kOCol + q4 * 32, o);
-          }
-          tmem_st_wait();
+          rescale_o<HD>(tmem + lane_base + C::kOCol, alpha);
         }
-        l *= alpha;
-        m_ref = m_new;
-        const float m_use = (m_ref == -CUDART_INF_F) ? 0.f : m_ref;
-        float rs = 0.f;
-        uint32_t pk[kBN / 2];
-#pragma unroll
-        for (int c = 0; c < kBN; c += 2) {
-          const float p0 = ex2_approx(fmaf(s[c], p.scale_log2, -m_use));
-          const float p1 = ex2_approx(fmaf(s[c + 1], p.scale_log2, -m_use));
-          rs += p0 + p1;
-          pk[c / 2] = pack_bf16x2(p0, p1);
-        }
-        l += rs;
-        tmem_st32(tmem + lane_base + sb * kBN, *reinterpret_cast<uint32_t(*)[32]>(&pk[0]));
-        tmem_st32(tmem + lane_base + sb * kBN + 32, *reinterpret_cast<uint32_t(*)[32]>(&pk[32]));
+        tmem_st64(tmem + lane_base + sb * kBN, pk);
         tmem_st_wait();
         tc_fence_before();
         mbar_arrive(&bars->p_full[sb]);
@@ -441,39 +424,30 @@ __global__ void __launch_bounds__(192, 1) attn_kernel(const __grid_constant__ At
       tc_fence_after();
       const float inv_l = l > 0.f ? 1.0f / l : 0.f;
       const float lse2 = l > 0.f ? m_ref + log2f(l) : -CUDART_INF_F;
+      uint32_t o[HD];
+      load_o<HD>(tmem + lane_base + C::kOCol, o);
       if (seg.complete) {
         const int hq_idx = seg.head * p.group + row % p.group;
         uint16_t *dst = p.out + (static_cast<int64_t>(t) * p.hq + hq_idx) * HD;
+        if (valid) {
 #pragma unroll
-        for (int q4 = 0; q4 < HD / 32; ++q4) {
-          uint32_t o[32];
-          tmem_ld32_wait(tmem + lane_base + C::kOCol + q4 * 32, o);
-          if (valid) {
-            uint32_t w[16];
+          for (int q8 = 0; q8 < HD / 8; ++q8) {
+            uint32_t w[4];
 #pragma unroll
-            for (int c = 0; c < 16; ++c)
-              w[c] = pack_bf16x2(__uint_as_float(o[2 * c]) * inv_l,
-                                 __uint_as_float(o[2 * c + 1]) * inv_l);
-            uint4 *d4 = reinterpret_cast<uint4 *>(dst + q4 * 32);
-#pragma unroll
-            for (int c = 0; c < 4; ++c) d4[c] = make_uint4(w[4 * c], w[4 * c + 1], w[4 * c + 2], w[4 * c + 3]);
+            for (int c = 0; c < 4; ++c)
+              w[c] = pack_bf16x2(__uint_as_float(o[q8 * 8 + 2 * c]) * inv_l,
+                                 __uint_as_float(o[q8 * 8 + 2 * c + 1]) * inv_l);
+            reinterpret_cast<uint4 *>(dst)[q8] = make_uint4(w[0], w[1], w[2], w[3]);
           }
         }
         if (valid && p.lse) p.lse[static_cast<int64_t>(hq_idx) * p.n + t] = lse2 * 0.69314718055994531f;
       } else {
-        const int slot = seg.first ? 0 : 1;
-        const int64_t base = (static_cast<int64_t>(blockIdx.x) * 2 + slot) * kBM + row;
-        float *dst = p.part_o + base * HD;
+        const int64_t base = static_cast<int64_t>(seg.item) * kBM + row;
+        float4 *d4 = reinterpret_cast<float4 *>(p.part_o + base * HD);
 #pragma unroll
-        for (int q4 = 0; q4 < HD / 32; ++q4) {
-          uint32_t o[32];
-          tmem_ld32_wait(tmem + lane_base + C::kOCol + q4 * 32, o);
-          float4 *d4 = reinterpret_cast<float4 *>(dst + q4 * 32);
-#pragma unroll
-          for (int c = 0; c < 8; ++c)
-            d4[c] = make_float4(__uint_as_float(o[4 * c]) * inv_l, __uint_as_float(o[4 * c + 1]) * inv_l,
-                                __uint_as_float(o[4 * c + 2]) * inv_l, __uint_as_float(o[4 * c + 3]) * inv_l);
-        }
+        for (int c = 0; c < HD / 4; ++c)
+          d4[c] = make_float4(__uint_as_float(o[4 * c]) * inv_l, __uint_as_float(o[4 * c + 1]) * inv_l,
+                              __uint_as_float(o[4 * c + 2]) * inv_l, __uint_as_float(o[4 * c + 3]) * inv_l);
         p.part_lse[base] = lse2;
       }
       tc_fence_before();
@@ -492,77 +466,61 @@ __global__ void __launch_bounds__(192, 1) attn_kernel(const __grid_constant__ At
 }
 
 // ------------------------------------------------------------------ K3 merge
-__device__ __forceinline__ int64_t cta_start(int64_t c, int64_t total, int64_t grid) {
-  return c * total / grid;
-}
-__device__ __forceinline__ int64_t cta_of(int64_t g, int64_t total, int64_t grid) {
-  int64_t c = ((g + 1) * grid - 1) / total;
-  return c < grid - 1 ? c : grid - 1;
-}
-
-// Merge the split pieces of one unit: lse = log2 sum_s 2^lse_s,
-// O = sum_s 2^(lse_s - lse) O_s (each O_s already normalised by its own sum).
+// Merge the key-chunk pieces of one row: lse = log2 sum_k 2^lse_k and
+// O = sum_k 2^(lse_k - lse) O_k (each O_k already normalised by its own sum).
+// One warp per packed row; lanes own head_dim/32 output columns.
 template <int HD>
 __global__ void __launch_bounds__(256) merge_kernel(const __grid_constant__ MergeParams p) {
   const int u = blockIdx.x;
   const int head = u / p.n_tiles;
-  const int tile = u % p.n_tiles;
+  const int tile = u - head * p.n_tiles;
   const int T = kBM / p.group;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  __shared__ int64_t s_cum;
-  if (warp == 0) {
-    const int per = (tile + 31) / 32;
-    const int t_begin = min(lane * per, tile);
-    const int t_end = min(t_begin + per, tile);
-    int64_t mine = 0;
-    for (int t = t_begin; t < t_end; ++t) mine += unit_iters(p.L, p.n, T, t);
+  const int64_t kv = unit_iters(p.L, p.n, T, tile);
+  const int nk = static_cast<int>((kv + p.chunk_tiles - 1) / p.chunk_tiles);
+  if (nk <= 1) return;  // written whole by the attention kernel
+  const int r = blockIdx.y * 8 + warp;
+  const int64_t t = static_cast<int64_t>(tile) * T + r / p.group;
+  if (r >= kBM || t >= p.n) return;
+  const int units = p.hkv * p.n_tiles;
+  auto item_of = [&](int k) { return static_cast<int64_t>(k) * units + u; };
+  float mx = -CUDART_INF_F;
+  for (int k = lane; k < nk; k += 32) mx = fmaxf(mx, p.part_lse[item_of(k) * kBM + r]);
 #pragma unroll
-    for (int off = 16; off > 0; off >>= 1) mine += __shfl_xor_sync(0xffffffffu, mine, off);
-    if (lane == 0) s_cum = mine;
-  }
-  __syncthreads();
-  const int64_t us = static_cast<int64_t>(head) * p.iters_per_head + s_cum;
-  const int64_t ue = us + unit_iters(p.L, p.n, T, tile);
-  const int64_t c_first = cta_of(us, p.total_iters, p.grid);
-  const int64_t c_last = cta_of(ue - 1, p.total_iters, p.grid);
-  if (c_first == c_last) return;  // written whole by one CTA
-  constexpr int kPer = HD / 32;   // floats per lane
-  for (int r = warp; r < kBM; r += 8) {
-    const int64_t t = static_cast<int64_t>(tile) * T + r / p.group;
-    if (t >= p.n) continue;
-    float mx = -CUDART_INF_F;
-    for (int64_t c = c_first; c <= c_last; ++c) {
-      const int slot = cta_start(c, p.total_iters, p.grid) >= us ? 0 : 1;
-      mx = fmaxf(mx, p.part_lse[(c * 2 + slot) * kBM + r]);
-    }
-    float acc[kPer];
+  for (int off = 16; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
+  constexpr int kPer = HD / 32;  // floats per lane
+  float acc[kPer];
 #pragma unroll
-    for (int e = 0; e < kPer; ++e) acc[e] = 0.f;
-    float lse2 = -CUDART_INF_F;
-    if (mx != -CUDART_INF_F) {
-      float sum = 0.f;
-      for (int64_t c = c_first; c <= c_last; ++c) {
-        const int slot = cta_start(c, p.total_iters, p.grid) >= us ? 0 : 1;
-        sum += ex2_approx(p.part_lse[(c * 2 + slot) * kBM + r] - mx);
+  for (int e = 0; e < kPer; ++e) acc[e] = 0.f;
+  float lse2 = -CUDART_INF_F;
+  if (mx != -CUDART_INF_F) {
+    float sum = 0.f;
+    for (int k = lane; k < nk; k += 32) sum += ex2_approx(p.part_lse[item_of(k) * kBM + r] - mx);
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, off);
+    lse2 = mx + log2f(sum);
+    for (int k = 0; k < nk; ++k) {
+      const int64_t base = item_of(k) * kBM + r;
+      const float w = ex2_approx(p.part_lse[base] - lse2);
+      const float *src = p.part_o + base * HD + lane * kPer;
+      float v[kPer];
+#pragma unroll
+      for (int e = 0; e < kPer; e += 2) {
+        const float2 x = *reinterpret_cast<const float2 *>(src + e);
+        v[e] = x.x;
+        v[e + 1] = x.y;
       }
-      lse2 = mx + log2f(sum);
-      for (int64_t c = c_first; c <= c_last; ++c) {
-        const int slot = cta_start(c, p.total_iters, p.grid) >= us ? 0 : 1;
-        const int64_t base = (c * 2 + slot) * kBM + r;
-        const float w = ex2_approx(p.part_lse[base] - lse2);
-        const float *src = p.part_o + base * HD + lane * kPer;
 #pragma unroll
-        for (int e = 0; e < kPer; ++e) acc[e] = fmaf(w, src[e], acc[e]);
-      }
+      for (int e = 0; e < kPer; ++e) acc[e] = fmaf(w, v[e], acc[e]);
     }
-    const int hq_idx = head * p.group + r % p.group;
-    uint16_t *dst = p.out + (t * p.hq + hq_idx) * HD + lane * kPer;
-#pragma unroll
-    for (int e = 0; e < kPer; e += 2) {
-      *reinterpret_cast<uint32_t *>(dst + e) = pack_bf16x2(acc[e], acc[e + 1]);
-    }
-    if (lane == 0 && p.lse) p.lse[static_cast<int64_t>(hq_idx) * p.n + t] = lse2 * 0.69314718055994531f;
   }
+  const int hq_idx = head * p.group + r % p.group;
+  uint16_t *dst = p.out + (t * p.hq + hq_idx) * HD + lane * kPer;
+#pragma unroll
+  for (int e = 0; e < kPer; e += 2) {
+    *reinterpret_cast<uint32_t *>(dst + e) = pack_bf16x2(acc[e], acc[e + 1]);
+  }
+  if (lane == 0 && p.lse) p.lse[static_cast<int64_t>(hq_idx) * p.n + t] = lse2 * 0.69314718055994531f;
 }
 
 cudaError_t attn_configure(int head_dim) {
@@ -582,11 +540,11 @@ cudaError_t launch_attention(const AttnParams &p, int head_dim, cudaStream_t s) 
 }
 
 cudaError_t launch_merge(const MergeParams &p, cudaStream_t s) {
-  const int units = p.hkv * p.n_tiles;
+  const dim3 grid(p.hkv * p.n_tiles, kBM / 8);
   if (p.d == 64)
-    merge_kernel<64><<<units, 256, 0, s>>>(p);
+    merge_kernel<64><<<grid, 256, 0, s>>>(p);
   else
-    merge_kernel<128><<<units, 256, 0, s>>>(p);
+    merge_kernel<128><<<grid, 256, 0, s>>>(p);
   return cudaGetLastError();
 }
 

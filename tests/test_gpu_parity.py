@@ -19,7 +19,7 @@ pytestmark = pytest.mark.gpu
 def test_tiny_config_full_session(libcsr):
     """8 q heads / 2 kv heads, d=64, page 16, base 1e4: 256-token prefix,
     3 chunks of 256, a 32-token suffix, truncate, one more chunk, suffix again."""
-    p = Pair(C1, pool_pages=256, max_seq=4096, max_new=512)
+    p = Pair(C1, pool_pages=256, max_seq=4096, max_new=512, fg_chunk_tiles=3)
     p.init_static(p.blk(0, 256))
     for i in range(3):
         p.append(p.blk(1 + i, 256))
@@ -49,8 +49,9 @@ def test_single_token_prefix_returns_v(libcsr):
 
 
 @pytest.mark.parametrize("shape", [C1, C2], ids=["d64_p16_g4", "d128_p64_g16"])
-def test_ragged_sizes(libcsr, shape):
-    p = Pair(shape, pool_pages=128, max_seq=4096, max_new=512)
+@pytest.mark.parametrize("chunk_tiles", [0, 2])
+def test_ragged_sizes(libcsr, shape, chunk_tiles):
+    p = Pair(shape, pool_pages=128, max_seq=4096, max_new=512, fg_chunk_tiles=chunk_tiles)
     p.init_static(p.blk(10, 37))
     for i, n in enumerate([1, 129, 64, 300, 17]):
         p.append(p.blk(11 + i, n))
@@ -64,11 +65,13 @@ def test_ragged_sizes(libcsr, shape):
     p.device_clean()
 
 
-@pytest.mark.parametrize("num_ctas", [1, 2, 3, 7, 19, 64])
-def test_split_kv_partials_any_grid(libcsr, num_ctas):
-    """Forced CTA counts cut units at arbitrary key tiles: every split must
-    merge back to the oracle."""
-    p = Pair(C2, pool_pages=256, max_seq=8192, max_new=1024, num_ctas=num_ctas)
+@pytest.mark.parametrize("num_ctas,chunk_tiles", [(1, 0), (3, 1), (7, 2), (19, 3), (64, 5),
+                                                   (152, 1), (0, 4)])
+def test_split_kv_partials_any_grid(libcsr, num_ctas, chunk_tiles):
+    """Forced CTA counts and key-chunk lengths: every split into items (down to
+    one 128-key tile per item) must merge back to the oracle."""
+    p = Pair(C2, pool_pages=256, max_seq=8192, max_new=1024, num_ctas=num_ctas,
+             fg_chunk_tiles=chunk_tiles)
     p.init_static(p.blk(30, 700))
     p.append(p.blk(31, 1000))
     p.append(p.blk(32, 33))

@@ -42,7 +42,8 @@ def _fresh_copy(p: Pair, prefix_block, chunk_ids):
 ])
 def test_evict_reconcile_swap(libcsr, shape, prefix, chunk, evict, n_catchup):
     csr = csr_mod()
-    p = Pair(shape, pool_pages=256, max_seq=8192, max_new=512, n_catchup=n_catchup)
+    p = Pair(shape, pool_pages=256, max_seq=8192, max_new=512, n_catchup=n_catchup,
+             rebuild_tiles_per_cta=2)   # short rebuild items: exercises the split merge
     lo = torch.cuda.Stream(priority=0)
     outs = {}
     p.ctx.set_reconciler(_provider(p, outs), lo)
