@@ -46,7 +46,9 @@ struct AttnCfg {
   static constexpr int kKOff = kQOff + kQBytes;
   static constexpr int kVOff = kKOff + kStages * kTileBytes;
   static constexpr int kBarOff = kVOff + kStages * kTileBytes;
-  static constexpr int kSmem = kBarOff + 1024 + 1024;    // barriers + alignment slack
+  static constexpr int kPtOff = kBarOff + 1024;          // staged page ids
+  static constexpr int kPtStage = 512;                   // entries per staging block
+  static constexpr int kSmem = kPtOff + kPtStage * 4 + 1024;  // + alignment slack
   static constexpr uint32_t kTmemCols = 512;
   static constexpr uint32_t kOCol = 2 * kBN;             // O accumulator after two S buffers
 };
@@ -130,20 +132,16 @@ __device__ __forceinline__ void load_o(uint32_t taddr, uint32_t (&o)[HD]) {
   else tmem_ld64_wait(taddr, o);
 }
 
+// Issue the TMA loads of one 128-key tile of `head` whose pages' physical ids
+// are phys[0 .. 128/P).
 template <int HD>
 __device__ __forceinline__ void load_kv_tile(const AttnParams &p, const CUtensorMap *map,
-                                             uint8_t *dst, uint64_t *bar, int head, int64_t j) {
+                                             uint8_t *dst, uint64_t *bar, int head,
+                                             const int32_t *phys) {
   const int P = p.page_size;
   const int ppt = kBN / P;
-  const int64_t lp0 = j * kBN / P;
   for (int pp = 0; pp < ppt; ++pp) {
-    const int64_t lp = lp0 + pp;
-    int32_t phys = (lp < p.n_pages_valid) ? p.page_table[lp] : p.page_table[0];
-    if (phys < 0 || phys >= p.pool_pages) {
-      atomicOr(p.err, CSR_DEVERR_BAD_PAGE);
-      phys = 0;
-    }
-    const int32_t row = (phys * p.hkv + head) * P;
+    const int32_t row = (phys[pp] * p.hkv + head) * P;
 #pragma unroll
     for (int b = 0; b < AttnCfg<HD>::kBoxes; ++b)
       tma_load_2d(dst + b * (kBN * 128) + pp * P * 128, map, bar, b * 64, row);
@@ -199,53 +197,79 @@ __global__ void __launch_bounds__(192, 1) attn_kernel(const __grid_constant__ At
   Seg seg;
 
   if (warp == 4) {
-    if (lane == 0) {
-      // ------------------------------------------------------ TMA producer
-      uint32_t q_round = 0, k_it = 0, v_it = 0;
-      bool ok = true;
-      while (ok && walk.next(p, T, seg)) {
+    // ------------------------------------------------------ TMA producer
+    // The whole warp stages the page ids of the next tiles into shared memory
+    // (coalesced page-table reads off the critical path); lane 0 issues the
+    // copies from there.
+    int32_t *stage = reinterpret_cast<int32_t *>(smem + C::kPtOff);
+    const int ppt = kBN / p.page_size;
+    const int tiles_per_block = C::kPtStage / ppt;
+    uint32_t q_round = 0, k_it = 0, v_it = 0;
+    bool ok = true;
+    while (ok && walk.next(p, T, seg)) {
+      if (lane == 0) {
         if (q_round > 0 && !mbar_wait(&bars->q_empty, (q_round - 1) & 1, abort, p.err,
                                       CSR_DEVERR_WAIT_TIMEOUT)) {
           ok = false;
-          break;
-        }
-        mbar_arrive_expect_tx(&bars->q_full, C::kQBytes);
-        const int32_t qrow = seg.head * p.rows_cap + seg.tile * kBM;
+        } else {
+          mbar_arrive_expect_tx(&bars->q_full, C::kQBytes);
+          const int32_t qrow = seg.head * p.rows_cap + seg.tile * kBM;
 #pragma unroll
-        for (int b = 0; b < C::kBoxes; ++b)
-          tma_load_2d(smem + C::kQOff + b * (kBM * 128), &p.tm_q, &bars->q_full, b * 64, qrow);
-        ++q_round;
-        for (int64_t j = seg.j0; j < seg.j1; ++j) {
-          const int ks = k_it % C::kStages;
-          if (!mbar_wait(&bars->k_empty[ks], ((k_it / C::kStages) & 1) ^ 1, abort, p.err,
-                         CSR_DEVERR_WAIT_TIMEOUT)) {
-            ok = false;
-            break;
-          }
-          mbar_arrive_expect_tx(&bars->k_full[ks], C::kTileBytes);
-          load_kv_tile<HD>(p, &p.tm_k, smem + C::kKOff + ks * C::kTileBytes, &bars->k_full[ks],
-                           seg.head, j);
-          ++k_it;
-          const int vs = v_it % C::kStages;
-          if (!mbar_wait(&bars->v_empty[vs], ((v_it / C::kStages) & 1) ^ 1, abort, p.err,
-                         CSR_DEVERR_WAIT_TIMEOUT)) {
-            ok = false;
-            break;
-          }
-          mbar_arrive_expect_tx(&bars->v_full[vs], C::kTileBytes);
-          load_kv_tile<HD>(p, &p.tm_v, smem + C::kVOff + vs * C::kTileBytes, &bars->v_full[vs],
-                           seg.head, j);
-          ++v_it;
+          for (int b = 0; b < C::kBoxes; ++b)
+            tma_load_2d(smem + C::kQOff + b * (kBM * 128), &p.tm_q, &bars->q_full, b * 64, qrow);
+          ++q_round;
         }
       }
-      if (!ok) {
-        // Let the copies already issued land before the CTA's memory goes away.
-        if (q_round > 0) drain_wait(&bars->q_full, (q_round - 1) & 1);
-        for (uint32_t i = (k_it > C::kStages ? k_it - C::kStages : 0); i < k_it; ++i)
-          drain_wait(&bars->k_full[i % C::kStages], (i / C::kStages) & 1);
-        for (uint32_t i = (v_it > C::kStages ? v_it - C::kStages : 0); i < v_it; ++i)
-          drain_wait(&bars->v_full[i % C::kStages], (i / C::kStages) & 1);
+      ok = __shfl_sync(0xffffffffu, ok, 0);
+      for (int64_t jb = seg.j0; ok && jb < seg.j1; jb += tiles_per_block) {
+        const int64_t je = min(jb + tiles_per_block, seg.j1);
+        const int npages = static_cast<int>(je - jb) * ppt;
+        __syncwarp();
+        for (int i = lane; i < npages; i += 32) {
+          const int64_t lp = jb * ppt + i;
+          int32_t phys = (lp < p.n_pages_valid) ? p.page_table[lp] : p.page_table[0];
+          if (phys < 0 || phys >= p.pool_pages) {
+            atomicOr(p.err, CSR_DEVERR_BAD_PAGE);
+            phys = 0;
+          }
+          stage[i] = phys;
+        }
+        __syncwarp();
+        if (lane == 0) {
+          for (int64_t j = jb; j < je; ++j) {
+            const int32_t *phys = stage + static_cast<int>(j - jb) * ppt;
+            const int ks = k_it % C::kStages;
+            if (!mbar_wait(&bars->k_empty[ks], ((k_it / C::kStages) & 1) ^ 1, abort, p.err,
+                           CSR_DEVERR_WAIT_TIMEOUT)) {
+              ok = false;
+              break;
+            }
+            mbar_arrive_expect_tx(&bars->k_full[ks], C::kTileBytes);
+            load_kv_tile<HD>(p, &p.tm_k, smem + C::kKOff + ks * C::kTileBytes, &bars->k_full[ks],
+                             seg.head, phys);
+            ++k_it;
+            const int vs = v_it % C::kStages;
+            if (!mbar_wait(&bars->v_empty[vs], ((v_it / C::kStages) & 1) ^ 1, abort, p.err,
+                           CSR_DEVERR_WAIT_TIMEOUT)) {
+              ok = false;
+              break;
+            }
+            mbar_arrive_expect_tx(&bars->v_full[vs], C::kTileBytes);
+            load_kv_tile<HD>(p, &p.tm_v, smem + C::kVOff + vs * C::kTileBytes, &bars->v_full[vs],
+                             seg.head, phys);
+            ++v_it;
+          }
+        }
+        ok = __shfl_sync(0xffffffffu, ok, 0);
       }
+    }
+    if (!ok && lane == 0) {
+      // Let the copies already issued land before the CTA's memory goes away.
+      if (q_round > 0) drain_wait(&bars->q_full, (q_round - 1) & 1);
+      for (uint32_t i = (k_it > C::kStages ? k_it - C::kStages : 0); i < k_it; ++i)
+        drain_wait(&bars->k_full[i % C::kStages], (i / C::kStages) & 1);
+      for (uint32_t i = (v_it > C::kStages ? v_it - C::kStages : 0); i < v_it; ++i)
+        drain_wait(&bars->v_full[i % C::kStages], (i / C::kStages) & 1);
     }
   } else if (warp == 5) {
     if (lane == 0) {
