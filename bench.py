@@ -232,7 +232,8 @@ def run_ours(args):
     max_tokens = L0 + CHUNK + SUFFIX
     pool_pages = math.ceil(max_tokens / P) + 16
     cfg = csr.make_config(HQ, HKV, D, P, BASE, max_new_tokens=PREFIX, pool_pages=pool_pages,
-                          max_seq_tokens=max_tokens + P)
+                          max_seq_tokens=max_tokens + P,
+                          flags=csr.FLAG_SINGLE_TILE if args.single_tile else 0)
     stream = torch.cuda.Stream(device=dev, priority=-1)
     gen = torch.Generator(device=dev).manual_seed(1234 + rank)
 
@@ -367,7 +368,8 @@ def run_ours(args):
         "roofline": {"bound": "tensor", "achieved": achieved, "peak": peak_burst, "unit": "TFLOP/s",
                      "frac": (achieved / peak_burst) if achieved else None,
                      "traffic": (traffic_step / 2) if traffic_step else None,
-                     "kernel": "attn_kernel<128> (tcgen05 QK^T and PV, TMA paged K/V)",
+                     "kernel": ("attn_kernel<128>" if args.single_tile else "attn_pair_kernel<128>") +
+                               " (tcgen05 QK^T and PV, TMA paged K/V)",
                      "launches": att_n, "avg_launch_us": att_ms / max(1, att_n) * 1e3,
                      "peak_source": f"bf16_tflops ({peak_kind}, burst)",
                      "frac_of_sustained": (achieved / peak_sust) if achieved else None},
@@ -398,6 +400,8 @@ def main(argv=None):
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--single-tile", action="store_true",
+                    help="attention CTAs own one query tile (the earlier kernel design)")
     ap.add_argument("--fill-chunk", type=int, default=CHUNK, choices=[256, 512, 1024, 2048, 4096],
                     help="chunk size used to fill the cache before timing (fewer launches "
                          "for profiler captures); the timed steps are unchanged")

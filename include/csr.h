@@ -69,9 +69,11 @@ typedef enum csr_status {
 #define CSR_DEVERR_ALLOC 0x4u        /* the compaction kernel found too few free pages */
 
 /* csr_config.flags */
-#define CSR_FLAG_PLAN_ONLY 0x1 /* layout planning only: no device memory is touched
-                                  and no kernel runs; compute calls update the page
-                                  tables and lengths but produce no outputs */
+#define CSR_FLAG_PLAN_ONLY 0x1   /* layout planning only: no device memory is touched
+                                    and no kernel runs; compute calls update the page
+                                    tables and lengths but produce no outputs */
+#define CSR_FLAG_SINGLE_TILE 0x2 /* attention CTAs own one 128-row query tile instead of
+                                    two (the earlier kernel design, kept for comparison) */
 
 typedef struct csr_config {
   int32_t num_q_heads;    /* H_q */

@@ -161,7 +161,8 @@ bool valid_config(const csr_config *c, std::string *why) {
 Layout make_layout(const csr_config *c) {
   Layout L{};
   const int g = c->num_q_heads / c->num_kv_heads;
-  L.rows_cap = static_cast<int32_t>(align_up(static_cast<size_t>(c->max_new_tokens) * g, kBM));
+  // whole pairs of 128-row tiles, so the two-tile kernel never reads past a head's rows
+  L.rows_cap = static_cast<int32_t>(align_up(static_cast<size_t>(c->max_new_tokens) * g, 2 * kBM));
   L.fg_cap = c->num_ctas > 0 ? c->num_ctas : kFgGridDefaultCap;
   L.max_pages = static_cast<int32_t>(ceil_div(c->max_seq_tokens, c->page_size) + 1);
   const size_t d = static_cast<size_t>(c->head_dim);
@@ -249,15 +250,18 @@ int64_t pages_for(const csr_ctx *c, int64_t len) { return ceil_div(len, c->cfg.p
 // launch waits at most one item for an SM.  Never more than kPartialItems
 // items when split.
 int32_t choose_chunk_tiles(int64_t units, int64_t kv_max, int64_t grid, int max_tiles,
-                           int head_dim) {
-  const double t_tile = 0.75, t_item = 2.0, t_part = head_dim == 128 ? 0.02 : 0.01;  // us
+                           int head_dim, int unit_tiles) {
+  // us per key tile per CTA, per item, per split partial (rough GB300 figures)
+  const double t_tile = 0.75 * unit_tiles, t_item = 2.0;
+  const double t_part = (head_dim == 128 ? 0.02 : 0.01) * unit_tiles;
+  const int64_t cap_items = kPartialItems / unit_tiles;
   int64_t best_c = kv_max;
   double best_t = 1e300;
   for (int64_t S = 1; S <= std::min<int64_t>(kv_max, 256); ++S) {
     const int64_t C = ceil_div(kv_max, S);
     const int64_t Se = ceil_div(kv_max, C);
     const int64_t items = units * Se;
-    if (Se > 1 && items > kPartialItems) break;
+    if (Se > 1 && items > cap_items) break;
     if (max_tiles > 0) {
       if (C <= max_tiles) return static_cast<int32_t>(C);
       best_c = C;  // the smallest chunk that still fits the partial buffer
@@ -355,15 +359,19 @@ csr_status run_block(csr_ctx *c, int slot, int ws, const void *q, const void *k,
   ap.n_pages_valid = static_cast<int32_t>(pages_for(c, L + n));
   ap.pool_pages = cf.pool_pages;
   const int T = kBM / c->group;
-  const int64_t units = static_cast<int64_t>(ap.n_tiles) * cf.num_kv_heads;
-  const int64_t kv_max = unit_iters(L, n, T, ap.n_tiles - 1);
+  ap.unit_tiles = (cf.flags & CSR_FLAG_SINGLE_TILE) ? 1 : 2;
+  const int64_t uph = ceil_div(ap.n_tiles, ap.unit_tiles);
+  const int64_t units = uph * cf.num_kv_heads;
+  const int64_t kv_max = unit_iters(L, n, T, static_cast<int32_t>(uph * ap.unit_tiles - 1));
   const int tpc = cf.rebuild_tiles_per_cta > 0 ? cf.rebuild_tiles_per_cta : kDefaultRebuildTiles;
   if (ws == 0 && cf.fg_chunk_tiles > 0) {
     // fixed chunk length, but never more split items than the partial buffer holds
-    const int64_t min_c = ceil_div(kv_max, std::max<int64_t>(1, kPartialItems / units));
+    const int64_t cap_units = std::max<int64_t>(1, kPartialItems / ap.unit_tiles / units);
+    const int64_t min_c = ceil_div(kv_max, cap_units);
     ap.chunk_tiles = static_cast<int32_t>(std::max<int64_t>(cf.fg_chunk_tiles, min_c));
   } else {
-    ap.chunk_tiles = choose_chunk_tiles(units, kv_max, c->fg_grid, ws == 0 ? 0 : tpc, cf.head_dim);
+    ap.chunk_tiles = choose_chunk_tiles(units, kv_max, c->fg_grid, ws == 0 ? 0 : tpc, cf.head_dim,
+                                        ap.unit_tiles);
   }
   const int64_t n_chunks = ceil_div(kv_max, ap.chunk_tiles);
   ap.n_items = static_cast<int32_t>(n_chunks * units);
@@ -386,6 +394,7 @@ csr_status run_block(csr_ctx *c, int slot, int ws, const void *q, const void *k,
     mp.group = ap.group;
     mp.n_tiles = ap.n_tiles;
     mp.chunk_tiles = ap.chunk_tiles;
+    mp.unit_tiles = ap.unit_tiles;
     mp.d = cf.head_dim;
     e = timed_launch(c, CSR_KERNEL_MERGE, fg, s, [&] { return launch_merge(mp, s); });
     if (e != cudaSuccess) return cuda_fail(c, e, "merge launch");

@@ -49,7 +49,8 @@ struct AttnParams {
   int64_t L;               // cached tokens before this call
   int32_t n, hq, hkv, group, page_size, rows_cap, n_tiles, n_pages_valid, pool_pages;
   int32_t chunk_tiles;     // key tiles per item
-  int32_t n_items;         // n_chunks * hkv * n_tiles, numbered (chunk, head, tile)
+  int32_t unit_tiles;      // query tiles per item: 1 (attn_kernel) or 2 (attn_pair_kernel)
+  int32_t n_items;         // n_chunks * hkv * units per head, numbered (chunk, head, unit)
   int32_t grid;            // CTAs; CTA c runs items c, c + grid, ...
   float scale_log2;        // softmax_scale * log2(e)
 };
@@ -61,7 +62,7 @@ struct MergeParams {
   uint16_t *out;
   float *lse;
   int64_t L;
-  int32_t n, hq, hkv, group, n_tiles, chunk_tiles, d;
+  int32_t n, hq, hkv, group, n_tiles, chunk_tiles, unit_tiles, d;
 };
 
 // K4: eviction / compaction: new version's page table from the free bitmap.
@@ -92,8 +93,9 @@ struct GatherParams {
   int32_t n, hkv, d, page_size, pool_pages;
 };
 
-// Shared-memory bytes of the attention kernel for a head dim.
+// Shared-memory bytes of the attention kernels for a head dim.
 size_t attn_smem_bytes(int head_dim);
+size_t attn_pair_smem_bytes(int head_dim);
 
 // Key tiles of query tile `tile` (kBN keys each).
 __host__ __device__ inline int64_t unit_iters(int64_t L, int32_t n, int32_t tokens_per_tile,

@@ -489,27 +489,442 @@ __global__ void __launch_bounds__(192, 1) attn_kernel(const __grid_constant__ At
   }
 }
 
+// ============================================================ two-tile kernel
+// Same work as attn_kernel, but one CTA owns two consecutive 128-row query
+// tiles (A, B) of a KV head: every K/V tile staged in shared memory feeds both,
+// halving the load traffic per FLOP, and two softmax warpgroups alternate with
+// the tensor core.  MMA issue order per key tile i (one thread):
+//   PV_A(i), S_A(i+1), PV_B(i), S_B(i+1)
+// so the commit that publishes S_X(i+1) also covers PV_X(i): a softmax
+// warpgroup that sees its next scores may rescale its O without another wait.
+// TMEM: S_A [0,128), S_B [128,256), O_A [256,256+d), O_B [256+d,256+2d).
+// 320 threads: warps 0-3 softmax A, warps 4-7 softmax B, warp 8 TMA producer,
+// warp 9 MMA issuer.
+template <int HD>
+struct PairCfg {
+  static constexpr int kStages = (HD == 64) ? 4 : 2;
+  static constexpr int kBoxes = HD / 64;
+  static constexpr int kQBytes = kBM * HD * 2;                 // one query tile
+  static constexpr int kTileBytes = kBN * HD * 2;
+  static constexpr int kQOff = 0;                              // Q_A, then Q_B
+  static constexpr int kKOff = 2 * kQBytes;
+  static constexpr int kVOff = kKOff + kStages * kTileBytes;
+  static constexpr int kBarOff = kVOff + kStages * kTileBytes;
+  static constexpr int kPtOff = kBarOff + 1024;
+  static constexpr int kPtStage = 512;
+  static constexpr int kSmem = kPtOff + kPtStage * 4 + 1024;
+  static constexpr uint32_t kTmemCols = 512;
+  static constexpr uint32_t kOCol = 2 * kBN;                   // O_A; O_B at kOCol + HD
+};
+
+struct PairBars {
+  uint64_t q_full, q_empty;
+  uint64_t k_full[4], k_empty[4], v_full[4], v_empty[4];
+  uint64_t s_full[2], p_full[2], o_final[2], o_free[2];
+  uint64_t drain;
+  uint32_t tmem_base;
+  int abort;
+};
+
+size_t attn_pair_smem_bytes(int head_dim) {
+  return head_dim == 64 ? PairCfg<64>::kSmem : PairCfg<128>::kSmem;
+}
+
+// Items of the two-tile kernel: (chunk, head, pair); the pair's key range is
+// that of its second tile.
+struct PairWalker {
+  int32_t item;
+  __device__ bool next(const AttnParams &p, int T, Seg &s) {
+    const int32_t n_pairs = (p.n_tiles + 1) / 2;
+    const int32_t units = p.hkv * n_pairs;
+    while (item < p.n_items) {
+      const int32_t it = item;
+      item += p.grid;
+      const int32_t k = it / units;
+      const int32_t rem = it - k * units;
+      const int32_t head = rem / n_pairs;
+      const int32_t pair = rem - head * n_pairs;
+      const int64_t kv = unit_iters(p.L, p.n, T, 2 * pair + 1);
+      const int64_t j0 = static_cast<int64_t>(k) * p.chunk_tiles;
+      if (j0 >= kv) continue;
+      s.head = head;
+      s.tile = pair;  // pair index
+      s.item = it;
+      s.j0 = j0;
+      s.j1 = min(j0 + p.chunk_tiles, kv);
+      s.complete = kv <= p.chunk_tiles;
+      return true;
+    }
+    return false;
+  }
+};
+
+template <int HD>
+__global__ void __launch_bounds__(320, 1) attn_pair_kernel(const __grid_constant__ AttnParams p) {
+  using C = PairCfg<HD>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t *smem = reinterpret_cast<uint8_t *>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  PairBars *bars = reinterpret_cast<PairBars *>(smem + C::kBarOff);
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const int T = kBM / p.group;
+
+  if (threadIdx.x == 0) {
+    mbar_init(&bars->q_full, 1);
+    mbar_init(&bars->q_empty, 1);
+    for (int s = 0; s < C::kStages; ++s) {
+      mbar_init(&bars->k_full[s], 1);
+      mbar_init(&bars->k_empty[s], 1);
+      mbar_init(&bars->v_full[s], 1);
+      mbar_init(&bars->v_empty[s], 1);
+    }
+    for (int w = 0; w < 2; ++w) {
+      mbar_init(&bars->s_full[w], 1);
+      mbar_init(&bars->p_full[w], 128);
+      mbar_init(&bars->o_final[w], 1);
+      mbar_init(&bars->o_free[w], 128);
+    }
+    mbar_init(&bars->drain, 1);
+    bars->abort = 0;
+    fence_barrier_init();
+  }
+  if (warp == 8 && lane == 0) {
+    tma_prefetch_desc(&p.tm_q);
+    tma_prefetch_desc(&p.tm_k);
+    tma_prefetch_desc(&p.tm_v);
+  }
+  if (warp == 9) {
+    tmem_alloc(&bars->tmem_base, C::kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = bars->tmem_base;
+  volatile int *abort = &bars->abort;
+  PairWalker walk{static_cast<int32_t>(blockIdx.x)};
+  Seg seg;
+
+  if (warp == 8) {
+    // ------------------------------------------------------ TMA producer
+    int32_t *stage = reinterpret_cast<int32_t *>(smem + C::kPtOff);
+    const int ppt = kBN / p.page_size;
+    const int tiles_per_block = C::kPtStage / ppt;
+    uint32_t q_round = 0, k_it = 0, v_it = 0;
+    bool ok = true;
+    while (ok && walk.next(p, T, seg)) {
+      if (lane == 0) {
+        if (q_round > 0 && !mbar_wait(&bars->q_empty, (q_round - 1) & 1, abort, p.err,
+                                      CSR_DEVERR_WAIT_TIMEOUT)) {
+          ok = false;
+        } else {
+          mbar_arrive_expect_tx(&bars->q_full, 2 * C::kQBytes);
+          const int32_t qrow = seg.head * p.rows_cap + seg.tile * 2 * kBM;
+#pragma unroll
+          for (int h = 0; h < 2; ++h)
+#pragma unroll
+            for (int b = 0; b < C::kBoxes; ++b)
+              tma_load_2d(smem + C::kQOff + h * C::kQBytes + b * (kBM * 128), &p.tm_q,
+                          &bars->q_full, b * 64, qrow + h * kBM);
+          ++q_round;
+        }
+      }
+      ok = __shfl_sync(0xffffffffu, ok, 0);
+      for (int64_t jb = seg.j0; ok && jb < seg.j1; jb += tiles_per_block) {
+        const int64_t je = min(jb + tiles_per_block, seg.j1);
+        const int npages = static_cast<int>(je - jb) * ppt;
+        __syncwarp();
+        for (int i = lane; i < npages; i += 32) {
+          const int64_t lp = jb * ppt + i;
+          int32_t phys = (lp < p.n_pages_valid) ? p.page_table[lp] : p.page_table[0];
+          if (phys < 0 || phys >= p.pool_pages) {
+            atomicOr(p.err, CSR_DEVERR_BAD_PAGE);
+            phys = 0;
+          }
+          stage[i] = phys;
+        }
+        __syncwarp();
+        if (lane == 0) {
+          for (int64_t j = jb; j < je; ++j) {
+            const int32_t *phys = stage + static_cast<int>(j - jb) * ppt;
+            const int ks = k_it % C::kStages;
+            if (!mbar_wait(&bars->k_empty[ks], ((k_it / C::kStages) & 1) ^ 1, abort, p.err,
+                           CSR_DEVERR_WAIT_TIMEOUT)) {
+              ok = false;
+              break;
+            }
+            mbar_arrive_expect_tx(&bars->k_full[ks], C::kTileBytes);
+            load_kv_tile<HD>(p, &p.tm_k, smem + C::kKOff + ks * C::kTileBytes, &bars->k_full[ks],
+                             seg.head, phys);
+            ++k_it;
+            const int vs = v_it % C::kStages;
+            if (!mbar_wait(&bars->v_empty[vs], ((v_it / C::kStages) & 1) ^ 1, abort, p.err,
+                           CSR_DEVERR_WAIT_TIMEOUT)) {
+              ok = false;
+              break;
+            }
+            mbar_arrive_expect_tx(&bars->v_full[vs], C::kTileBytes);
+            load_kv_tile<HD>(p, &p.tm_v, smem + C::kVOff + vs * C::kTileBytes, &bars->v_full[vs],
+                             seg.head, phys);
+            ++v_it;
+          }
+        }
+        ok = __shfl_sync(0xffffffffu, ok, 0);
+      }
+    }
+    if (!ok && lane == 0) {
+      if (q_round > 0) drain_wait(&bars->q_full, (q_round - 1) & 1);
+      for (uint32_t i = (k_it > C::kStages ? k_it - C::kStages : 0); i < k_it; ++i)
+        drain_wait(&bars->k_full[i % C::kStages], (i / C::kStages) & 1);
+      for (uint32_t i = (v_it > C::kStages ? v_it - C::kStages : 0); i < v_it; ++i)
+        drain_wait(&bars->v_full[i % C::kStages], (i / C::kStages) & 1);
+    }
+  } else if (warp == 9) {
+    if (lane == 0) {
+      // ------------------------------------------------------ MMA issuer
+      constexpr uint32_t idesc_s = idesc_bf16_f32(kBM, kBN, false, false);
+      constexpr uint32_t idesc_pv = idesc_bf16_f32(kBM, HD, false, true);
+      const uint32_t q_base = smem_u32(smem + C::kQOff);
+      const uint32_t k_base = smem_u32(smem + C::kKOff);
+      const uint32_t v_base = smem_u32(smem + C::kVOff);
+      uint32_t q_round = 0, k_it = 0, v_it = 0, seg_n = 0;
+      uint32_t pv_n[2] = {0, 0};
+      bool ok = true;
+      auto wait = [&](uint64_t *bar, uint32_t parity) {
+        if (ok && !mbar_wait(bar, parity, abort, p.err, CSR_DEVERR_WAIT_TIMEOUT)) ok = false;
+        return ok;
+      };
+      // S_X = Q_X K^T for tile x from K stage ks
+      auto issue_s = [&](int x, int ks) {
+        const uint32_t qx = q_base + x * C::kQBytes;
+        const uint32_t kst = k_base + ks * C::kTileBytes;
+#pragma unroll
+        for (int kk = 0; kk < HD / 16; ++kk) {
+          const uint64_t a = sdesc_sw128(qx + (kk >> 2) * (kBM * 128) + (kk & 3) * 32, 16, 1024);
+          const uint64_t b = sdesc_sw128(kst + (kk >> 2) * (kBN * 128) + (kk & 3) * 32, 16, 1024);
+          mma_bf16_ss(tmem + x * kBN, a, b, idesc_s, kk > 0 ? 1u : 0u);
+        }
+        mma_commit(&bars->s_full[x]);
+      };
+      // O_X += P_X V for tile x from V stage vs
+      auto issue_pv = [&](int x, int vs, bool first) {
+        const uint32_t vst = v_base + vs * C::kTileBytes;
+#pragma unroll
+        for (int kk = 0; kk < kBN / 16; ++kk) {
+          const uint64_t b = sdesc_sw128(vst + kk * (16 * 128), kBN * 128, 1024);
+          mma_bf16_ts(tmem + C::kOCol + x * HD, tmem + x * kBN + kk * 8, b, idesc_pv,
+                      (!first || kk > 0) ? 1u : 0u);
+        }
+      };
+      while (ok && walk.next(p, T, seg)) {
+        if (!wait(&bars->q_full, q_round & 1)) break;
+        ++q_round;
+        tc_fence_after();
+        const int nj = static_cast<int>(seg.j1 - seg.j0);
+        int ks = k_it % C::kStages;
+        if (!wait(&bars->k_full[ks], (k_it / C::kStages) & 1)) break;
+        tc_fence_after();
+        issue_s(0, ks);
+        issue_s(1, ks);
+        mma_commit(&bars->k_empty[ks]);
+        ++k_it;
+        if (nj == 1) mma_commit(&bars->q_empty);
+        for (int i = 0; i < nj; ++i) {
+          const int vs = v_it % C::kStages;
+          const bool more = i + 1 < nj;
+          // ---- tile A
+          if (!wait(&bars->p_full[0], pv_n[0] & 1)) break;
+          if (!wait(&bars->v_full[vs], (v_it / C::kStages) & 1)) break;
+          if (i == 0 && seg_n > 0 && !wait(&bars->o_free[0], (seg_n & 1) ^ 1)) break;
+          tc_fence_after();
+          issue_pv(0, vs, i == 0);
+          if (i == nj - 1) mma_commit(&bars->o_final[0]);
+          ++pv_n[0];
+          if (more) {
+            ks = k_it % C::kStages;
+            if (!wait(&bars->k_full[ks], (k_it / C::kStages) & 1)) break;
+            tc_fence_after();
+            issue_s(0, ks);
+          }
+          // ---- tile B
+          if (!wait(&bars->p_full[1], pv_n[1] & 1)) break;
+          if (i == 0 && seg_n > 0 && !wait(&bars->o_free[1], (seg_n & 1) ^ 1)) break;
+          tc_fence_after();
+          issue_pv(1, vs, i == 0);
+          if (i == nj - 1) mma_commit(&bars->o_final[1]);
+          ++pv_n[1];
+          mma_commit(&bars->v_empty[vs]);
+          ++v_it;
+          if (more) {
+            issue_s(1, ks);
+            mma_commit(&bars->k_empty[ks]);
+            ++k_it;
+            if (i + 1 == nj - 1) mma_commit(&bars->q_empty);
+          }
+        }
+        ++seg_n;
+      }
+      if (!ok) {
+        mma_commit(&bars->drain);
+        drain_wait(&bars->drain, 0);
+      }
+    }
+  } else {
+    // ------------------------------------------------------ softmax warpgroups
+    const int wg = warp >> 2;                  // 0: tile A, 1: tile B
+    const int row = threadIdx.x - wg * 128;    // TMEM lane
+    const uint32_t lane_base = static_cast<uint32_t>((warp & 3) * 32) << 16;
+    const uint32_t s_col = wg * kBN;
+    const uint32_t o_col = C::kOCol + wg * HD;
+    uint32_t s_it = 0, seg_n = 0;
+    bool ok = true;
+    while (ok && walk.next(p, T, seg)) {
+      const int tile = seg.tile * 2 + wg;
+      const int64_t t = static_cast<int64_t>(tile) * T + row / p.group;
+      const bool valid = tile < p.n_tiles && t < p.n;
+      const int64_t limit = valid ? p.L + t : -1;
+      float m_ref = -CUDART_INF_F;
+      float l = 0.f;
+      const int nj = static_cast<int>(seg.j1 - seg.j0);
+      for (int i = 0; i < nj; ++i) {
+        const int64_t j = seg.j0 + i;
+        const bool got = mbar_wait(&bars->s_full[wg], s_it & 1, abort, p.err,
+                                   CSR_DEVERR_WAIT_TIMEOUT);
+        if (!__all_sync(0xffffffffu, got)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        uint32_t sr[kBN];
+        tmem_ld128_wait(tmem + lane_base + s_col, sr);
+        float s[kBN];
+#pragma unroll
+        for (int c = 0; c < kBN; ++c) s[c] = __uint_as_float(sr[c]);
+        const int64_t key0 = j * kBN;
+        if (key0 + kBN - 1 > limit) {
+#pragma unroll
+          for (int c = 0; c < kBN; ++c)
+            if (key0 + c > limit) s[c] = -CUDART_INF_F;
+        }
+        float mp[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) mp[e] = s[e];
+#pragma unroll
+        for (int c = 8; c < kBN; ++c) mp[c & 7] = fmaxf(mp[c & 7], s[c]);
+        const float mx = fmaxf(fmaxf(fmaxf(mp[0], mp[1]), fmaxf(mp[2], mp[3])),
+                               fmaxf(fmaxf(mp[4], mp[5]), fmaxf(mp[6], mp[7])));
+        const float mx_s = mx * p.scale_log2;
+        const bool need = mx_s > m_ref + 8.0f;
+        const float m_new = need ? mx_s : m_ref;
+        const float alpha = need ? ex2_approx(m_ref - m_new) : 1.0f;
+        const bool had_mass = l > 0.f;
+        l *= alpha;
+        m_ref = m_new;
+        const float m_use = (m_ref == -CUDART_INF_F) ? 0.f : m_ref;
+        float rp[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) rp[e] = 0.f;
+        uint32_t pk[kBN / 2];
+#pragma unroll
+        for (int c = 0; c < kBN; c += 2) {
+          const float p0 = ex2_approx(fmaf(s[c], p.scale_log2, -m_use));
+          const float p1 = ex2_approx(fmaf(s[c + 1], p.scale_log2, -m_use));
+          rp[(c >> 1) & 7] += p0 + p1;
+          pk[c / 2] = pack_bf16x2(p0, p1);
+        }
+        l += ((rp[0] + rp[1]) + (rp[2] + rp[3])) + ((rp[4] + rp[5]) + (rp[6] + rp[7]));
+        tmem_st64(tmem + lane_base + s_col, pk);
+        // PV of the previous tile finished before these scores were published
+        // (same commit), so O can be rescaled here without another wait.
+        if (i > 0 && __any_sync(0xffffffffu, need && had_mass))
+          rescale_o<HD>(tmem + lane_base + o_col, alpha);
+        tmem_st_wait();
+        tc_fence_before();
+        mbar_arrive(&bars->p_full[wg]);
+        ++s_it;
+      }
+      if (!ok) break;
+      // ---------------------------------------------------- epilogue
+      const bool got_o = mbar_wait(&bars->o_final[wg], seg_n & 1, abort, p.err,
+                                   CSR_DEVERR_WAIT_TIMEOUT);
+      if (!__all_sync(0xffffffffu, got_o)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      const float inv_l = l > 0.f ? 1.0f / l : 0.f;
+      const float lse2 = l > 0.f ? m_ref + log2f(l) : -CUDART_INF_F;
+      uint32_t o[HD];
+      load_o<HD>(tmem + lane_base + o_col, o);
+      if (seg.complete) {
+        if (valid) {
+          const int hq_idx = seg.head * p.group + row % p.group;
+          uint16_t *dst = p.out + (static_cast<int64_t>(t) * p.hq + hq_idx) * HD;
+#pragma unroll
+          for (int q8 = 0; q8 < HD / 8; ++q8) {
+            uint32_t w[4];
+#pragma unroll
+            for (int c = 0; c < 4; ++c)
+              w[c] = pack_bf16x2(__uint_as_float(o[q8 * 8 + 2 * c]) * inv_l,
+                                 __uint_as_float(o[q8 * 8 + 2 * c + 1]) * inv_l);
+            reinterpret_cast<uint4 *>(dst)[q8] = make_uint4(w[0], w[1], w[2], w[3]);
+          }
+          if (p.lse) p.lse[static_cast<int64_t>(hq_idx) * p.n + t] = lse2 * 0.69314718055994531f;
+        }
+      } else {
+        const int64_t base = static_cast<int64_t>(seg.item) * (2 * kBM) + wg * kBM + row;
+        float4 *d4 = reinterpret_cast<float4 *>(p.part_o + base * HD);
+#pragma unroll
+        for (int c = 0; c < HD / 4; ++c)
+          d4[c] = make_float4(__uint_as_float(o[4 * c]) * inv_l, __uint_as_float(o[4 * c + 1]) * inv_l,
+                              __uint_as_float(o[4 * c + 2]) * inv_l, __uint_as_float(o[4 * c + 3]) * inv_l);
+        p.part_lse[base] = lse2;
+      }
+      tc_fence_before();
+      mbar_arrive(&bars->o_free[wg]);
+      ++seg_n;
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 9) {
+    __syncwarp();
+    tc_fence_after();
+    tmem_dealloc(tmem, C::kTmemCols);
+  }
+}
+
 // ------------------------------------------------------------------ K3 merge
 // Merge the key-chunk pieces of one row: lse = log2 sum_k 2^lse_k and
 // O = sum_k 2^(lse_k - lse) O_k (each O_k already normalised by its own sum).
 // One warp per packed row; lanes own head_dim/32 output columns.
 template <int HD>
 __global__ void __launch_bounds__(256) merge_kernel(const __grid_constant__ MergeParams p) {
-  const int u = blockIdx.x;
-  const int head = u / p.n_tiles;
-  const int tile = u - head * p.n_tiles;
+  const int head = blockIdx.x / p.n_tiles;
+  const int tile = blockIdx.x - head * p.n_tiles;
   const int T = kBM / p.group;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int64_t kv = unit_iters(p.L, p.n, T, tile);
+  const int uph = (p.n_tiles + p.unit_tiles - 1) / p.unit_tiles;  // units per head
+  const int unit = tile / p.unit_tiles;
+  const int half = tile - unit * p.unit_tiles;
+  const int64_t kv = unit_iters(p.L, p.n, T, unit * p.unit_tiles + p.unit_tiles - 1);
   const int nk = static_cast<int>((kv + p.chunk_tiles - 1) / p.chunk_tiles);
   if (nk <= 1) return;  // written whole by the attention kernel
   const int r = blockIdx.y * 8 + warp;
   const int64_t t = static_cast<int64_t>(tile) * T + r / p.group;
   if (r >= kBM || t >= p.n) return;
-  const int units = p.hkv * p.n_tiles;
-  auto item_of = [&](int k) { return static_cast<int64_t>(k) * units + u; };
+  const int64_t units = static_cast<int64_t>(p.hkv) * uph;
+  const int64_t rows_per_item = static_cast<int64_t>(p.unit_tiles) * kBM;
+  const int64_t row_in_item = static_cast<int64_t>(half) * kBM + r;
+  // row index (item * rows_per_item + row_in_item) of chunk k's partial
+  auto prow = [&](int k) {
+    return (static_cast<int64_t>(k) * units + static_cast<int64_t>(head) * uph + unit) * rows_per_item +
+           row_in_item;
+  };
   float mx = -CUDART_INF_F;
-  for (int k = lane; k < nk; k += 32) mx = fmaxf(mx, p.part_lse[item_of(k) * kBM + r]);
+  for (int k = lane; k < nk; k += 32) mx = fmaxf(mx, p.part_lse[prow(k)]);
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
   constexpr int kPer = HD / 32;  // floats per lane
@@ -519,12 +934,12 @@ __global__ void __launch_bounds__(256) merge_kernel(const __grid_constant__ Merg
   float lse2 = -CUDART_INF_F;
   if (mx != -CUDART_INF_F) {
     float sum = 0.f;
-    for (int k = lane; k < nk; k += 32) sum += ex2_approx(p.part_lse[item_of(k) * kBM + r] - mx);
+    for (int k = lane; k < nk; k += 32) sum += ex2_approx(p.part_lse[prow(k)] - mx);
 #pragma unroll
     for (int off = 16; off > 0; off >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, off);
     lse2 = mx + log2f(sum);
     for (int k = 0; k < nk; ++k) {
-      const int64_t base = item_of(k) * kBM + r;
+      const int64_t base = prow(k);
       const float w = ex2_approx(p.part_lse[base] - lse2);
       const float *src = p.part_o + base * HD + lane * kPer;
       float v[kPer];
@@ -548,18 +963,30 @@ __global__ void __launch_bounds__(256) merge_kernel(const __grid_constant__ Merg
 }
 
 cudaError_t attn_configure(int head_dim) {
-  if (head_dim == 64)
-    return cudaFuncSetAttribute(attn_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                AttnCfg<64>::kSmem);
-  return cudaFuncSetAttribute(attn_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              AttnCfg<128>::kSmem);
+  const auto attr = cudaFuncAttributeMaxDynamicSharedMemorySize;
+  cudaError_t e;
+  if (head_dim == 64) {
+    e = cudaFuncSetAttribute(attn_kernel<64>, attr, AttnCfg<64>::kSmem);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(attn_pair_kernel<64>, attr, PairCfg<64>::kSmem);
+  } else {
+    e = cudaFuncSetAttribute(attn_kernel<128>, attr, AttnCfg<128>::kSmem);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(attn_pair_kernel<128>, attr, PairCfg<128>::kSmem);
+  }
+  return e;
 }
 
 cudaError_t launch_attention(const AttnParams &p, int head_dim, cudaStream_t s) {
-  if (head_dim == 64)
-    attn_kernel<64><<<p.grid, 192, AttnCfg<64>::kSmem, s>>>(p);
-  else
-    attn_kernel<128><<<p.grid, 192, AttnCfg<128>::kSmem, s>>>(p);
+  if (p.unit_tiles == 2) {
+    if (head_dim == 64)
+      attn_pair_kernel<64><<<p.grid, 320, PairCfg<64>::kSmem, s>>>(p);
+    else
+      attn_pair_kernel<128><<<p.grid, 320, PairCfg<128>::kSmem, s>>>(p);
+  } else {
+    if (head_dim == 64)
+      attn_kernel<64><<<p.grid, 192, AttnCfg<64>::kSmem, s>>>(p);
+    else
+      attn_kernel<128><<<p.grid, 192, AttnCfg<128>::kSmem, s>>>(p);
+  }
   return cudaGetLastError();
 }
 

@@ -159,3 +159,17 @@ def test_rewind_then_append_matches_never_appended(libcsr):
     assert a.ctx.layout() == b.ctx.layout()
     a.check_layout()
     a.device_clean()
+
+
+@pytest.mark.parametrize("shape", [C1, C2], ids=["d64_p16_g4", "d128_p64_g16"])
+@pytest.mark.parametrize("chunk_tiles", [0, 2])
+def test_single_tile_kernel_matches_oracle(libcsr, shape, chunk_tiles):
+    """The one-tile-per-CTA kernel (CSR_FLAG_SINGLE_TILE) stays correct too."""
+    p = Pair(shape, pool_pages=128, max_seq=4096, max_new=512, fg_chunk_tiles=chunk_tiles,
+             flags=libcsr.FLAG_SINGLE_TILE)
+    p.init_static(p.blk(10, 37))
+    for i, n in enumerate([1, 129, 300]):
+        p.append(p.blk(11 + i, n))
+    p.suffix(p.blk(20, 70))
+    p.truncate()
+    p.device_clean()
