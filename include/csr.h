@@ -302,6 +302,55 @@ csr_status csr_get_timing(csr_ctx *ctx, csr_timing *out);
 /* Text of the last failure on this context (never NULL). */
 const char *csr_last_error(const csr_ctx *ctx);
 
+/*
+ * Arguments of csr_attend_block_noalloc.  All pointers are device pointers
+ * of the current device, owned by the caller; q, k, v, out 16-byte aligned.
+ */
+typedef struct csr_block_args {
+  const void *q, *k, *v;      /* the n new tokens, before RoPE: [n][H][head_dim] bf16 */
+  void *k_pool, *v_pool;      /* [pool_pages][num_kv_heads][page_size][head_dim] bf16 */
+  const int32_t *page_table;  /* logical page -> physical page; must cover positions
+                                 0 .. L+n-1 (the new tokens' slots included) */
+  void *out;                  /* [n][num_q_heads][head_dim] bf16 */
+  float *lse;                 /* [num_q_heads][n] or NULL */
+  int64_t L;                  /* cached tokens before the block (positions of the block: L..L+n-1) */
+  int32_t n;
+  int32_t num_q_heads, num_kv_heads, head_dim, page_size, pool_pages;
+  double rope_base;
+  float softmax_scale;        /* 0 selects 1/sqrt(head_dim) */
+} csr_block_args;
+
+/*
+ * The block path of csr_append_chunk / csr_attend_suffix (RoPE and append of
+ * the new keys/values through the caller's page table, causal attention of
+ * the new queries over positions 0..L+n-1, merge of split partials) for
+ * callers that cannot allocate device memory: code that may not call
+ * cudaMalloc at all, e.g. a real-time control loop that must not take the
+ * allocator's locks or wait on it, or a process whose device memory belongs
+ * to another allocator (a framework's caching allocator) so that it cannot
+ * size and hand over the workspace csr_create needs.  The paper has no
+ * counterpart: it is a property of this library, not of the method.
+ *
+ * Allocates nothing (no cudaMalloc, cudaFree or allocating library call).  Its
+ * scratch is one static device array of 32.5 MiB that every GPU loading the
+ * library holds until the process exits: 8 MiB of packed rotated queries
+ * (so n * num_q_heads * head_dim * 2 bytes, rounded up to whole pairs of
+ * 128-row tiles, must not exceed 8 MiB: n <= 512 for 64 query heads of 128
+ * dims; larger n returns CSR_EINVAL), 24.5 MiB of split-KV partials (the key
+ * range is split only as far as they fit) and the device error word.  The
+ * first call on a device resolves that array's address and sets the kernels'
+ * shared-memory limit for the device (cudaGetSymbolAddress,
+ * cudaFuncSetAttribute); make that first call before any stream capture.
+ * Every call shares the array and it keeps the last call's contents; the
+ * error word is cleared at the start of each call and not reported.  Calls
+ * that overlap on the same GPU (issued on different streams and not ordered)
+ * race on the array: order them.  Each GPU has its own copy of the array.
+ * Asynchronous on `stream`.
+ * CSR_EINVAL for bad arguments or sizes beyond the limit, CSR_ECUDA if a CUDA
+ * call fails.
+ */
+csr_status csr_attend_block_noalloc(const csr_block_args *args, csr_stream_t stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -25,7 +25,7 @@ CUDA_HOME = os.environ.get("CUDA_HOME", "/usr/local/cuda")
 NVCC = os.path.join(CUDA_HOME, "bin", "nvcc")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
-SOURCES = ["csr_api.cpp", "kernels_attn.cu", "kernels_misc.cu"]
+SOURCES = ["csr_api.cpp", "kernels_attn.cu", "kernels_misc.cu", "csr_noalloc.cu"]
 HEADERS = ["internal.h", "ptx.cuh"]
 
 

@@ -1,0 +1,219 @@
+// csr_noalloc.cu -- csr_attend_block_noalloc: the block path (RoPE + paged
+// append, attention, split merge) for callers that cannot allocate device
+// memory.  Its scratch (packed rotated queries, split-KV partials, the device
+// error word) lives in one file-scope static device array instead of a
+// caller-allocated workspace.
+#include <cmath>
+#include <cstring>
+#include <mutex>
+
+#include <cuda.h>
+#include <cudaTypedefs.h>
+#include <cuda_runtime.h>
+
+#include "../../include/csr.h"
+#include "internal.h"
+
+namespace {
+
+using namespace csr;
+
+constexpr size_t kQBytes = 8ull << 20;     // packed rotated queries
+constexpr size_t kPartOBytes = 24ull << 20; // split partial outputs (fp32)
+constexpr size_t kPartLseBytes = 512ull << 10;
+constexpr size_t kErrBytes = 256;
+constexpr size_t kScratchBytes = kQBytes + kPartOBytes + kPartLseBytes + kErrBytes;
+constexpr int kMaxDevices = 64;
+
+// One copy per device that loads the library, kept until the process exits.
+// Device code could name it directly; host code must use the address that
+// cudaGetSymbolAddress returns for the current device.
+static __device__ __align__(256) uint8_t g_block_scratch[kScratchBytes];
+
+struct DeviceSetup {
+  bool ready = false;
+  uint8_t *scratch = nullptr;  // device address of g_block_scratch on this device
+  int num_sms = 0;
+};
+std::mutex g_setup_mu;
+DeviceSetup g_setup[kMaxDevices];
+
+PFN_cuTensorMapEncodeTiled_v12000 encoder() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (!fn) {
+    void *p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  }
+  return fn;
+}
+
+bool encode(CUtensorMap *m, const void *base, uint64_t rows, uint64_t d, uint32_t box_rows) {
+  auto fn = encoder();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {d, rows};
+  cuuint64_t strides[1] = {d * 2};
+  cuuint32_t box[2] = {64, box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims, strides, box,
+            estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+int64_t cdiv(int64_t a, int64_t b) { return (a + b - 1) / b; }
+
+// Once per device, with that device current: resolve the scratch array's
+// device address and raise the attention kernels' shared-memory limit.
+csr_status setup_device(int dev, DeviceSetup **out) {
+  if (dev < 0 || dev >= kMaxDevices) return CSR_EINVAL;
+  std::lock_guard<std::mutex> lock(g_setup_mu);
+  DeviceSetup &s = g_setup[dev];
+  if (!s.ready) {
+    void *ptr = nullptr;
+    if (cudaGetSymbolAddress(&ptr, g_block_scratch) != cudaSuccess) return CSR_ECUDA;
+    if (attn_configure(64) != cudaSuccess || attn_configure(128) != cudaSuccess) return CSR_ECUDA;
+    int sms = 0;
+    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+      return CSR_ECUDA;
+    s.scratch = static_cast<uint8_t *>(ptr);
+    s.num_sms = sms;
+    s.ready = true;
+  }
+  *out = &s;
+  return CSR_OK;
+}
+
+bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+}  // namespace
+
+extern "C" csr_status csr_attend_block_noalloc(const csr_block_args *a, csr_stream_t stream) {
+  if (!a) return CSR_EINVAL;
+  const int32_t hq = a->num_q_heads, hkv = a->num_kv_heads, d = a->head_dim, P = a->page_size;
+  if (hq <= 0 || hkv <= 0 || hq % hkv) return CSR_EINVAL;
+  const int32_t g = hq / hkv;
+  if ((g & (g - 1)) != 0 || g > kBM) return CSR_EINVAL;
+  if (d != 64 && d != 128) return CSR_EINVAL;
+  if (P != 16 && P != 32 && P != 64 && P != 128) return CSR_EINVAL;
+  if (a->n < 1 || a->L < 0 || a->pool_pages < 1 || !(a->rope_base > 1.0) || a->softmax_scale < 0.f)
+    return CSR_EINVAL;
+  if (static_cast<int64_t>(a->pool_pages) * hkv * P >= (1ll << 31)) return CSR_EINVAL;
+  for (const void *p : {a->q, a->k, a->v, static_cast<const void *>(a->out)})
+    if (!p || !aligned16(p)) return CSR_EINVAL;
+  if (!a->k_pool || !a->v_pool || !a->page_table || !aligned16(a->k_pool) || !aligned16(a->v_pool))
+    return CSR_EINVAL;
+  // the packed queries of this call must fit the static scratch
+  const int64_t rows_cap = cdiv(static_cast<int64_t>(a->n) * g, 2 * kBM) * 2 * kBM;
+  if (rows_cap * hkv * d * 2 > static_cast<int64_t>(kQBytes)) return CSR_EINVAL;
+
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return CSR_ECUDA;
+  DeviceSetup *ds = nullptr;
+  csr_status st = setup_device(dev, &ds);
+  if (st != CSR_OK) return st;
+  uint16_t *q_pack = reinterpret_cast<uint16_t *>(ds->scratch);
+  float *part_o = reinterpret_cast<float *>(ds->scratch + kQBytes);
+  float *part_lse = reinterpret_cast<float *>(ds->scratch + kQBytes + kPartOBytes);
+  uint32_t *err = reinterpret_cast<uint32_t *>(ds->scratch + kQBytes + kPartOBytes + kPartLseBytes);
+  const cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  // the error word accumulates with atomicOr: start every call from zero
+  if (cudaMemsetAsync(err, 0, sizeof(uint32_t), s) != cudaSuccess) return CSR_ECUDA;
+
+  // K1: rotate, append the new keys/values through the caller's page table,
+  // pack the rotated queries into the scratch
+  RopeAppendParams rp{};
+  rp.q = static_cast<const uint16_t *>(a->q);
+  rp.k = static_cast<const uint16_t *>(a->k);
+  rp.v = static_cast<const uint16_t *>(a->v);
+  rp.k_pool = static_cast<uint16_t *>(a->k_pool);
+  rp.v_pool = static_cast<uint16_t *>(a->v_pool);
+  rp.q_pack = q_pack;
+  rp.page_table = const_cast<int32_t *>(a->page_table);  // read only: n_ids == 0
+  rp.err = err;
+  rp.pos0 = a->L;
+  rp.n = a->n;
+  rp.hq = hq;
+  rp.hkv = hkv;
+  rp.d = d;
+  rp.page_size = P;
+  rp.group = g;
+  rp.rows_cap = static_cast<int32_t>(rows_cap);
+  rp.pool_pages = a->pool_pages;
+  rp.first_lp = 0;
+  rp.n_ids = 0;
+  const double two_pi = 6.283185307179586476925286766559;
+  for (int i = 0; i < d / 2; ++i) rp.inv_turns[i] = std::pow(a->rope_base, -2.0 * i / d) / two_pi;
+  if (launch_rope_append(rp, s) != cudaSuccess) return CSR_ECUDA;
+
+  // K2: two-tile attention over keys [0, L + n)
+  AttnParams ap{};
+  const uint64_t pool_rows = static_cast<uint64_t>(a->pool_pages) * hkv * P;
+  if (!encode(&ap.tm_q, q_pack, static_cast<uint64_t>(hkv) * rows_cap, d, kBM) ||
+      !encode(&ap.tm_k, a->k_pool, pool_rows, d, P) || !encode(&ap.tm_v, a->v_pool, pool_rows, d, P))
+    return CSR_ECUDA;
+  ap.page_table = a->page_table;
+  ap.out = static_cast<uint16_t *>(a->out);
+  ap.lse = a->lse;
+  ap.part_o = part_o;
+  ap.part_lse = part_lse;
+  ap.err = err;
+  ap.L = a->L;
+  ap.n = a->n;
+  ap.hq = hq;
+  ap.hkv = hkv;
+  ap.group = g;
+  ap.page_size = P;
+  ap.rows_cap = static_cast<int32_t>(rows_cap);
+  ap.n_tiles = static_cast<int32_t>(cdiv(static_cast<int64_t>(a->n) * g, kBM));
+  ap.n_pages_valid = static_cast<int32_t>(cdiv(a->L + a->n, P));
+  ap.pool_pages = a->pool_pages;
+  ap.unit_tiles = 2;
+  const int T = kBM / g;
+  const int64_t uph = cdiv(ap.n_tiles, 2);
+  const int64_t units = uph * hkv;
+  const int64_t kv_max = unit_iters(a->L, a->n, T, static_cast<int32_t>(uph * 2 - 1));
+  // Split the key range only as far as the static partial buffer allows:
+  // one chunk per unit when there are enough units to fill the SMs, else
+  // the most chunks (up to one wave) whose partials fit.
+  const int64_t cap_items = static_cast<int64_t>(kPartOBytes / (2ull * kBM * d * 4));
+  const int64_t lse_items = static_cast<int64_t>(kPartLseBytes / (2ull * kBM * 4));
+  const int64_t max_items = cap_items < lse_items ? cap_items : lse_items;
+  int64_t chunks = 1;
+  if (units < ds->num_sms) {
+    chunks = ds->num_sms / units;
+    if (chunks * units > max_items) chunks = max_items / units;
+    if (chunks < 1) chunks = 1;
+    if (chunks > kv_max) chunks = kv_max;
+  }
+  ap.chunk_tiles = static_cast<int32_t>(cdiv(kv_max, chunks));
+  const int64_t n_chunks = cdiv(kv_max, ap.chunk_tiles);
+  ap.n_items = static_cast<int32_t>(n_chunks * units);
+  ap.grid = static_cast<int32_t>(ap.n_items < ds->num_sms ? ap.n_items : ds->num_sms);
+  const double scale = a->softmax_scale > 0.f ? static_cast<double>(a->softmax_scale)
+                                              : 1.0 / std::sqrt(static_cast<double>(d));
+  ap.scale_log2 = static_cast<float>(scale * 1.4426950408889634);
+  if (launch_attention(ap, d, s) != cudaSuccess) return CSR_ECUDA;
+
+  // K3: merge the split partials
+  if (n_chunks > 1) {
+    MergeParams mp{};
+    mp.part_o = part_o;
+    mp.part_lse = part_lse;
+    mp.out = ap.out;
+    mp.lse = a->lse;
+    mp.L = a->L;
+    mp.n = a->n;
+    mp.hq = hq;
+    mp.hkv = hkv;
+    mp.group = g;
+    mp.n_tiles = ap.n_tiles;
+    mp.chunk_tiles = ap.chunk_tiles;
+    mp.unit_tiles = 2;
+    mp.d = d;
+    if (launch_merge(mp, s) != cudaSuccess) return CSR_ECUDA;
+  }
+  return CSR_OK;
+}
