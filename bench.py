@@ -70,7 +70,8 @@ def _traffic_per_launch_step():
     summary, if it was taken on the current kernel source; else None."""
     try:
         with open(TRAFFIC_FILE) as f:
-            kv = dict(line.strip().split("=", 1) for line in f if "=" in line)
+            kv = dict(line.strip().split("=", 1) for line in f
+                      if "=" in line and not line.startswith("#"))
         if kv.get("kernel_source_sha256_16") != _attention_source_hash():
             return None
         return float(kv["dram_bytes_per_step"])
@@ -393,6 +394,206 @@ def run_ours(args):
     return 0
 
 
+# ------------------------------------------------------------------ ASR leg
+ASR_CAP, ASR_EVICT = 131072, 32768
+
+
+def run_asr(args):
+    """The ASR cycle run: cache capped at 131,072 tokens (4,096-token prefix),
+    foreground steps (256-token chunk + 512-token suffix + truncate) at a fixed
+    cadence; reaching the cap evicts the oldest 32,768 tokens of chunks and
+    rebuilds the retained ~98K tokens on a low-priority stream (Algorithm 1),
+    then swaps.  Reports foreground step latency during and outside rebuilds
+    and checks every post-swap page table against the oracle's allocator."""
+    import numpy as np
+    import torch
+    from oracle import oracle as orc
+    from paper_2605_07325_gb300 import csr
+
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    pool_pages = (ASR_CAP + (ASR_CAP - ASR_EVICT) + 8 * CHUNK * 64) // P + 64
+    cfg = csr.make_config(HQ, HKV, D, P, BASE, max_new_tokens=PREFIX, pool_pages=pool_pages,
+                          max_seq_tokens=ASR_CAP + 64 * CHUNK, cap_tokens=ASR_CAP,
+                          evict_tokens=ASR_EVICT, n_catchup=0)
+    fg = torch.cuda.Stream(device=dev, priority=-1)     # high priority
+    lo = torch.cuda.Stream(device=dev, priority=0)      # low priority (rebuild, R_2)
+    gen = torch.Generator(device=dev).manual_seed(4321)
+
+    def rnd(n, h):
+        return torch.randn((n, h, D), generator=gen, device=dev, dtype=torch.float32).to(torch.bfloat16)
+
+    chunks = {}
+
+    def provider(cid, n):
+        q, k, v = chunks[cid]
+        return q, k, v, None
+
+    # layout model: the oracle's allocator on the same operations (attention off)
+    model = orc.OracleCSR(1, 1, 2, P, BASE, pool_pages)
+    model.attend = False
+    z = lambda n: (np.zeros((n, 1, 2)), np.zeros((n, 1, 2)), np.zeros((n, 1, 2)))
+    with torch.cuda.stream(fg):
+        ctx = csr.Context(cfg, device=str(dev), stream=fg)
+        ctx.set_reconciler(provider, lo)
+        ctx.init_static(rnd(PREFIX, HQ), rnd(PREFIX, HKV), rnd(PREFIX, HKV), stream=fg)
+        model.init_static(*z(PREFIX))
+        fout = torch.empty((CHUNK, HQ, D), dtype=torch.bfloat16, device=dev)
+        while ctx.layout()[1] + CHUNK < ASR_CAP:
+            q, k, v = rnd(CHUNK, HQ), rnd(CHUNK, HKV), rnd(CHUNK, HKV)
+            _, _, cid = ctx.append_chunk(q, k, v, out=fout, stream=fg)
+            chunks[cid] = (q, k, v)
+            model.append_chunk(*z(CHUNK))
+        sq, sk, sv = rnd(SUFFIX, HQ), rnd(SUFFIX, HKV), rnd(SUFFIX, HKV)
+        so = torch.empty((SUFFIX, HQ, D), dtype=torch.bfloat16, device=dev)
+    fg.synchronize()
+
+    period = 1.0 / args.asr_cadence_hz if args.asr_cadence_hz > 0 else 0.0
+    records, rebuilds, layout_ok = [], [], True
+    cycles, step = 0, 0
+    rb_start = None
+    next_t = time.perf_counter()
+    while cycles < args.asr_cycles:
+        was = model.is_reconciling
+        with torch.cuda.stream(fg):
+            q, k, v = rnd(CHUNK, HQ), rnd(CHUNK, HKV), rnd(CHUNK, HKV)
+        fg.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        t0 = time.perf_counter()
+        e0.record(fg)
+        _, _, cid = ctx.append_chunk(q, k, v, out=fout, stream=fg)
+        chunks[cid] = (q, k, v)
+        ctx.attend_suffix(sq, sk, sv, out=so, stream=fg)
+        ctx.truncate_suffix()
+        e1.record(fg)
+        e1.synchronize()
+        t1 = time.perf_counter()
+        model.append_chunk(*z(CHUNK))
+        if not was and model.length() >= ASR_CAP:
+            model.evict(ASR_EVICT)          # the library started it inside append_chunk
+            rb_start = time.perf_counter()
+            lo_ev = torch.cuda.Event(enable_timing=True)
+            lo_ev.record(lo)                # after every rebuild launch
+        state = ctx.poll_swap(fg)
+        during = was or model.is_reconciling
+        records.append((t1 - t0, e0.elapsed_time(e1) / 1e3, during))
+        if state == csr.RECON_SWAPPED:
+            model.reconcile()
+            pt, length = ctx.layout()
+            ok = pt == model.page_table() and ctx.free_pages() == model.free_ids() \
+                and length == model.length()
+            layout_ok = layout_ok and ok
+            rebuilds.append(time.perf_counter() - rb_start)
+            cycles += 1
+        step += 1
+        if period:
+            next_t += period
+            time.sleep(max(0.0, next_t - time.perf_counter()))
+    flags = ctx.device_status()
+
+    def pct(xs, q):
+        return float(np.percentile(np.array(xs) * 1e3, q)) if xs else None
+
+    dur = [r[0] for r in records if r[2]]
+    out = [r[0] for r in records if not r[2]]
+    dev_dur = [r[1] for r in records if r[2]]
+    dev_out = [r[1] for r in records if not r[2]]
+    line = {
+        "workload": ("ASR cycle run: cap 131,072 tokens, 4,096-token prefix, 256-token chunks + "
+                     "512-token suffix per step, evict oldest 32,768 tokens, rebuild on a "
+                     "low-priority stream, 64 q / 4 kv heads, d 128, page 64, 1 layer"),
+        "cadence_hz": args.asr_cadence_hz, "cycles": cycles, "steps": step,
+        "steps_during_rebuild": len(dur),
+        "fg_ms_host": {"p50_outside": pct(out, 50), "p99_outside": pct(out, 99),
+                       "p50_during": pct(dur, 50), "p99_during": pct(dur, 99)},
+        "fg_ms_device": {"p50_outside": pct(dev_out, 50), "p99_outside": pct(dev_out, 99),
+                         "p50_during": pct(dev_dur, 50), "p99_during": pct(dev_dur, 99)},
+        "rebuild_to_swap_s": {"mean": statistics.mean(rebuilds) if rebuilds else None,
+                              "max": max(rebuilds) if rebuilds else None,
+                              "note": "eviction to the first poll that saw the swap"},
+        "layout_bit_exact_vs_oracle": layout_ok,
+        "device_error_flags": flags,
+    }
+    if out and dur:
+        line["p99_increase_during_rebuild"] = pct(dur, 99) / pct(out, 99) - 1.0
+    print(json.dumps(line), flush=True)
+    ctx.close()
+    return 0 if layout_ok and flags == 0 else 1
+
+
+# ---------------------------------------------------------------- sweep leg
+SWEEP_L = (16384, 32768, 65536, 98304, 131072)
+SWEEP_N = (16, 64, 256, 1024, 4096)
+
+
+def run_sweep(args):
+    """One attend call of n new tokens over L cached tokens for every sweep
+    point: device time per call, the attention kernel's time, achieved
+    TFLOP/s and GB/s, and the fraction of the roofline floor
+    max(FLOPs / bf16 peak, bytes / HBM peak)."""
+    import torch
+    from paper_2605_07325_gb300 import costmodel, csr
+
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    hbm, peak, _, kind = _peaks()
+    max_L = max(SWEEP_L)
+    cfg = csr.make_config(HQ, HKV, D, P, BASE, max_new_tokens=4096,
+                          pool_pages=(max_L + 4096) // P + 16, max_seq_tokens=max_L + 4096 + P)
+    stream = torch.cuda.Stream(device=dev, priority=-1)
+    gen = torch.Generator(device=dev).manual_seed(99)
+
+    def rnd(n, h):
+        return torch.randn((n, h, D), generator=gen, device=dev, dtype=torch.float32).to(torch.bfloat16)
+
+    K, W = max(3, args.steps // 10), args.warmup
+    points = []
+    with torch.cuda.stream(stream):
+        ctx = csr.Context(cfg, device=str(dev), stream=stream)
+        ctx.init_static(rnd(PREFIX, HQ), rnd(PREFIX, HKV), rnd(PREFIX, HKV), stream=stream)
+        fill_q = rnd(4096, HQ)
+        fill_o = torch.empty((4096, HQ, D), dtype=torch.bfloat16, device=dev)
+        blocks = {n: (rnd(n, HQ), rnd(n, HKV), rnd(n, HKV),
+                      torch.empty((n, HQ, D), dtype=torch.bfloat16, device=dev)) for n in SWEEP_N}
+        for L in SWEEP_L:
+            while ctx.layout()[1] < L:
+                ctx.append_chunk(fill_q, rnd(4096, HKV), rnd(4096, HKV), out=fill_o, stream=stream)
+            assert ctx.layout()[1] == L
+            for n in SWEEP_N:
+                q, k, v, o = blocks[n]
+                for _ in range(W):
+                    ctx.attend_suffix(q, k, v, out=o, stream=stream)
+                    ctx.truncate_suffix()
+                stream.synchronize()
+                ctx.set_timing(True)
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                e0.record(stream)
+                for _ in range(K):
+                    ctx.attend_suffix(q, k, v, out=o, stream=stream)
+                    ctx.truncate_suffix()
+                e1.record(stream)
+                stream.synchronize()
+                t = ctx.get_timing()
+                ctx.set_timing(False)
+                us = e0.elapsed_time(e1) / K * 1e3
+                f = costmodel.attention_flops(HQ, D, L, n)
+                b = costmodel.call_bytes(HQ, HKV, D, L, n)
+                floor = costmodel.floor_seconds(f, b, peak, hbm) * 1e6
+                att_us = t["attention"][0] / max(1, t["attention"][1]) * 1e3
+                pt = {"L": L, "n": n, "us_per_call": us, "attention_us": att_us,
+                      "tflops": f / (us * 1e-6) / 1e12, "gbs": b / (us * 1e-6) / 1e9,
+                      "floor_us": floor, "bound": "tensor" if f / (peak * 1e12) > b / (hbm * 1e9) else "hbm",
+                      "roofline_frac": floor / us}
+                points.append(pt)
+                print(json.dumps(pt), flush=True)
+    print(json.dumps({"sweep": "L x n, one attend call each", "peaks": {"bf16_tflops": peak, "hbm_gbs": hbm,
+                      "source": kind}, "points": len(points),
+                      "min_frac": min(p["roofline_frac"] for p in points),
+                      "device_error_flags": ctx.device_status()}), flush=True)
+    ctx.close()
+    return 0
+
+
 def main(argv=None):
     ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
     ap.add_argument("--gpus", type=int, default=1)
@@ -405,9 +606,20 @@ def main(argv=None):
     ap.add_argument("--fill-chunk", type=int, default=CHUNK, choices=[256, 512, 1024, 2048, 4096],
                     help="chunk size used to fill the cache before timing (fewer launches "
                          "for profiler captures); the timed steps are unchanged")
+    ap.add_argument("--asr", action="store_true",
+                    help="run the ASR cycle workload instead of the 120K step line")
+    ap.add_argument("--asr-cycles", type=int, default=10)
+    ap.add_argument("--asr-cadence-hz", type=float, default=2.0,
+                    help="foreground step rate; 0 runs steps back to back")
+    ap.add_argument("--sweep", action="store_true",
+                    help="run the L x n sweep instead of the 120K step line")
     args = ap.parse_args(argv)
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
+    if args.sweep:
+        return run_sweep(args)
+    if args.asr:
+        return run_asr(args)
     if args.impl == "reference":
         return run_reference(args)
     return run_ours(args)
