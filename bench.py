@@ -441,8 +441,8 @@ def run_asr(args):
         fout = torch.empty((CHUNK, HQ, D), dtype=torch.bfloat16, device=dev)
         while ctx.layout()[1] + CHUNK < ASR_CAP:
             q, k, v = rnd(CHUNK, HQ), rnd(CHUNK, HKV), rnd(CHUNK, HKV)
-            _, _, cid = ctx.append_chunk(q, k, v, out=fout, stream=fg)
-            chunks[cid] = (q, k, v)
+            chunks[len(chunks)] = (q, k, v)      # ids are 0, 1, 2, ... in append order
+            ctx.append_chunk(q, k, v, out=fout, stream=fg)
             model.append_chunk(*z(CHUNK))
         sq, sk, sv = rnd(SUFFIX, HQ), rnd(SUFFIX, HKV), rnd(SUFFIX, HKV)
         so = torch.empty((SUFFIX, HQ, D), dtype=torch.bfloat16, device=dev)
@@ -461,8 +461,9 @@ def run_asr(args):
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         t0 = time.perf_counter()
         e0.record(fg)
+        chunks[len(chunks)] = (q, k, v)          # before the call: it may start a rebuild
         _, _, cid = ctx.append_chunk(q, k, v, out=fout, stream=fg)
-        chunks[cid] = (q, k, v)
+        assert cid == len(chunks) - 1
         ctx.attend_suffix(sq, sk, sv, out=so, stream=fg)
         ctx.truncate_suffix()
         e1.record(fg)
