@@ -79,6 +79,19 @@ def _traffic_per_launch_step():
         return None
 
 
+# ------------------------------------------------------------------ replicas
+def reduce_max_over_ranks(values, device=None):
+    """Max over ranks of each value (the slowest replica defines the time);
+    identity when torch.distributed is not initialised or has one rank."""
+    import torch
+    import torch.distributed as dist
+    if not dist.is_available() or not dist.is_initialized() or dist.get_world_size() == 1:
+        return [float(v) for v in values]
+    t = torch.tensor([float(v) for v in values], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return [float(x) for x in t.cpu()]
+
+
 # --------------------------------------------------------------------- clocks
 class ClockSampler:
     FIELDS = ("timestamp,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
@@ -234,7 +247,8 @@ def run_ours(args):
     pool_pages = math.ceil(max_tokens / P) + 16
     cfg = csr.make_config(HQ, HKV, D, P, BASE, max_new_tokens=PREFIX, pool_pages=pool_pages,
                           max_seq_tokens=max_tokens + P,
-                          flags=csr.FLAG_SINGLE_TILE if args.single_tile else 0)
+                          flags={"pair": 0, "pipe": csr.FLAG_PIPE_64,
+                                 "single": csr.FLAG_SINGLE_TILE}[args.kernel])
     stream = torch.cuda.Stream(device=dev, priority=-1)
     gen = torch.Generator(device=dev).manual_seed(1234 + rank)
 
@@ -337,10 +351,7 @@ def run_ours(args):
     ms_e2e = e2.elapsed_time(e3)
     flags = ctx.device_status()
 
-    if world > 1:
-        t = torch.tensor([ms_total, ms_e2e], device=dev, dtype=torch.float64)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms_total, ms_e2e = float(t[0]), float(t[1])
+    ms_total, ms_e2e = reduce_max_over_ranks([ms_total, ms_e2e], device=dev)
 
     # ------------------------------------------------ roofline of the attention kernel
     hbm, peak_burst, peak_sust, peak_kind = _peaks()
@@ -369,7 +380,8 @@ def run_ours(args):
         "roofline": {"bound": "tensor", "achieved": achieved, "peak": peak_burst, "unit": "TFLOP/s",
                      "frac": (achieved / peak_burst) if achieved else None,
                      "traffic": (traffic_step / 2) if traffic_step else None,
-                     "kernel": ("attn_kernel<128>" if args.single_tile else "attn_pair_kernel<128>") +
+                     "kernel": {"pipe": "attn_pipe_kernel<128>", "pair": "attn_pair_kernel<128>",
+                                "single": "attn_kernel<128>"}[args.kernel] +
                                " (tcgen05 QK^T and PV, TMA paged K/V)",
                      "launches": att_n, "avg_launch_us": att_ms / max(1, att_n) * 1e3,
                      "peak_source": f"bf16_tflops ({peak_kind}, burst)",
@@ -412,9 +424,12 @@ def run_asr(args):
 
     dev = torch.device("cuda", 0)
     torch.cuda.set_device(dev)
-    pool_pages = (ASR_CAP + (ASR_CAP - ASR_EVICT) + 8 * CHUNK * 64) // P + 64
+    # N_max of App. D: the active version may grow past tau_mem while the rebuild and its
+    # catch-up run (Eq. oom_time); one eviction's worth of headroom covers back-to-back steps
+    n_max = ASR_CAP + ASR_EVICT
+    pool_pages = (2 * n_max) // P + 64
     cfg = csr.make_config(HQ, HKV, D, P, BASE, max_new_tokens=PREFIX, pool_pages=pool_pages,
-                          max_seq_tokens=ASR_CAP + 64 * CHUNK, cap_tokens=ASR_CAP,
+                          max_seq_tokens=n_max, cap_tokens=ASR_CAP,
                           evict_tokens=ASR_EVICT, n_catchup=0)
     fg = torch.cuda.Stream(device=dev, priority=-1)     # high priority
     lo = torch.cuda.Stream(device=dev, priority=0)      # low priority (rebuild, R_2)
@@ -452,14 +467,24 @@ def run_asr(args):
     records, rebuilds, layout_ok = [], [], True
     cycles, step = 0, 0
     rb_start = None
+    peak_len = 0
     next_t = time.perf_counter()
     while cycles < args.asr_cycles:
-        was = model.is_reconciling
         with torch.cuda.stream(fg):
             q, k, v = rnd(CHUNK, HQ), rnd(CHUNK, HKV), rnd(CHUNK, HKV)
         fg.synchronize()
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         t0 = time.perf_counter()
+        # the task starts by polling the reconciliation (the swap happens between tasks)
+        if ctx.poll_swap(fg) == csr.RECON_SWAPPED:
+            model.reconcile()
+            pt, length = ctx.layout()
+            ok = pt == model.page_table() and ctx.free_pages() == model.free_ids() \
+                and length == model.length()
+            layout_ok = layout_ok and ok
+            rebuilds.append(time.perf_counter() - rb_start)
+            cycles += 1
+        was = model.is_reconciling
         e0.record(fg)
         chunks[len(chunks)] = (q, k, v)          # before the call: it may start a rebuild
         _, _, cid = ctx.append_chunk(q, k, v, out=fout, stream=fg)
@@ -475,17 +500,9 @@ def run_asr(args):
             rb_start = time.perf_counter()
             lo_ev = torch.cuda.Event(enable_timing=True)
             lo_ev.record(lo)                # after every rebuild launch
-        state = ctx.poll_swap(fg)
+        peak_len = max(peak_len, model.length())
         during = was or model.is_reconciling
         records.append((t1 - t0, e0.elapsed_time(e1) / 1e3, during))
-        if state == csr.RECON_SWAPPED:
-            model.reconcile()
-            pt, length = ctx.layout()
-            ok = pt == model.page_table() and ctx.free_pages() == model.free_ids() \
-                and length == model.length()
-            layout_ok = layout_ok and ok
-            rebuilds.append(time.perf_counter() - rb_start)
-            cycles += 1
         step += 1
         if period:
             next_t += period
@@ -511,7 +528,8 @@ def run_asr(args):
                          "p50_during": pct(dev_dur, 50), "p99_during": pct(dev_dur, 99)},
         "rebuild_to_swap_s": {"mean": statistics.mean(rebuilds) if rebuilds else None,
                               "max": max(rebuilds) if rebuilds else None,
-                              "note": "eviction to the first poll that saw the swap"},
+                              "note": "eviction to the poll (start of a step) that swapped"},
+        "peak_cached_tokens": peak_len, "n_max_tokens": n_max,
         "layout_bit_exact_vs_oracle": layout_ok,
         "device_error_flags": flags,
     }
@@ -602,8 +620,10 @@ def main(argv=None):
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--single-tile", action="store_true",
-                    help="attention CTAs own one query tile (the earlier kernel design)")
+    ap.add_argument("--kernel", choices=["pair", "pipe", "single"], default="pair",
+                    help="attention kernel: pair (default: two query tiles per CTA, 128-key "
+                         "tiles), pipe (two query tiles, 64-key tiles, two score buffers each), "
+                         "single (one query tile per CTA)")
     ap.add_argument("--fill-chunk", type=int, default=CHUNK, choices=[256, 512, 1024, 2048, 4096],
                     help="chunk size used to fill the cache before timing (fewer launches "
                          "for profiler captures); the timed steps are unchanged")

@@ -72,8 +72,11 @@ typedef enum csr_status {
 #define CSR_FLAG_PLAN_ONLY 0x1   /* layout planning only: no device memory is touched
                                     and no kernel runs; compute calls update the page
                                     tables and lengths but produce no outputs */
-#define CSR_FLAG_SINGLE_TILE 0x2 /* attention CTAs own one 128-row query tile instead of
-                                    two (the earlier kernel design, kept for comparison) */
+#define CSR_FLAG_SINGLE_TILE 0x2 /* attention CTAs own one 128-row query tile, 128-key tiles
+                                    (the first kernel design, kept for comparison) */
+#define CSR_FLAG_PIPE_64 0x4     /* two query tiles per CTA with 64-key tiles and two score
+                                    buffers each (an experimental third design); the default
+                                    uses 128-key tiles and one score buffer per query tile */
 
 typedef struct csr_config {
   int32_t num_q_heads;    /* H_q */
@@ -133,7 +136,8 @@ csr_status csr_init_static(csr_ctx *ctx, const void *q, const void *k,
  * len..len+n-1 of the active version, attend its queries over the whole cache,
  * and return its id in *chunk_id (may be NULL).  While a reconciliation runs
  * the chunk is also reserved in the version being rebuilt and buffered for its
- * catch-up.  If a reconciler is set, cap_tokens > 0 and the length reaches
+ * catch-up; with n_catchup = 0 its catch-up is enqueued on the low-priority
+ * stream at once (the provider is called for it inside this call).  If a reconciler is set, cap_tokens > 0 and the length reaches
  * cap_tokens, an eviction of evict_tokens starts (Algorithm 1, Increment); if
  * it cannot start, the chunk stays appended and its error code is returned.
  * CSR_ESTATE while a suffix is live.
@@ -216,8 +220,10 @@ csr_status csr_evict_and_reconcile(csr_ctx *ctx, int32_t evict_tokens,
 #define CSR_RECON_SWAPPED 2 /* this call swapped the versions */
 
 /*
- * Non-blocking step of Algorithm 1's catch-up loop.  When the rebuild's last
- * launch has finished: while more than n_catchup chunks are buffered, enqueue
+ * Non-blocking step of Algorithm 1's catch-up loop.  Call it between tasks,
+ * before the task's first compute call: right after an append that enqueued a
+ * catch-up it would see that work unfinished.  When the rebuild's last launch
+ * has finished: while more than n_catchup chunks are buffered, enqueue
  * their catch-up on the low-priority stream; otherwise compute the remaining
  * buffered chunks on fg_stream ("computed at next task inference") and swap
  * the active version atomically (App. D step 5).  The old version's own pages

@@ -250,9 +250,9 @@ int64_t pages_for(const csr_ctx *c, int64_t len) { return ceil_div(len, c->cfg.p
 // launch waits at most one item for an SM.  Never more than kPartialItems
 // items when split.
 int32_t choose_chunk_tiles(int64_t units, int64_t kv_max, int64_t grid, int max_tiles,
-                           int head_dim, int unit_tiles) {
+                           int head_dim, int unit_tiles, int kv_tile) {
   // us per key tile per CTA, per item, per split partial (rough GB300 figures)
-  const double t_tile = 0.75 * unit_tiles, t_item = 2.0;
+  const double t_tile = 0.75 * unit_tiles * kv_tile / kBN, t_item = 2.0;
   const double t_part = (head_dim == 128 ? 0.02 : 0.01) * unit_tiles;
   const int64_t cap_items = kPartialItems / unit_tiles;
   int64_t best_c = kv_max;
@@ -360,9 +360,11 @@ csr_status run_block(csr_ctx *c, int slot, int ws, const void *q, const void *k,
   ap.pool_pages = cf.pool_pages;
   const int T = kBM / c->group;
   ap.unit_tiles = (cf.flags & CSR_FLAG_SINGLE_TILE) ? 1 : 2;
+  ap.kv_tile = (!(cf.flags & CSR_FLAG_SINGLE_TILE) && (cf.flags & CSR_FLAG_PIPE_64)) ? kBN64 : kBN;
   const int64_t uph = ceil_div(ap.n_tiles, ap.unit_tiles);
   const int64_t units = uph * cf.num_kv_heads;
-  const int64_t kv_max = unit_iters(L, n, T, static_cast<int32_t>(uph * ap.unit_tiles - 1));
+  const int64_t kv_max =
+      unit_iters(L, n, T, static_cast<int32_t>(uph * ap.unit_tiles - 1), ap.kv_tile);
   const int tpc = cf.rebuild_tiles_per_cta > 0 ? cf.rebuild_tiles_per_cta : kDefaultRebuildTiles;
   if (ws == 0 && cf.fg_chunk_tiles > 0) {
     // fixed chunk length, but never more split items than the partial buffer holds
@@ -371,7 +373,7 @@ csr_status run_block(csr_ctx *c, int slot, int ws, const void *q, const void *k,
     ap.chunk_tiles = static_cast<int32_t>(std::max<int64_t>(cf.fg_chunk_tiles, min_c));
   } else {
     ap.chunk_tiles = choose_chunk_tiles(units, kv_max, c->fg_grid, ws == 0 ? 0 : tpc, cf.head_dim,
-                                        ap.unit_tiles);
+                                        ap.unit_tiles, ap.kv_tile);
   }
   const int64_t n_chunks = ceil_div(kv_max, ap.chunk_tiles);
   ap.n_items = static_cast<int32_t>(n_chunks * units);
@@ -395,6 +397,7 @@ csr_status run_block(csr_ctx *c, int slot, int ws, const void *q, const void *k,
     mp.n_tiles = ap.n_tiles;
     mp.chunk_tiles = ap.chunk_tiles;
     mp.unit_tiles = ap.unit_tiles;
+    mp.kv_tile = ap.kv_tile;
     mp.d = cf.head_dim;
     e = timed_launch(c, CSR_KERNEL_MERGE, fg, s, [&] { return launch_merge(mp, s); });
     if (e != cudaSuccess) return cuda_fail(c, e, "merge launch");
@@ -404,6 +407,8 @@ csr_status run_block(csr_ctx *c, int slot, int ws, const void *q, const void *k,
 }
 
 enum class Kind { Prefix, Chunk, Suffix };
+
+csr_status catch_up_now(csr_ctx *c);
 
 csr_status add_block(csr_ctx *c, Kind kind, const void *q, const void *k, const void *v,
                      int32_t n, void *out, float *lse, cudaStream_t s, int64_t *chunk_id) {
@@ -446,15 +451,16 @@ csr_status add_block(csr_ctx *c, Kind kind, const void *q, const void *k, const 
     case Kind::Chunk: A.chunks.push_back({id, n}); break;
     case Kind::Suffix: A.suffix_len = n; break;
   }
+  if (chunk_id) *chunk_id = id;
   if (fork) {
-    // Algorithm 1, Increment: fork the chunk into the buffer of the rebuild;
-    // its pages in the rebuilt version are reserved now (after the active ones).
+    // Algorithm 1, Increment: fork the chunk into the rebuild; its pages in
+    // the rebuilt version are reserved now (after the active ones).
     Version &B = c->pend();
     for (int64_t i = 0; i < needB; ++i) B.pages.push_back(c->pool.take());
     B.chunks.push_back({id, n});
     c->buffer.push_back({id, n});
+    if (c->cfg.n_catchup == 0) return catch_up_now(c);
   }
-  if (chunk_id) *chunk_id = id;
   return CSR_OK;
 }
 
@@ -491,6 +497,30 @@ csr_status materialise(csr_ctx *c, const std::vector<ChunkRec> &chunks, int ws, 
     if (st != CSR_OK) return st;
     c->rebuilt_len += ch.len;
   }
+  return CSR_OK;
+}
+
+// N_catchup = 0: Algorithm 1's reconcile loop drains the buffer completely
+// before the swap.  On one GPU the low-priority stream is R_2's queue, so each
+// chunk that arrives while reconciling is appended to X_eps on that stream as
+// soon as it is buffered (in arrival order); the swap happens at the first
+// poll after the stream has finished.  (Computing the buffer only when a poll
+// finds the previous round done would never drain it while one chunk arrives
+// per step.)
+csr_status catch_up_now(csr_ctx *c) {
+  std::vector<ChunkRec> batch;
+  batch.swap(c->buffer);
+  if (c->plan_only) {
+    for (const auto &ch : batch) c->rebuilt_len += ch.len;
+    return CSR_OK;
+  }
+  csr_status st = materialise(c, batch, 1, c->lo);
+  if (st != CSR_OK) {
+    abort_reconcile(c);
+    return st;
+  }
+  const cudaError_t e = cudaEventRecord(c->ev_rb, c->lo);
+  if (e != cudaSuccess) return cuda_fail(c, e, "recording the catch-up event");
   return CSR_OK;
 }
 
@@ -549,8 +579,9 @@ csr_status csr_create(const csr_config *cfg, void *k_pool, void *v_pool, void *w
     }
     c->fg_grid = cfg->num_ctas > 0 ? cfg->num_ctas : std::min(c->num_sms, c->lay.fg_cap);
     const uint64_t pool_rows = static_cast<uint64_t>(cfg->pool_pages) * cfg->num_kv_heads * cfg->page_size;
-    bool ok = encode_rows(&c->tm_k, k_pool, pool_rows, cfg->head_dim, cfg->page_size) &&
-              encode_rows(&c->tm_v, v_pool, pool_rows, cfg->head_dim, cfg->page_size);
+    const uint32_t kv_box = static_cast<uint32_t>(std::min(cfg->page_size, 64));
+    bool ok = encode_rows(&c->tm_k, k_pool, pool_rows, cfg->head_dim, kv_box) &&
+              encode_rows(&c->tm_v, v_pool, pool_rows, cfg->head_dim, kv_box);
     for (int i = 0; i < 2 && ok; ++i)
       ok = encode_rows(&c->tm_q[i], c->ws + c->lay.qpack[i],
                        static_cast<uint64_t>(cfg->num_kv_heads) * c->lay.rows_cap, cfg->head_dim, kBM);

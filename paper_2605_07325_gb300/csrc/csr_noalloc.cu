@@ -152,7 +152,8 @@ extern "C" csr_status csr_attend_block_noalloc(const csr_block_args *a, csr_stre
   AttnParams ap{};
   const uint64_t pool_rows = static_cast<uint64_t>(a->pool_pages) * hkv * P;
   if (!encode(&ap.tm_q, q_pack, static_cast<uint64_t>(hkv) * rows_cap, d, kBM) ||
-      !encode(&ap.tm_k, a->k_pool, pool_rows, d, P) || !encode(&ap.tm_v, a->v_pool, pool_rows, d, P))
+      !encode(&ap.tm_k, a->k_pool, pool_rows, d, P < 64 ? P : 64) ||
+      !encode(&ap.tm_v, a->v_pool, pool_rows, d, P < 64 ? P : 64))
     return CSR_ECUDA;
   ap.page_table = a->page_table;
   ap.out = static_cast<uint16_t *>(a->out);
@@ -171,10 +172,11 @@ extern "C" csr_status csr_attend_block_noalloc(const csr_block_args *a, csr_stre
   ap.n_pages_valid = static_cast<int32_t>(cdiv(a->L + a->n, P));
   ap.pool_pages = a->pool_pages;
   ap.unit_tiles = 2;
+  ap.kv_tile = kBN;
   const int T = kBM / g;
   const int64_t uph = cdiv(ap.n_tiles, 2);
   const int64_t units = uph * hkv;
-  const int64_t kv_max = unit_iters(a->L, a->n, T, static_cast<int32_t>(uph * 2 - 1));
+  const int64_t kv_max = unit_iters(a->L, a->n, T, static_cast<int32_t>(uph * 2 - 1), kBN);
   // Split the key range only as far as the static partial buffer allows:
   // one chunk per unit when there are enough units to fill the SMs, else
   // the most chunks (up to one wave) whose partials fit.
@@ -212,6 +214,7 @@ extern "C" csr_status csr_attend_block_noalloc(const csr_block_args *a, csr_stre
     mp.n_tiles = ap.n_tiles;
     mp.chunk_tiles = ap.chunk_tiles;
     mp.unit_tiles = 2;
+    mp.kv_tile = kBN;
     mp.d = d;
     if (launch_merge(mp, s) != cudaSuccess) return CSR_ECUDA;
   }

@@ -49,7 +49,8 @@ struct AttnParams {
   int64_t L;               // cached tokens before this call
   int32_t n, hq, hkv, group, page_size, rows_cap, n_tiles, n_pages_valid, pool_pages;
   int32_t chunk_tiles;     // key tiles per item
-  int32_t unit_tiles;      // query tiles per item: 1 (attn_kernel) or 2 (attn_pair_kernel)
+  int32_t unit_tiles;      // query tiles per item: 1 (attn_kernel) or 2 (pair / pipe kernels)
+  int32_t kv_tile;         // keys per key tile: 128, or 64 for attn_pipe_kernel
   int32_t n_items;         // n_chunks * hkv * units per head, numbered (chunk, head, unit)
   int32_t grid;            // CTAs; CTA c runs items c, c + grid, ...
   float scale_log2;        // softmax_scale * log2(e)
@@ -62,7 +63,7 @@ struct MergeParams {
   uint16_t *out;
   float *lse;
   int64_t L;
-  int32_t n, hq, hkv, group, n_tiles, chunk_tiles, unit_tiles, d;
+  int32_t n, hq, hkv, group, n_tiles, chunk_tiles, unit_tiles, kv_tile, d;
 };
 
 // K4: eviction / compaction: new version's page table from the free bitmap.
@@ -96,14 +97,19 @@ struct GatherParams {
 // Shared-memory bytes of the attention kernels for a head dim.
 size_t attn_smem_bytes(int head_dim);
 size_t attn_pair_smem_bytes(int head_dim);
+size_t attn_pipe_smem_bytes(int head_dim);
 
-// Key tiles of query tile `tile` (kBN keys each).
+// Key tiles (of `bn` keys) of query tile `tile`: its keys are [0, L + last token].
 __host__ __device__ inline int64_t unit_iters(int64_t L, int32_t n, int32_t tokens_per_tile,
-                                              int32_t tile) {
+                                              int32_t tile, int32_t bn = kBN) {
   int64_t hi = static_cast<int64_t>(tile + 1) * tokens_per_tile;
   if (hi > n) hi = n;
-  return (L + hi + kBN - 1) / kBN;
+  return (L + hi + bn - 1) / bn;
 }
+
+// Key tile of the pipelined kernel (attn_pipe_kernel): 64 keys, so two score
+// buffers per query tile fit TMEM next to the two output accumulators.
+constexpr int kBN64 = 64;
 
 cudaError_t launch_rope_append(const RopeAppendParams &p, cudaStream_t s);
 cudaError_t launch_attention(const AttnParams &p, int head_dim, cudaStream_t s);

@@ -132,20 +132,41 @@ __device__ __forceinline__ void load_o(uint32_t taddr, uint32_t (&o)[HD]) {
   else tmem_ld64_wait(taddr, o);
 }
 
-// Issue the TMA loads of one 128-key tile of `head` whose pages' physical ids
-// are phys[0 .. 128/P).
+// Issue the TMA loads of keys [key0, key0 + bn) of `head` into a 128B-swizzled
+// tile (box b of 64 columns at dst + b * bn * 128).  The copies are pieces of
+// min(P, 64) rows (the tensor maps' box height); `phys` holds the physical ids
+// of logical pages lp_base, lp_base + 1, ...
 template <int HD>
-__device__ __forceinline__ void load_kv_tile(const AttnParams &p, const CUtensorMap *map,
-                                             uint8_t *dst, uint64_t *bar, int head,
-                                             const int32_t *phys) {
+__device__ __forceinline__ void load_kv_keys(const AttnParams &p, const CUtensorMap *map,
+                                             uint8_t *dst, int bn, uint64_t *bar, int head,
+                                             const int32_t *phys, int64_t lp_base, int64_t key0) {
   const int P = p.page_size;
-  const int ppt = kBN / P;
-  for (int pp = 0; pp < ppt; ++pp) {
-    const int32_t row = (phys[pp] * p.hkv + head) * P;
+  const int seg = P < 64 ? P : 64;
+  for (int r = 0; r < bn; r += seg) {
+    const int64_t key = key0 + r;
+    const int64_t lp = key / P;
+    const int32_t row = (phys[lp - lp_base] * p.hkv + head) * P + static_cast<int32_t>(key - lp * P);
 #pragma unroll
-    for (int b = 0; b < AttnCfg<HD>::kBoxes; ++b)
-      tma_load_2d(dst + b * (kBN * 128) + pp * P * 128, map, bar, b * 64, row);
+    for (int b = 0; b < HD / 64; ++b) tma_load_2d(dst + b * (bn * 128) + r * 128, map, bar, b * 64, row);
   }
+}
+
+// Stage the physical ids of the logical pages covering key tiles [jb, je)
+// (tiles of bn keys) into `stage`, one id per page (whole producer warp).
+// Returns the first staged logical page.
+__device__ __forceinline__ int64_t stage_pages(const AttnParams &p, int32_t *stage, int bn,
+                                               int64_t jb, int64_t je, int lane) {
+  const int64_t lp0 = jb * bn / p.page_size;
+  const int64_t lp1 = (je * bn + p.page_size - 1) / p.page_size;
+  for (int64_t lp = lp0 + lane; lp < lp1; lp += 32) {
+    int32_t phys = (lp < p.n_pages_valid) ? p.page_table[lp] : p.page_table[0];
+    if (phys < 0 || phys >= p.pool_pages) {
+      atomicOr(p.err, CSR_DEVERR_BAD_PAGE);
+      phys = 0;
+    }
+    stage[lp - lp0] = phys;
+  }
+  return lp0;
 }
 
 template <int HD>
@@ -202,8 +223,8 @@ __global__ void __launch_bounds__(192, 1) attn_kernel(const __grid_constant__ At
     // (coalesced page-table reads off the critical path); lane 0 issues the
     // copies from there.
     int32_t *stage = reinterpret_cast<int32_t *>(smem + C::kPtOff);
-    const int ppt = kBN / p.page_size;
-    const int tiles_per_block = C::kPtStage / ppt;
+    // key tiles whose pages fit one staging block (a tile may end mid-page)
+    const int tiles_per_block = (C::kPtStage - 2) * p.page_size / kBN;
     uint32_t q_round = 0, k_it = 0, v_it = 0;
     bool ok = true;
     while (ok && walk.next(p, T, seg)) {
@@ -223,21 +244,12 @@ __global__ void __launch_bounds__(192, 1) attn_kernel(const __grid_constant__ At
       ok = __shfl_sync(0xffffffffu, ok, 0);
       for (int64_t jb = seg.j0; ok && jb < seg.j1; jb += tiles_per_block) {
         const int64_t je = min(jb + tiles_per_block, seg.j1);
-        const int npages = static_cast<int>(je - jb) * ppt;
         __syncwarp();
-        for (int i = lane; i < npages; i += 32) {
-          const int64_t lp = jb * ppt + i;
-          int32_t phys = (lp < p.n_pages_valid) ? p.page_table[lp] : p.page_table[0];
-          if (phys < 0 || phys >= p.pool_pages) {
-            atomicOr(p.err, CSR_DEVERR_BAD_PAGE);
-            phys = 0;
-          }
-          stage[i] = phys;
-        }
+        const int64_t lp_base = stage_pages(p, stage, kBN, jb, je, lane);
         __syncwarp();
         if (lane == 0) {
           for (int64_t j = jb; j < je; ++j) {
-            const int32_t *phys = stage + static_cast<int>(j - jb) * ppt;
+
             const int ks = k_it % C::kStages;
             if (!mbar_wait(&bars->k_empty[ks], ((k_it / C::kStages) & 1) ^ 1, abort, p.err,
                            CSR_DEVERR_WAIT_TIMEOUT)) {
@@ -245,8 +257,8 @@ __global__ void __launch_bounds__(192, 1) attn_kernel(const __grid_constant__ At
               break;
             }
             mbar_arrive_expect_tx(&bars->k_full[ks], C::kTileBytes);
-            load_kv_tile<HD>(p, &p.tm_k, smem + C::kKOff + ks * C::kTileBytes, &bars->k_full[ks],
-                             seg.head, phys);
+            load_kv_keys<HD>(p, &p.tm_k, smem + C::kKOff + ks * C::kTileBytes, kBN, &bars->k_full[ks],
+                             seg.head, stage, lp_base, j * kBN);
             ++k_it;
             const int vs = v_it % C::kStages;
             if (!mbar_wait(&bars->v_empty[vs], ((v_it / C::kStages) & 1) ^ 1, abort, p.err,
@@ -255,8 +267,8 @@ __global__ void __launch_bounds__(192, 1) attn_kernel(const __grid_constant__ At
               break;
             }
             mbar_arrive_expect_tx(&bars->v_full[vs], C::kTileBytes);
-            load_kv_tile<HD>(p, &p.tm_v, smem + C::kVOff + vs * C::kTileBytes, &bars->v_full[vs],
-                             seg.head, phys);
+            load_kv_keys<HD>(p, &p.tm_v, smem + C::kVOff + vs * C::kTileBytes, kBN, &bars->v_full[vs],
+                             seg.head, stage, lp_base, j * kBN);
             ++v_it;
           }
         }
@@ -544,7 +556,7 @@ struct PairWalker {
       const int32_t rem = it - k * units;
       const int32_t head = rem / n_pairs;
       const int32_t pair = rem - head * n_pairs;
-      const int64_t kv = unit_iters(p.L, p.n, T, 2 * pair + 1);
+      const int64_t kv = unit_iters(p.L, p.n, T, 2 * pair + 1, p.kv_tile);
       const int64_t j0 = static_cast<int64_t>(k) * p.chunk_tiles;
       if (j0 >= kv) continue;
       s.head = head;
@@ -609,8 +621,8 @@ __global__ void __launch_bounds__(320, 1) attn_pair_kernel(const __grid_constant
   if (warp == 8) {
     // ------------------------------------------------------ TMA producer
     int32_t *stage = reinterpret_cast<int32_t *>(smem + C::kPtOff);
-    const int ppt = kBN / p.page_size;
-    const int tiles_per_block = C::kPtStage / ppt;
+    // key tiles whose pages fit one staging block (a tile may end mid-page)
+    const int tiles_per_block = (C::kPtStage - 2) * p.page_size / kBN;
     uint32_t q_round = 0, k_it = 0, v_it = 0;
     bool ok = true;
     while (ok && walk.next(p, T, seg)) {
@@ -633,21 +645,12 @@ __global__ void __launch_bounds__(320, 1) attn_pair_kernel(const __grid_constant
       ok = __shfl_sync(0xffffffffu, ok, 0);
       for (int64_t jb = seg.j0; ok && jb < seg.j1; jb += tiles_per_block) {
         const int64_t je = min(jb + tiles_per_block, seg.j1);
-        const int npages = static_cast<int>(je - jb) * ppt;
         __syncwarp();
-        for (int i = lane; i < npages; i += 32) {
-          const int64_t lp = jb * ppt + i;
-          int32_t phys = (lp < p.n_pages_valid) ? p.page_table[lp] : p.page_table[0];
-          if (phys < 0 || phys >= p.pool_pages) {
-            atomicOr(p.err, CSR_DEVERR_BAD_PAGE);
-            phys = 0;
-          }
-          stage[i] = phys;
-        }
+        const int64_t lp_base = stage_pages(p, stage, kBN, jb, je, lane);
         __syncwarp();
         if (lane == 0) {
           for (int64_t j = jb; j < je; ++j) {
-            const int32_t *phys = stage + static_cast<int>(j - jb) * ppt;
+
             const int ks = k_it % C::kStages;
             if (!mbar_wait(&bars->k_empty[ks], ((k_it / C::kStages) & 1) ^ 1, abort, p.err,
                            CSR_DEVERR_WAIT_TIMEOUT)) {
@@ -655,8 +658,8 @@ __global__ void __launch_bounds__(320, 1) attn_pair_kernel(const __grid_constant
               break;
             }
             mbar_arrive_expect_tx(&bars->k_full[ks], C::kTileBytes);
-            load_kv_tile<HD>(p, &p.tm_k, smem + C::kKOff + ks * C::kTileBytes, &bars->k_full[ks],
-                             seg.head, phys);
+            load_kv_keys<HD>(p, &p.tm_k, smem + C::kKOff + ks * C::kTileBytes, kBN, &bars->k_full[ks],
+                             seg.head, stage, lp_base, j * kBN);
             ++k_it;
             const int vs = v_it % C::kStages;
             if (!mbar_wait(&bars->v_empty[vs], ((v_it / C::kStages) & 1) ^ 1, abort, p.err,
@@ -665,8 +668,8 @@ __global__ void __launch_bounds__(320, 1) attn_pair_kernel(const __grid_constant
               break;
             }
             mbar_arrive_expect_tx(&bars->v_full[vs], C::kTileBytes);
-            load_kv_tile<HD>(p, &p.tm_v, smem + C::kVOff + vs * C::kTileBytes, &bars->v_full[vs],
-                             seg.head, phys);
+            load_kv_keys<HD>(p, &p.tm_v, smem + C::kVOff + vs * C::kTileBytes, kBN, &bars->v_full[vs],
+                             seg.head, stage, lp_base, j * kBN);
             ++v_it;
           }
         }
@@ -896,6 +899,410 @@ __global__ void __launch_bounds__(320, 1) attn_pair_kernel(const __grid_constant
   }
 }
 
+// ============================================================ pipelined two-tile kernel
+// Two 128-row query tiles per CTA as in attn_pair_kernel, but 64-key tiles,
+// which leaves TMEM room for two score buffers per query tile:
+//   S_A0 [0,64) S_A1 [64,128) S_B0 [128,192) S_B1 [192,256)  O_A [256,256+d)  O_B [..+d)
+// The MMA issuer runs two key tiles ahead: while softmax works on tile i of a
+// query tile, the scores of tile i+1 already sit in the other buffer, so a
+// softmax warpgroup never waits for the tensor core between its tiles.  Issue
+// order per key tile i:  PV_A(i), S_A(i+2), PV_B(i), S_B(i+2)  (S_X(i+2) reuses
+// the buffer PV_X(i) has just read, in issue order).
+template <int HD>
+struct PipeCfg {
+  static constexpr int kStages = (HD == 64) ? 8 : 4;
+  static constexpr int kBoxes = HD / 64;
+  static constexpr int kQBytes = kBM * HD * 2;                 // one query tile
+  static constexpr int kTileBytes = kBN64 * HD * 2;            // one 64-key K or V tile
+  static constexpr int kQOff = 0;
+  static constexpr int kKOff = 2 * kQBytes;
+  static constexpr int kVOff = kKOff + kStages * kTileBytes;
+  static constexpr int kBarOff = kVOff + kStages * kTileBytes;
+  static constexpr int kPtOff = kBarOff + 1024;
+  static constexpr int kPtStage = 512;
+  static constexpr int kSmem = kPtOff + kPtStage * 4 + 1024;
+  static constexpr uint32_t kTmemCols = 512;
+  static constexpr uint32_t kOCol = 4 * kBN64;
+};
+
+struct PipeBars {
+  uint64_t q_full, q_empty;
+  uint64_t k_full[8], k_empty[8], v_full[8], v_empty[8];
+  uint64_t s_full[2][2], p_full[2][2];   // [query tile][score buffer]
+  uint64_t o_done[2], o_final[2], o_free[2];
+  uint64_t drain;
+  uint32_t tmem_base;
+  int abort;
+};
+
+size_t attn_pipe_smem_bytes(int head_dim) {
+  return head_dim == 64 ? PipeCfg<64>::kSmem : PipeCfg<128>::kSmem;
+}
+
+template <int HD>
+__global__ void __launch_bounds__(320, 1) attn_pipe_kernel(const __grid_constant__ AttnParams p) {
+  using C = PipeCfg<HD>;
+  constexpr int BN = kBN64;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t *smem = reinterpret_cast<uint8_t *>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  PipeBars *bars = reinterpret_cast<PipeBars *>(smem + C::kBarOff);
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const int T = kBM / p.group;
+
+  if (threadIdx.x == 0) {
+    mbar_init(&bars->q_full, 1);
+    mbar_init(&bars->q_empty, 1);
+    for (int s = 0; s < C::kStages; ++s) {
+      mbar_init(&bars->k_full[s], 1);
+      mbar_init(&bars->k_empty[s], 1);
+      mbar_init(&bars->v_full[s], 1);
+      mbar_init(&bars->v_empty[s], 1);
+    }
+    for (int w = 0; w < 2; ++w) {
+      for (int b = 0; b < 2; ++b) {
+        mbar_init(&bars->s_full[w][b], 1);
+        mbar_init(&bars->p_full[w][b], 128);
+      }
+      mbar_init(&bars->o_done[w], 1);
+      mbar_init(&bars->o_final[w], 1);
+      mbar_init(&bars->o_free[w], 128);
+    }
+    mbar_init(&bars->drain, 1);
+    bars->abort = 0;
+    fence_barrier_init();
+  }
+  if (warp == 8 && lane == 0) {
+    tma_prefetch_desc(&p.tm_q);
+    tma_prefetch_desc(&p.tm_k);
+    tma_prefetch_desc(&p.tm_v);
+  }
+  if (warp == 9) {
+    tmem_alloc(&bars->tmem_base, C::kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = bars->tmem_base;
+  volatile int *abort = &bars->abort;
+  PairWalker walk{static_cast<int32_t>(blockIdx.x)};
+  Seg seg;
+
+  if (warp == 8) {
+    // ------------------------------------------------------ TMA producer
+    // Order per item: K(0), K(1), then for each i: K(i+2), V(i) -- the MMA
+    // issuer consumes keys two tiles ahead of values.
+    int32_t *stage = reinterpret_cast<int32_t *>(smem + C::kPtOff);
+    const int tiles_per_block = (C::kPtStage - 2) * p.page_size / BN;
+    uint32_t q_round = 0, k_it = 0, v_it = 0;
+    bool ok = true;
+    auto load_k = [&](int64_t j, int64_t lp_base) {
+      const int ks = k_it % C::kStages;
+      if (!mbar_wait(&bars->k_empty[ks], ((k_it / C::kStages) & 1) ^ 1, abort, p.err,
+                     CSR_DEVERR_WAIT_TIMEOUT))
+        return false;
+      mbar_arrive_expect_tx(&bars->k_full[ks], C::kTileBytes);
+      load_kv_keys<HD>(p, &p.tm_k, smem + C::kKOff + ks * C::kTileBytes, BN, &bars->k_full[ks],
+                       seg.head, stage, lp_base, j * BN);
+      ++k_it;
+      return true;
+    };
+    auto load_v = [&](int64_t j, int64_t lp_base) {
+      const int vs = v_it % C::kStages;
+      if (!mbar_wait(&bars->v_empty[vs], ((v_it / C::kStages) & 1) ^ 1, abort, p.err,
+                     CSR_DEVERR_WAIT_TIMEOUT))
+        return false;
+      mbar_arrive_expect_tx(&bars->v_full[vs], C::kTileBytes);
+      load_kv_keys<HD>(p, &p.tm_v, smem + C::kVOff + vs * C::kTileBytes, BN, &bars->v_full[vs],
+                       seg.head, stage, lp_base, j * BN);
+      ++v_it;
+      return true;
+    };
+    while (ok && walk.next(p, T, seg)) {
+      if (lane == 0) {
+        if (q_round > 0 && !mbar_wait(&bars->q_empty, (q_round - 1) & 1, abort, p.err,
+                                      CSR_DEVERR_WAIT_TIMEOUT)) {
+          ok = false;
+        } else {
+          mbar_arrive_expect_tx(&bars->q_full, 2 * C::kQBytes);
+          const int32_t qrow = seg.head * p.rows_cap + seg.tile * 2 * kBM;
+#pragma unroll
+          for (int h = 0; h < 2; ++h)
+#pragma unroll
+            for (int b = 0; b < C::kBoxes; ++b)
+              tma_load_2d(smem + C::kQOff + h * C::kQBytes + b * (kBM * 128), &p.tm_q,
+                          &bars->q_full, b * 64, qrow + h * kBM);
+          ++q_round;
+        }
+      }
+      ok = __shfl_sync(0xffffffffu, ok, 0);
+      // Stage blocks of key tiles; V of a block's first two tiles may trail
+      // into the next block, so each block stages its pages plus the two
+      // tiles before it.
+      for (int64_t jb = seg.j0; ok && jb < seg.j1; jb += tiles_per_block - 2) {
+        const int64_t je = min(jb + tiles_per_block - 2, seg.j1);
+        const int64_t sb = max(seg.j0, jb - 2);
+        __syncwarp();
+        const int64_t lp_base = stage_pages(p, stage, BN, sb, je, lane);
+        __syncwarp();
+        if (lane == 0) {
+          for (int64_t j = jb; j < je && ok; ++j) {
+            // K(j) is loaded in the step of V(j - 2); the first two K tiles lead
+            if (j < seg.j0 + 2) {
+              ok = load_k(j, lp_base);
+              continue;
+            }
+            ok = load_k(j, lp_base) && load_v(j - 2, lp_base);
+          }
+          if (ok && je == seg.j1) {
+            // values of the last two tiles
+            for (int64_t j = max(seg.j0, seg.j1 - 2); j < seg.j1 && ok; ++j) ok = load_v(j, lp_base);
+          }
+        }
+        ok = __shfl_sync(0xffffffffu, ok, 0);
+      }
+    }
+    if (!ok && lane == 0) {
+      if (q_round > 0) drain_wait(&bars->q_full, (q_round - 1) & 1);
+      for (uint32_t i = (k_it > C::kStages ? k_it - C::kStages : 0); i < k_it; ++i)
+        drain_wait(&bars->k_full[i % C::kStages], (i / C::kStages) & 1);
+      for (uint32_t i = (v_it > C::kStages ? v_it - C::kStages : 0); i < v_it; ++i)
+        drain_wait(&bars->v_full[i % C::kStages], (i / C::kStages) & 1);
+    }
+  } else if (warp == 9) {
+    if (lane == 0) {
+      // ------------------------------------------------------ MMA issuer
+      constexpr uint32_t idesc_s = idesc_bf16_f32(kBM, BN, false, false);
+      constexpr uint32_t idesc_pv = idesc_bf16_f32(kBM, HD, false, true);
+      const uint32_t q_base = smem_u32(smem + C::kQOff);
+      const uint32_t k_base = smem_u32(smem + C::kKOff);
+      const uint32_t v_base = smem_u32(smem + C::kVOff);
+      uint32_t q_round = 0, k_it = 0, v_it = 0, seg_n = 0;
+      uint32_t p_cnt[2][2] = {{0, 0}, {0, 0}};
+      bool ok = true;
+      auto wait = [&](uint64_t *bar, uint32_t parity) {
+        if (ok && !mbar_wait(bar, parity, abort, p.err, CSR_DEVERR_WAIT_TIMEOUT)) ok = false;
+        return ok;
+      };
+      auto issue_s = [&](int x, int buf, int ks) {
+        const uint32_t qx = q_base + x * C::kQBytes;
+        const uint32_t kst = k_base + ks * C::kTileBytes;
+#pragma unroll
+        for (int kk = 0; kk < HD / 16; ++kk) {
+          const uint64_t a = sdesc_sw128(qx + (kk >> 2) * (kBM * 128) + (kk & 3) * 32, 16, 1024);
+          const uint64_t b = sdesc_sw128(kst + (kk >> 2) * (BN * 128) + (kk & 3) * 32, 16, 1024);
+          mma_bf16_ss(tmem + (2 * x + buf) * BN, a, b, idesc_s, kk > 0 ? 1u : 0u);
+        }
+        mma_commit(&bars->s_full[x][buf]);
+      };
+      auto issue_pv = [&](int x, int buf, int vs, bool first) {
+        const uint32_t vst = v_base + vs * C::kTileBytes;
+#pragma unroll
+        for (int kk = 0; kk < BN / 16; ++kk) {
+          const uint64_t b = sdesc_sw128(vst + kk * (16 * 128), BN * 128, 1024);
+          mma_bf16_ts(tmem + C::kOCol + x * HD, tmem + (2 * x + buf) * BN + kk * 8, b, idesc_pv,
+                      (!first || kk > 0) ? 1u : 0u);
+        }
+      };
+      while (ok && walk.next(p, T, seg)) {
+        if (!wait(&bars->q_full, q_round & 1)) break;
+        ++q_round;
+        tc_fence_after();
+        const int nj = static_cast<int>(seg.j1 - seg.j0);
+        const int lead = nj < 2 ? nj : 2;
+        for (int t = 0; t < lead && ok; ++t) {
+          const int ks = k_it % C::kStages;
+          if (!wait(&bars->k_full[ks], (k_it / C::kStages) & 1)) break;
+          tc_fence_after();
+          issue_s(0, t, ks);
+          issue_s(1, t, ks);
+          mma_commit(&bars->k_empty[ks]);
+          ++k_it;
+        }
+        if (!ok) break;
+        if (nj <= 2) mma_commit(&bars->q_empty);
+        for (int i = 0; i < nj; ++i) {
+          const int buf = i & 1;
+          const int vs = v_it % C::kStages;
+          const bool more = i + 2 < nj;
+          int ks = 0;
+          // ---- tile A
+          if (!wait(&bars->p_full[0][buf], p_cnt[0][buf] & 1)) break;
+          ++p_cnt[0][buf];
+          if (!wait(&bars->v_full[vs], (v_it / C::kStages) & 1)) break;
+          if (i == 0 && seg_n > 0 && !wait(&bars->o_free[0], (seg_n & 1) ^ 1)) break;
+          tc_fence_after();
+          issue_pv(0, buf, vs, i == 0);
+          mma_commit(&bars->o_done[0]);
+          if (i == nj - 1) mma_commit(&bars->o_final[0]);
+          if (more) {
+            ks = k_it % C::kStages;
+            if (!wait(&bars->k_full[ks], (k_it / C::kStages) & 1)) break;
+            tc_fence_after();
+            issue_s(0, buf, ks);
+          }
+          // ---- tile B
+          if (!wait(&bars->p_full[1][buf], p_cnt[1][buf] & 1)) break;
+          ++p_cnt[1][buf];
+          if (i == 0 && seg_n > 0 && !wait(&bars->o_free[1], (seg_n & 1) ^ 1)) break;
+          tc_fence_after();
+          issue_pv(1, buf, vs, i == 0);
+          mma_commit(&bars->o_done[1]);
+          if (i == nj - 1) mma_commit(&bars->o_final[1]);
+          mma_commit(&bars->v_empty[vs]);
+          ++v_it;
+          if (more) {
+            issue_s(1, buf, ks);
+            mma_commit(&bars->k_empty[ks]);
+            ++k_it;
+            if (i + 2 == nj - 1) mma_commit(&bars->q_empty);
+          }
+        }
+        ++seg_n;
+      }
+      if (!ok) {
+        mma_commit(&bars->drain);
+        drain_wait(&bars->drain, 0);
+      }
+    }
+  } else {
+    // ------------------------------------------------------ softmax warpgroups
+    const int wg = warp >> 2;
+    const int row = threadIdx.x - wg * 128;
+    const uint32_t lane_base = static_cast<uint32_t>((warp & 3) * 32) << 16;
+    const uint32_t o_col = C::kOCol + wg * HD;
+    uint32_t s_cnt[2] = {0, 0};
+    uint32_t g_tiles = 0, seg_n = 0;   // tiles (= PVs) of this warpgroup so far, items
+    bool ok = true;
+    while (ok && walk.next(p, T, seg)) {
+      const int tile = seg.tile * 2 + wg;
+      const int64_t t = static_cast<int64_t>(tile) * T + row / p.group;
+      const bool valid = tile < p.n_tiles && t < p.n;
+      const int64_t limit = valid ? p.L + t : -1;
+      float m_ref = -CUDART_INF_F;
+      float l = 0.f;
+      const int nj = static_cast<int>(seg.j1 - seg.j0);
+      for (int i = 0; i < nj; ++i) {
+        const int buf = i & 1;
+        const uint32_t s_col = (2 * wg + buf) * BN;
+        const int64_t j = seg.j0 + i;
+        const bool got = mbar_wait(&bars->s_full[wg][buf], s_cnt[buf] & 1, abort, p.err,
+                                   CSR_DEVERR_WAIT_TIMEOUT);
+        ++s_cnt[buf];
+        if (!__all_sync(0xffffffffu, got)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        uint32_t sr[BN];
+        tmem_ld64_wait(tmem + lane_base + s_col, sr);
+        float s[BN];
+#pragma unroll
+        for (int c = 0; c < BN; ++c) s[c] = __uint_as_float(sr[c]);
+        const int64_t key0 = j * BN;
+        if (key0 + BN - 1 > limit) {
+#pragma unroll
+          for (int c = 0; c < BN; ++c)
+            if (key0 + c > limit) s[c] = -CUDART_INF_F;
+        }
+        float mp[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) mp[e] = s[e];
+#pragma unroll
+        for (int c = 8; c < BN; ++c) mp[c & 7] = fmaxf(mp[c & 7], s[c]);
+        const float mx = fmaxf(fmaxf(fmaxf(mp[0], mp[1]), fmaxf(mp[2], mp[3])),
+                               fmaxf(fmaxf(mp[4], mp[5]), fmaxf(mp[6], mp[7])));
+        const float mx_s = mx * p.scale_log2;
+        const bool need = mx_s > m_ref + 8.0f;
+        const float m_new = need ? mx_s : m_ref;
+        const float alpha = need ? ex2_approx(m_ref - m_new) : 1.0f;
+        const bool had_mass = l > 0.f;
+        l *= alpha;
+        m_ref = m_new;
+        const float m_use = (m_ref == -CUDART_INF_F) ? 0.f : m_ref;
+        float rp[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) rp[e] = 0.f;
+        uint32_t pk[BN / 2];
+#pragma unroll
+        for (int c = 0; c < BN; c += 2) {
+          const float p0 = ex2_approx(fmaf(s[c], p.scale_log2, -m_use));
+          const float p1 = ex2_approx(fmaf(s[c + 1], p.scale_log2, -m_use));
+          rp[(c >> 1) & 7] += p0 + p1;
+          pk[c / 2] = pack_bf16x2(p0, p1);
+        }
+        l += ((rp[0] + rp[1]) + (rp[2] + rp[3])) + ((rp[4] + rp[5]) + (rp[6] + rp[7]));
+        tmem_st32(tmem + lane_base + s_col, pk);
+        if (i > 0 && __any_sync(0xffffffffu, need && had_mass)) {
+          // the previous tile's PV must land before O is rescaled
+          const bool got_o = mbar_wait(&bars->o_done[wg], (g_tiles - 1) & 1, abort, p.err,
+                                       CSR_DEVERR_WAIT_TIMEOUT);
+          if (!__all_sync(0xffffffffu, got_o)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          rescale_o<HD>(tmem + lane_base + o_col, alpha);
+        }
+        tmem_st_wait();
+        tc_fence_before();
+        mbar_arrive(&bars->p_full[wg][buf]);
+        ++g_tiles;
+      }
+      if (!ok) break;
+      // ---------------------------------------------------- epilogue
+      const bool got_o = mbar_wait(&bars->o_final[wg], seg_n & 1, abort, p.err,
+                                   CSR_DEVERR_WAIT_TIMEOUT);
+      if (!__all_sync(0xffffffffu, got_o)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      const float inv_l = l > 0.f ? 1.0f / l : 0.f;
+      const float lse2 = l > 0.f ? m_ref + log2f(l) : -CUDART_INF_F;
+      uint32_t o[HD];
+      load_o<HD>(tmem + lane_base + o_col, o);
+      if (seg.complete) {
+        if (valid) {
+          const int hq_idx = seg.head * p.group + row % p.group;
+          uint16_t *dst = p.out + (static_cast<int64_t>(t) * p.hq + hq_idx) * HD;
+#pragma unroll
+          for (int q8 = 0; q8 < HD / 8; ++q8) {
+            uint32_t w[4];
+#pragma unroll
+            for (int c = 0; c < 4; ++c)
+              w[c] = pack_bf16x2(__uint_as_float(o[q8 * 8 + 2 * c]) * inv_l,
+                                 __uint_as_float(o[q8 * 8 + 2 * c + 1]) * inv_l);
+            reinterpret_cast<uint4 *>(dst)[q8] = make_uint4(w[0], w[1], w[2], w[3]);
+          }
+          if (p.lse) p.lse[static_cast<int64_t>(hq_idx) * p.n + t] = lse2 * 0.69314718055994531f;
+        }
+      } else {
+        const int64_t base = static_cast<int64_t>(seg.item) * (2 * kBM) + wg * kBM + row;
+        float4 *d4 = reinterpret_cast<float4 *>(p.part_o + base * HD);
+#pragma unroll
+        for (int c = 0; c < HD / 4; ++c)
+          d4[c] = make_float4(__uint_as_float(o[4 * c]) * inv_l, __uint_as_float(o[4 * c + 1]) * inv_l,
+                              __uint_as_float(o[4 * c + 2]) * inv_l, __uint_as_float(o[4 * c + 3]) * inv_l);
+        p.part_lse[base] = lse2;
+      }
+      tc_fence_before();
+      mbar_arrive(&bars->o_free[wg]);
+      ++seg_n;
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 9) {
+    __syncwarp();
+    tc_fence_after();
+    tmem_dealloc(tmem, C::kTmemCols);
+  }
+}
+
 // ------------------------------------------------------------------ K3 merge
 // Merge the key-chunk pieces of one row: lse = log2 sum_k 2^lse_k and
 // O = sum_k 2^(lse_k - lse) O_k (each O_k already normalised by its own sum).
@@ -909,7 +1316,7 @@ __global__ void __launch_bounds__(256) merge_kernel(const __grid_constant__ Merg
   const int uph = (p.n_tiles + p.unit_tiles - 1) / p.unit_tiles;  // units per head
   const int unit = tile / p.unit_tiles;
   const int half = tile - unit * p.unit_tiles;
-  const int64_t kv = unit_iters(p.L, p.n, T, unit * p.unit_tiles + p.unit_tiles - 1);
+  const int64_t kv = unit_iters(p.L, p.n, T, unit * p.unit_tiles + p.unit_tiles - 1, p.kv_tile);
   const int nk = static_cast<int>((kv + p.chunk_tiles - 1) / p.chunk_tiles);
   if (nk <= 1) return;  // written whole by the attention kernel
   const int r = blockIdx.y * 8 + warp;
@@ -968,15 +1375,22 @@ cudaError_t attn_configure(int head_dim) {
   if (head_dim == 64) {
     e = cudaFuncSetAttribute(attn_kernel<64>, attr, AttnCfg<64>::kSmem);
     if (e == cudaSuccess) e = cudaFuncSetAttribute(attn_pair_kernel<64>, attr, PairCfg<64>::kSmem);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(attn_pipe_kernel<64>, attr, PipeCfg<64>::kSmem);
   } else {
     e = cudaFuncSetAttribute(attn_kernel<128>, attr, AttnCfg<128>::kSmem);
     if (e == cudaSuccess) e = cudaFuncSetAttribute(attn_pair_kernel<128>, attr, PairCfg<128>::kSmem);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(attn_pipe_kernel<128>, attr, PipeCfg<128>::kSmem);
   }
   return e;
 }
 
 cudaError_t launch_attention(const AttnParams &p, int head_dim, cudaStream_t s) {
-  if (p.unit_tiles == 2) {
+  if (p.unit_tiles == 2 && p.kv_tile == kBN64) {
+    if (head_dim == 64)
+      attn_pipe_kernel<64><<<p.grid, 320, PipeCfg<64>::kSmem, s>>>(p);
+    else
+      attn_pipe_kernel<128><<<p.grid, 320, PipeCfg<128>::kSmem, s>>>(p);
+  } else if (p.unit_tiles == 2) {
     if (head_dim == 64)
       attn_pair_kernel<64><<<p.grid, 320, PairCfg<64>::kSmem, s>>>(p);
     else

@@ -163,10 +163,13 @@ def test_rewind_then_append_matches_never_appended(libcsr):
 
 @pytest.mark.parametrize("shape", [C1, C2], ids=["d64_p16_g4", "d128_p64_g16"])
 @pytest.mark.parametrize("chunk_tiles", [0, 2])
-def test_single_tile_kernel_matches_oracle(libcsr, shape, chunk_tiles):
-    """The one-tile-per-CTA kernel (CSR_FLAG_SINGLE_TILE) stays correct too."""
+@pytest.mark.parametrize("kernel", ["single", "pipe64"])
+def test_other_kernel_designs_match_oracle(libcsr, shape, chunk_tiles, kernel):
+    """The one-tile-per-CTA kernel (CSR_FLAG_SINGLE_TILE) and the 64-key-tile
+    pipelined kernel (CSR_FLAG_PIPE_64) stay correct too."""
+    flags = libcsr.FLAG_SINGLE_TILE if kernel == "single" else libcsr.FLAG_PIPE_64
     p = Pair(shape, pool_pages=128, max_seq=4096, max_new=512, fg_chunk_tiles=chunk_tiles,
-             flags=libcsr.FLAG_SINGLE_TILE)
+             flags=flags)
     p.init_static(p.blk(10, 37))
     for i, n in enumerate([1, 129, 300]):
         p.append(p.blk(11 + i, n))

@@ -88,8 +88,10 @@ def test_reconcile_state_machine_matches_oracle(libcsr, prefix, n_catchup):
     m.o.reconcile()
     _same(ctx, m, libcsr)
     assert ctx.poll_swap() == libcsr.RECON_IDLE
-    # catch-up rounds: n_catchup=0 drains the 2 buffered chunks on the low stream first
-    assert states[0] == (libcsr.RECON_RUNNING if n_catchup == 0 else libcsr.RECON_RUNNING)
+    # n_catchup = 0 computes each arriving chunk at once, so the first poll swaps;
+    # n_catchup = 1 first catches up the 2 buffered chunks, then swaps
+    assert states == ([libcsr.RECON_SWAPPED] if n_catchup == 0
+                      else [libcsr.RECON_RUNNING, libcsr.RECON_SWAPPED])
 
 
 def test_swap_waits_for_live_suffix(libcsr):
