@@ -248,7 +248,8 @@ def run_ours(args):
     cfg = csr.make_config(HQ, HKV, D, P, BASE, max_new_tokens=PREFIX, pool_pages=pool_pages,
                           max_seq_tokens=max_tokens + P,
                           flags={"pair": 0, "pipe": csr.FLAG_PIPE_64,
-                                 "single": csr.FLAG_SINGLE_TILE}[args.kernel])
+                                 "single": csr.FLAG_SINGLE_TILE}[args.kernel] |
+                          (csr.FLAG_SEPARATE_MERGE if args.separate_merge else 0))
     stream = torch.cuda.Stream(device=dev, priority=-1)
     gen = torch.Generator(device=dev).manual_seed(1234 + rank)
 
@@ -540,6 +541,77 @@ def run_asr(args):
     return 0 if layout_ok and flags == 0 else 1
 
 
+# ------------------------------------------------------------- unordered leg
+def run_unordered(args):
+    """Per-layer analogue of the paper's unordered baseline (Table II,
+    'Unord.'): the whole prompt is dynamic, so every step recomputes the
+    cache from scratch -- a causal prefill of the 4,096-token prefix, the
+    chunks and the 512-token suffix (123,648 tokens, in 4,096-token blocks) --
+    against the CSR step (append 256 + attend 512 + truncate over 122,880
+    cached tokens) measured in the same run."""
+    import torch
+    from paper_2605_07325_gb300 import costmodel, csr
+
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    total = L0 + CHUNK + SUFFIX
+    cfg = csr.make_config(HQ, HKV, D, P, BASE, max_new_tokens=4096,
+                          pool_pages=total // P + 16, max_seq_tokens=total + P)
+    stream = torch.cuda.Stream(device=dev, priority=-1)
+    gen = torch.Generator(device=dev).manual_seed(777)
+
+    def rnd(n, h):
+        return torch.randn((n, h, D), generator=gen, device=dev, dtype=torch.float32).to(torch.bfloat16)
+
+    blocks = []
+    left = total
+    while left > 0:
+        n = min(4096, left)
+        blocks.append((rnd(n, HQ), rnd(n, HKV), rnd(n, HKV),
+                       torch.empty((n, HQ, D), dtype=torch.bfloat16, device=dev)))
+        left -= n
+    times = []
+    with torch.cuda.stream(stream):
+        for step in range(args.warmup + max(1, args.steps // 100)):
+            ctx = csr.Context(cfg, device=str(dev), stream=stream)
+            stream.synchronize()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            q, k, v, o = blocks[0]
+            ctx.init_static(q, k, v, out=o, stream=stream)
+            for q, k, v, o in blocks[1:]:
+                ctx.append_chunk(q, k, v, out=o, stream=stream)
+            e1.record(stream)
+            stream.synchronize()
+            if step >= args.warmup:
+                times.append(e0.elapsed_time(e1))
+            assert ctx.device_status() == 0
+            ctx.close()
+    unordered_ms = statistics.mean(times)
+    flops = costmodel.attention_flops(HQ, D, 0, total)
+    line = {"workload": "unordered baseline: full causal prefill of 123,648 tokens per step, "
+                        "64 q / 4 kv heads, d 128, page 64, bf16, 1 layer",
+            "unordered_ms_per_layer": unordered_ms, "steps": len(times),
+            "tflops": flops / (unordered_ms * 1e-3) / 1e12,
+            "note": "compare with the CSR step (value of the default bench line) measured "
+                    "in the same process below"}
+    csr_args = argparse.Namespace(**vars(args))
+    csr_args.no_cpu_baseline = True
+    csr_args.steps = min(args.steps, 100)
+    import io
+    import contextlib
+    buf = io.StringIO()
+    with contextlib.redirect_stdout(buf):
+        run_ours(csr_args)
+    csr_line = json.loads(buf.getvalue().strip().splitlines()[-1])
+    line["csr_us_per_layer"] = csr_line["value"]
+    line["speedup_csr_over_unordered"] = unordered_ms * 1e3 / csr_line["value"]
+    line["paper_context"] = ("paper Table II, 120K tokens: unordered 14.67 s vs CSR M=1024 0.56 s "
+                             "(26x), end-to-end TTFT of a 235B model on 4xH100")
+    print(json.dumps(line), flush=True)
+    return 0
+
+
 # ---------------------------------------------------------------- sweep leg
 SWEEP_L = (16384, 32768, 65536, 98304, 131072)
 SWEEP_N = (16, 64, 256, 1024, 4096)
@@ -624,6 +696,8 @@ def main(argv=None):
                     help="attention kernel: pair (default: two query tiles per CTA, 128-key "
                          "tiles), pipe (two query tiles, 64-key tiles, two score buffers each), "
                          "single (one query tile per CTA)")
+    ap.add_argument("--separate-merge", action="store_true",
+                    help="merge split-KV partials in a separate kernel (default: fused)")
     ap.add_argument("--fill-chunk", type=int, default=CHUNK, choices=[256, 512, 1024, 2048, 4096],
                     help="chunk size used to fill the cache before timing (fewer launches "
                          "for profiler captures); the timed steps are unchanged")
@@ -634,11 +708,15 @@ def main(argv=None):
                     help="foreground step rate; 0 runs steps back to back")
     ap.add_argument("--sweep", action="store_true",
                     help="run the L x n sweep instead of the 120K step line")
+    ap.add_argument("--unordered", action="store_true",
+                    help="time the unordered baseline (full recompute per step) beside CSR")
     args = ap.parse_args(argv)
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
     if args.sweep:
         return run_sweep(args)
+    if args.unordered:
+        return run_unordered(args)
     if args.asr:
         return run_asr(args)
     if args.impl == "reference":

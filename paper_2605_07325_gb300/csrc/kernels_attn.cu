@@ -69,6 +69,7 @@ size_t attn_smem_bytes(int head_dim) {
 // One item: a run of key tiles [j0, j1) of one unit.
 struct Seg {
   int32_t head, tile, item;
+  int32_t nk;  // key chunks of the item's unit
   int64_t j0, j1;
   bool complete;
 };
@@ -532,10 +533,11 @@ struct PairCfg {
 struct PairBars {
   uint64_t q_full, q_empty;
   uint64_t k_full[4], k_empty[4], v_full[4], v_empty[4];
-  uint64_t s_full[2], p_full[2], o_final[2], o_free[2];
+  uint64_t s_full[2], p_half[2], p_full[2], o_final[2], o_free[2];
   uint64_t drain;
   uint32_t tmem_base;
   int abort;
+  int last;  // this CTA completed a unit's last key chunk: it merges the unit
 };
 
 size_t attn_pair_smem_bytes(int head_dim) {
@@ -562,6 +564,7 @@ struct PairWalker {
       s.head = head;
       s.tile = pair;  // pair index
       s.item = it;
+      s.nk = static_cast<int32_t>((kv + p.chunk_tiles - 1) / p.chunk_tiles);
       s.j0 = j0;
       s.j1 = min(j0 + p.chunk_tiles, kv);
       s.complete = kv <= p.chunk_tiles;
@@ -571,8 +574,15 @@ struct PairWalker {
   }
 };
 
+// Register budget: launched with 384 x 168 registers; the two softmax
+// warpgroups take 208 each, warpgroup 2 (producer, MMA issuer, two idle
+// warps) keeps 80: 2 x 128 x 208 + 128 x 80 = 63,488 <= 64,512 = 384 x 168.
+constexpr int kPairThreads = 384;
+constexpr int kSoftmaxRegs = 208;
+constexpr int kControlRegs = 80;
+
 template <int HD>
-__global__ void __launch_bounds__(320, 1) attn_pair_kernel(const __grid_constant__ AttnParams p) {
+__global__ void __launch_bounds__(kPairThreads, 1) attn_pair_kernel(const __grid_constant__ AttnParams p) {
   using C = PairCfg<HD>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = reinterpret_cast<uint8_t *>(
@@ -593,6 +603,7 @@ __global__ void __launch_bounds__(320, 1) attn_pair_kernel(const __grid_constant
     }
     for (int w = 0; w < 2; ++w) {
       mbar_init(&bars->s_full[w], 1);
+      mbar_init(&bars->p_half[w], 128);
       mbar_init(&bars->p_full[w], 128);
       mbar_init(&bars->o_final[w], 1);
       mbar_init(&bars->o_free[w], 128);
@@ -617,7 +628,8 @@ __global__ void __launch_bounds__(320, 1) attn_pair_kernel(const __grid_constant
   volatile int *abort = &bars->abort;
   PairWalker walk{static_cast<int32_t>(blockIdx.x)};
   Seg seg;
-
+  if (warp >= 8) {
+  regs_decrease<kControlRegs>();
   if (warp == 8) {
     // ------------------------------------------------------ TMA producer
     int32_t *stage = reinterpret_cast<int32_t *>(smem + C::kPtOff);
@@ -710,15 +722,27 @@ __global__ void __launch_bounds__(320, 1) attn_pair_kernel(const __grid_constant
         }
         mma_commit(&bars->s_full[x]);
       };
-      // O_X += P_X V for tile x from V stage vs
-      auto issue_pv = [&](int x, int vs, bool first) {
+      // O_X += P_X V for tile x from V stage vs, keys [64 h, 64 h + 64) (half h)
+      auto issue_pv = [&](int x, int vs, bool first, int h) {
         const uint32_t vst = v_base + vs * C::kTileBytes;
 #pragma unroll
-        for (int kk = 0; kk < kBN / 16; ++kk) {
+        for (int k4 = 0; k4 < kBN / 32; ++k4) {
+          const int kk = h * (kBN / 32) + k4;
           const uint64_t b = sdesc_sw128(vst + kk * (16 * 128), kBN * 128, 1024);
           mma_bf16_ts(tmem + C::kOCol + x * HD, tmem + x * kBN + kk * 8, b, idesc_pv,
                       (!first || kk > 0) ? 1u : 0u);
         }
+      };
+      // P of tile x arrives in two halves; the first half's MMAs overlap the
+      // softmax of the second half.
+      auto pv_tile = [&](int x, int vs, bool first) {
+        if (!wait(&bars->p_half[x], pv_n[x] & 1)) return false;
+        tc_fence_after();
+        issue_pv(x, vs, first, 0);
+        if (!wait(&bars->p_full[x], pv_n[x] & 1)) return false;
+        tc_fence_after();
+        issue_pv(x, vs, first, 1);
+        return true;
       };
       while (ok && walk.next(p, T, seg)) {
         if (!wait(&bars->q_full, q_round & 1)) break;
@@ -737,11 +761,9 @@ __global__ void __launch_bounds__(320, 1) attn_pair_kernel(const __grid_constant
           const int vs = v_it % C::kStages;
           const bool more = i + 1 < nj;
           // ---- tile A
-          if (!wait(&bars->p_full[0], pv_n[0] & 1)) break;
           if (!wait(&bars->v_full[vs], (v_it / C::kStages) & 1)) break;
           if (i == 0 && seg_n > 0 && !wait(&bars->o_free[0], (seg_n & 1) ^ 1)) break;
-          tc_fence_after();
-          issue_pv(0, vs, i == 0);
+          if (!pv_tile(0, vs, i == 0)) break;
           if (i == nj - 1) mma_commit(&bars->o_final[0]);
           ++pv_n[0];
           if (more) {
@@ -751,10 +773,8 @@ __global__ void __launch_bounds__(320, 1) attn_pair_kernel(const __grid_constant
             issue_s(0, ks);
           }
           // ---- tile B
-          if (!wait(&bars->p_full[1], pv_n[1] & 1)) break;
           if (i == 0 && seg_n > 0 && !wait(&bars->o_free[1], (seg_n & 1) ^ 1)) break;
-          tc_fence_after();
-          issue_pv(1, vs, i == 0);
+          if (!pv_tile(1, vs, i == 0)) break;
           if (i == nj - 1) mma_commit(&bars->o_final[1]);
           ++pv_n[1];
           mma_commit(&bars->v_empty[vs]);
@@ -773,7 +793,9 @@ __global__ void __launch_bounds__(320, 1) attn_pair_kernel(const __grid_constant
         drain_wait(&bars->drain, 0);
       }
     }
+  }
   } else {
+    regs_increase<kSoftmaxRegs>();
     // ------------------------------------------------------ softmax warpgroups
     const int wg = warp >> 2;                  // 0: tile A, 1: tile B
     const int row = threadIdx.x - wg * 128;    // TMEM lane
@@ -825,25 +847,36 @@ __global__ void __launch_bounds__(320, 1) attn_pair_kernel(const __grid_constant
         l *= alpha;
         m_ref = m_new;
         const float m_use = (m_ref == -CUDART_INF_F) ? 0.f : m_ref;
+        // PV of the previous tile finished before these scores were published
+        // (same commit), so O can be rescaled without another wait; when it
+        // must be (rarely), both halves of P are published after the rescale.
+        const bool resc = i > 0 && __any_sync(0xffffffffu, need && had_mass);
         float rp[8];
 #pragma unroll
         for (int e = 0; e < 8; ++e) rp[e] = 0.f;
-        uint32_t pk[kBN / 2];
 #pragma unroll
-        for (int c = 0; c < kBN; c += 2) {
-          const float p0 = ex2_approx(fmaf(s[c], p.scale_log2, -m_use));
-          const float p1 = ex2_approx(fmaf(s[c + 1], p.scale_log2, -m_use));
-          rp[(c >> 1) & 7] += p0 + p1;
-          pk[c / 2] = pack_bf16x2(p0, p1);
+        for (int h = 0; h < 2; ++h) {
+          uint32_t pk[kBN / 4];
+#pragma unroll
+          for (int c = 0; c < kBN / 2; c += 2) {
+            const int cc = h * (kBN / 2) + c;
+            const float p0 = ex2_approx(fmaf(s[cc], p.scale_log2, -m_use));
+            const float p1 = ex2_approx(fmaf(s[cc + 1], p.scale_log2, -m_use));
+            rp[(c >> 1) & 7] += p0 + p1;
+            pk[c / 2] = pack_bf16x2(p0, p1);
+          }
+          tmem_st32(tmem + lane_base + s_col + h * (kBN / 4), pk);
+          if (h == 0 && !resc) {
+            tmem_st_wait();
+            tc_fence_before();
+            mbar_arrive(&bars->p_half[wg]);
+          }
         }
         l += ((rp[0] + rp[1]) + (rp[2] + rp[3])) + ((rp[4] + rp[5]) + (rp[6] + rp[7]));
-        tmem_st64(tmem + lane_base + s_col, pk);
-        // PV of the previous tile finished before these scores were published
-        // (same commit), so O can be rescaled here without another wait.
-        if (i > 0 && __any_sync(0xffffffffu, need && had_mass))
-          rescale_o<HD>(tmem + lane_base + o_col, alpha);
+        if (resc) rescale_o<HD>(tmem + lane_base + o_col, alpha);
         tmem_st_wait();
         tc_fence_before();
+        if (resc) mbar_arrive(&bars->p_half[wg]);
         mbar_arrive(&bars->p_full[wg]);
         ++s_it;
       }
@@ -860,6 +893,8 @@ __global__ void __launch_bounds__(320, 1) attn_pair_kernel(const __grid_constant
       const float lse2 = l > 0.f ? m_ref + log2f(l) : -CUDART_INF_F;
       uint32_t o[HD];
       load_o<HD>(tmem + lane_base + o_col, o);
+      tc_fence_before();
+      mbar_arrive(&bars->o_free[wg]);  // O is in registers: the next item may start
       if (seg.complete) {
         if (valid) {
           const int hq_idx = seg.head * p.group + row % p.group;
@@ -883,9 +918,64 @@ __global__ void __launch_bounds__(320, 1) attn_pair_kernel(const __grid_constant
           d4[c] = make_float4(__uint_as_float(o[4 * c]) * inv_l, __uint_as_float(o[4 * c + 1]) * inv_l,
                               __uint_as_float(o[4 * c + 2]) * inv_l, __uint_as_float(o[4 * c + 3]) * inv_l);
         p.part_lse[base] = lse2;
+        if (p.counters) {
+          // The CTA that finishes a unit's last key chunk merges the unit:
+          // lse = log2 sum_k 2^lse_k, O = sum_k 2^(lse_k - lse) O_k, in chunk order.
+          const int32_t n_pairs = (p.n_tiles + 1) / 2;
+          const int32_t unit = seg.head * n_pairs + seg.tile;
+          named_bar_sync(1, 256);
+          if (threadIdx.x == 0) {
+            __threadfence();
+            bars->last = atomicAdd(&p.counters[unit], 1) == seg.nk - 1;
+          }
+          named_bar_sync(1, 256);
+          if (bars->last) {
+            __threadfence();
+            const int64_t units = static_cast<int64_t>(p.hkv) * n_pairs;
+            const int64_t rin = wg * kBM + row;
+            float mx = -CUDART_INF_F;
+            for (int k = 0; k < seg.nk; ++k)
+              mx = fmaxf(mx, __ldcg(p.part_lse + (k * units + unit) * (2 * kBM) + rin));
+            float accum[HD];
+#pragma unroll
+            for (int c = 0; c < HD; ++c) accum[c] = 0.f;
+            float tot = -CUDART_INF_F;
+            if (mx != -CUDART_INF_F) {
+              float sum = 0.f;
+              for (int k = 0; k < seg.nk; ++k)
+                sum += ex2_approx(__ldcg(p.part_lse + (k * units + unit) * (2 * kBM) + rin) - mx);
+              tot = mx + log2f(sum);
+              for (int k = 0; k < seg.nk; ++k) {
+                const int64_t b = (k * units + unit) * (2 * kBM) + rin;
+                const float w = ex2_approx(__ldcg(p.part_lse + b) - tot);
+                const float4 *src = reinterpret_cast<const float4 *>(p.part_o + b * HD);
+#pragma unroll
+                for (int c = 0; c < HD / 4; ++c) {
+                  const float4 v = __ldcg(src + c);
+                  accum[4 * c] = fmaf(w, v.x, accum[4 * c]);
+                  accum[4 * c + 1] = fmaf(w, v.y, accum[4 * c + 1]);
+                  accum[4 * c + 2] = fmaf(w, v.z, accum[4 * c + 2]);
+                  accum[4 * c + 3] = fmaf(w, v.w, accum[4 * c + 3]);
+                }
+              }
+            }
+            if (valid) {
+              const int hq_idx = seg.head * p.group + row % p.group;
+              uint16_t *dst = p.out + (static_cast<int64_t>(t) * p.hq + hq_idx) * HD;
+#pragma unroll
+              for (int q8 = 0; q8 < HD / 8; ++q8) {
+                uint32_t w4[4];
+#pragma unroll
+                for (int c = 0; c < 4; ++c)
+                  w4[c] = pack_bf16x2(accum[q8 * 8 + 2 * c], accum[q8 * 8 + 2 * c + 1]);
+                reinterpret_cast<uint4 *>(dst)[q8] = make_uint4(w4[0], w4[1], w4[2], w4[3]);
+              }
+              if (p.lse) p.lse[static_cast<int64_t>(hq_idx) * p.n + t] = tot * 0.69314718055994531f;
+            }
+            if (threadIdx.x == 0) p.counters[unit] = 0;
+          }
+        }
       }
-      tc_fence_before();
-      mbar_arrive(&bars->o_free[wg]);
       ++seg_n;
     }
   }
@@ -1392,9 +1482,9 @@ cudaError_t launch_attention(const AttnParams &p, int head_dim, cudaStream_t s) 
       attn_pipe_kernel<128><<<p.grid, 320, PipeCfg<128>::kSmem, s>>>(p);
   } else if (p.unit_tiles == 2) {
     if (head_dim == 64)
-      attn_pair_kernel<64><<<p.grid, 320, PairCfg<64>::kSmem, s>>>(p);
+      attn_pair_kernel<64><<<p.grid, kPairThreads, PairCfg<64>::kSmem, s>>>(p);
     else
-      attn_pair_kernel<128><<<p.grid, 320, PairCfg<128>::kSmem, s>>>(p);
+      attn_pair_kernel<128><<<p.grid, kPairThreads, PairCfg<128>::kSmem, s>>>(p);
   } else {
     if (head_dim == 64)
       attn_kernel<64><<<p.grid, 192, AttnCfg<64>::kSmem, s>>>(p);
