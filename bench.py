@@ -248,8 +248,7 @@ def run_ours(args):
     cfg = csr.make_config(HQ, HKV, D, P, BASE, max_new_tokens=PREFIX, pool_pages=pool_pages,
                           max_seq_tokens=max_tokens + P,
                           flags={"pair": 0, "pipe": csr.FLAG_PIPE_64,
-                                 "single": csr.FLAG_SINGLE_TILE}[args.kernel] |
-                          (csr.FLAG_SEPARATE_MERGE if args.separate_merge else 0))
+                                 "single": csr.FLAG_SINGLE_TILE}[args.kernel])
     stream = torch.cuda.Stream(device=dev, priority=-1)
     gen = torch.Generator(device=dev).manual_seed(1234 + rank)
 
@@ -696,8 +695,6 @@ def main(argv=None):
                     help="attention kernel: pair (default: two query tiles per CTA, 128-key "
                          "tiles), pipe (two query tiles, 64-key tiles, two score buffers each), "
                          "single (one query tile per CTA)")
-    ap.add_argument("--separate-merge", action="store_true",
-                    help="merge split-KV partials in a separate kernel (default: fused)")
     ap.add_argument("--fill-chunk", type=int, default=CHUNK, choices=[256, 512, 1024, 2048, 4096],
                     help="chunk size used to fill the cache before timing (fewer launches "
                          "for profiler captures); the timed steps are unchanged")

@@ -77,9 +77,6 @@ typedef enum csr_status {
 #define CSR_FLAG_PIPE_64 0x4     /* two query tiles per CTA with 64-key tiles and two score
                                     buffers each (an experimental third design); the default
                                     uses 128-key tiles and one score buffer per query tile */
-#define CSR_FLAG_SEPARATE_MERGE 0x8 /* merge split-KV partials in a separate kernel; by
-                                       default the two-tile kernel's CTA that finishes a unit's
-                                       last key chunk merges it */
 
 typedef struct csr_config {
   int32_t num_q_heads;    /* H_q */

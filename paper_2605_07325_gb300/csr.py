@@ -31,7 +31,6 @@ DEVERR_WAIT_TIMEOUT, DEVERR_BAD_PAGE, DEVERR_ALLOC = 0x1, 0x2, 0x4
 FLAG_PLAN_ONLY = 0x1
 FLAG_SINGLE_TILE = 0x2
 FLAG_PIPE_64 = 0x4
-FLAG_SEPARATE_MERGE = 0x8
 RECON_IDLE, RECON_RUNNING, RECON_SWAPPED = 0, 1, 2
 VERSION_ACTIVE, VERSION_PENDING = 0, 1
 

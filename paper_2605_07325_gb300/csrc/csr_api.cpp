@@ -124,8 +124,7 @@ bool encode_rows(CUtensorMap *m, void *base, uint64_t rows, uint64_t d, uint32_t
 }
 
 struct Layout {  // workspace carve-out (byte offsets)
-  size_t qpack[2], rb_out, part_o[2], part_lse[2], counters[2], pt[2], ids_out, err, total;
-  int32_t n_counters;
+  size_t qpack[2], rb_out, part_o[2], part_lse[2], pt[2], ids_out, err, total;
   int32_t rows_cap, fg_cap, max_pages;
 };
 
@@ -179,9 +178,6 @@ Layout make_layout(const csr_config *c) {
     L.part_o[i] = take(static_cast<size_t>(kPartialItems) * kBM * d * 4);
     L.part_lse[i] = take(static_cast<size_t>(kPartialItems) * kBM * 4);
   }
-  // one counter per two-tile unit of a launch: kv heads x pairs of 128-row tiles
-  L.n_counters = c->num_kv_heads * (L.rows_cap / (2 * kBM));
-  for (int i = 0; i < 2; ++i) L.counters[i] = take(static_cast<size_t>(L.n_counters) * 4);
   for (int i = 0; i < 2; ++i) L.pt[i] = take(static_cast<size_t>(L.max_pages) * 4);
   L.ids_out = take(static_cast<size_t>(L.max_pages) * 4);
   L.err = take(256);
@@ -381,21 +377,13 @@ csr_status run_block(csr_ctx *c, int slot, int ws, const void *q, const void *k,
   // foreground: persistent CTAs over the items; rebuild: one item per CTA
   ap.grid = ws == 0 ? static_cast<int32_t>(std::min<int64_t>(c->fg_grid, ap.n_items)) : ap.n_items;
   ap.scale_log2 = c->scale_log2;
-  // the two-tile kernel merges split units itself (per-unit counters, zeroed by K1)
-  const bool fused = ap.unit_tiles == 2 && ap.kv_tile == kBN && n_chunks > 1 &&
-                     !(cf.flags & CSR_FLAG_SEPARATE_MERGE) && units <= c->lay.n_counters;
-  if (fused) {
-    ap.counters = c->wsp<int32_t>(c->lay.counters[ws]);
-    rp.counters = ap.counters;
-    rp.n_counters = static_cast<int32_t>(units);
-  }
   cudaError_t e = timed_launch(c, CSR_KERNEL_ROPE_APPEND, fg, s, [&] { return launch_rope_append(rp, s); });
   if (e != cudaSuccess) return cuda_fail(c, e, "rope_append launch");
   ++c->launches;
   e = timed_launch(c, CSR_KERNEL_ATTENTION, fg, s, [&] { return launch_attention(ap, cf.head_dim, s); });
   if (e != cudaSuccess) return cuda_fail(c, e, "attention launch");
   ++c->launches;
-  if (n_chunks > 1 && !fused) {
+  if (n_chunks > 1) {
     MergeParams mp{};
     mp.part_o = ap.part_o;
     mp.part_lse = ap.part_lse;

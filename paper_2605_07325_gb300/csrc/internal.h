@@ -31,8 +31,6 @@ struct RopeAppendParams {
   int32_t n, hq, hkv, d, page_size, group, rows_cap, pool_pages;
   int32_t first_lp;        // logical page of pos0
   int32_t n_ids;           // > 0: ids[] give the physical pages first_lp..; 0: read page_table
-  int32_t *counters;       // per-unit chunk counters of the next attention launch, zeroed here
-  int32_t n_counters;
   double inv_turns[kMaxHalfDim];  // base^(-2i/d) / (2 pi), i < d/2
   int32_t ids[kMaxIdsPerCall];
 };
@@ -47,8 +45,6 @@ struct AttnParams {
   float *lse;              // [hq][n] natural log, or null
   float *part_o;           // [n_items][kBM][d] fp32 (normalised partial outputs)
   float *part_lse;         // [n_items][kBM] fp32 (log2 domain)
-  int32_t *counters;       // per-unit finished-chunk counts (zero at launch), or null:
-                           // with them the two-tile kernel merges split units itself
   uint32_t *err;
   int64_t L;               // cached tokens before this call
   int32_t n, hq, hkv, group, page_size, rows_cap, n_tiles, n_pages_valid, pool_pages;

@@ -152,6 +152,26 @@ __device__ __forceinline__ void load_kv_keys(const AttnParams &p, const CUtensor
   }
 }
 
+// Issue the TMA loads of one 128-key tile of `head` whose pages' physical ids
+// are phys[0 .. 128/P): one 64-column box per page and column half (two
+// 64-row boxes per page when P = 128).
+template <int HD>
+__device__ __forceinline__ void load_kv_tile(const AttnParams &p, const CUtensorMap *map,
+                                             uint8_t *dst, uint64_t *bar, int head,
+                                             const int32_t *phys) {
+  const int P = p.page_size;
+  const int ppt = kBN / P;
+  const int seg = P < 64 ? P : 64;
+  for (int pp = 0; pp < ppt; ++pp) {
+    const int32_t row0 = (phys[pp] * p.hkv + head) * P;
+    for (int r = 0; r < P; r += seg) {
+#pragma unroll
+      for (int b = 0; b < HD / 64; ++b)
+        tma_load_2d(dst + b * (kBN * 128) + (pp * P + r) * 128, map, bar, b * 64, row0 + r);
+    }
+  }
+}
+
 // Stage the physical ids of the logical pages covering key tiles [jb, je)
 // (tiles of bn keys) into `stage`, one id per page (whole producer warp).
 // Returns the first staged logical page.
@@ -533,11 +553,10 @@ struct PairCfg {
 struct PairBars {
   uint64_t q_full, q_empty;
   uint64_t k_full[4], k_empty[4], v_full[4], v_empty[4];
-  uint64_t s_full[2], p_half[2], p_full[2], o_final[2], o_free[2];
+  uint64_t s_full[2], p_full[2], o_final[2], o_free[2];
   uint64_t drain;
   uint32_t tmem_base;
   int abort;
-  int last;  // this CTA completed a unit's last key chunk: it merges the unit
 };
 
 size_t attn_pair_smem_bytes(int head_dim) {
@@ -574,12 +593,7 @@ struct PairWalker {
   }
 };
 
-// Register budget: launched with 384 x 168 registers; the two softmax
-// warpgroups take 208 each, warpgroup 2 (producer, MMA issuer, two idle
-// warps) keeps 80: 2 x 128 x 208 + 128 x 80 = 63,488 <= 64,512 = 384 x 168.
-constexpr int kPairThreads = 384;
-constexpr int kSoftmaxRegs = 208;
-constexpr int kControlRegs = 80;
+constexpr int kPairThreads = 320;
 
 template <int HD>
 __global__ void __launch_bounds__(kPairThreads, 1) attn_pair_kernel(const __grid_constant__ AttnParams p) {
@@ -603,7 +617,6 @@ __global__ void __launch_bounds__(kPairThreads, 1) attn_pair_kernel(const __grid
     }
     for (int w = 0; w < 2; ++w) {
       mbar_init(&bars->s_full[w], 1);
-      mbar_init(&bars->p_half[w], 128);
       mbar_init(&bars->p_full[w], 128);
       mbar_init(&bars->o_final[w], 1);
       mbar_init(&bars->o_free[w], 128);
@@ -628,13 +641,12 @@ __global__ void __launch_bounds__(kPairThreads, 1) attn_pair_kernel(const __grid
   volatile int *abort = &bars->abort;
   PairWalker walk{static_cast<int32_t>(blockIdx.x)};
   Seg seg;
-  if (warp >= 8) {
-  regs_decrease<kControlRegs>();
+
   if (warp == 8) {
     // ------------------------------------------------------ TMA producer
     int32_t *stage = reinterpret_cast<int32_t *>(smem + C::kPtOff);
-    // key tiles whose pages fit one staging block (a tile may end mid-page)
-    const int tiles_per_block = (C::kPtStage - 2) * p.page_size / kBN;
+    const int ppt = kBN / p.page_size;
+    const int tiles_per_block = C::kPtStage / ppt;
     uint32_t q_round = 0, k_it = 0, v_it = 0;
     bool ok = true;
     while (ok && walk.next(p, T, seg)) {
@@ -657,12 +669,21 @@ __global__ void __launch_bounds__(kPairThreads, 1) attn_pair_kernel(const __grid
       ok = __shfl_sync(0xffffffffu, ok, 0);
       for (int64_t jb = seg.j0; ok && jb < seg.j1; jb += tiles_per_block) {
         const int64_t je = min(jb + tiles_per_block, seg.j1);
+        const int npages = static_cast<int>(je - jb) * ppt;
         __syncwarp();
-        const int64_t lp_base = stage_pages(p, stage, kBN, jb, je, lane);
+        for (int i = lane; i < npages; i += 32) {
+          const int64_t lp = jb * ppt + i;
+          int32_t phys = (lp < p.n_pages_valid) ? p.page_table[lp] : p.page_table[0];
+          if (phys < 0 || phys >= p.pool_pages) {
+            atomicOr(p.err, CSR_DEVERR_BAD_PAGE);
+            phys = 0;
+          }
+          stage[i] = phys;
+        }
         __syncwarp();
         if (lane == 0) {
           for (int64_t j = jb; j < je; ++j) {
-
+            const int32_t *phys = stage + static_cast<int>(j - jb) * ppt;
             const int ks = k_it % C::kStages;
             if (!mbar_wait(&bars->k_empty[ks], ((k_it / C::kStages) & 1) ^ 1, abort, p.err,
                            CSR_DEVERR_WAIT_TIMEOUT)) {
@@ -670,8 +691,8 @@ __global__ void __launch_bounds__(kPairThreads, 1) attn_pair_kernel(const __grid
               break;
             }
             mbar_arrive_expect_tx(&bars->k_full[ks], C::kTileBytes);
-            load_kv_keys<HD>(p, &p.tm_k, smem + C::kKOff + ks * C::kTileBytes, kBN, &bars->k_full[ks],
-                             seg.head, stage, lp_base, j * kBN);
+            load_kv_tile<HD>(p, &p.tm_k, smem + C::kKOff + ks * C::kTileBytes, &bars->k_full[ks],
+                             seg.head, phys);
             ++k_it;
             const int vs = v_it % C::kStages;
             if (!mbar_wait(&bars->v_empty[vs], ((v_it / C::kStages) & 1) ^ 1, abort, p.err,
@@ -680,8 +701,8 @@ __global__ void __launch_bounds__(kPairThreads, 1) attn_pair_kernel(const __grid
               break;
             }
             mbar_arrive_expect_tx(&bars->v_full[vs], C::kTileBytes);
-            load_kv_keys<HD>(p, &p.tm_v, smem + C::kVOff + vs * C::kTileBytes, kBN, &bars->v_full[vs],
-                             seg.head, stage, lp_base, j * kBN);
+            load_kv_tile<HD>(p, &p.tm_v, smem + C::kVOff + vs * C::kTileBytes, &bars->v_full[vs],
+                             seg.head, phys);
             ++v_it;
           }
         }
@@ -722,27 +743,15 @@ __global__ void __launch_bounds__(kPairThreads, 1) attn_pair_kernel(const __grid
         }
         mma_commit(&bars->s_full[x]);
       };
-      // O_X += P_X V for tile x from V stage vs, keys [64 h, 64 h + 64) (half h)
-      auto issue_pv = [&](int x, int vs, bool first, int h) {
+      // O_X += P_X V for tile x from V stage vs
+      auto issue_pv = [&](int x, int vs, bool first) {
         const uint32_t vst = v_base + vs * C::kTileBytes;
 #pragma unroll
-        for (int k4 = 0; k4 < kBN / 32; ++k4) {
-          const int kk = h * (kBN / 32) + k4;
+        for (int kk = 0; kk < kBN / 16; ++kk) {
           const uint64_t b = sdesc_sw128(vst + kk * (16 * 128), kBN * 128, 1024);
           mma_bf16_ts(tmem + C::kOCol + x * HD, tmem + x * kBN + kk * 8, b, idesc_pv,
                       (!first || kk > 0) ? 1u : 0u);
         }
-      };
-      // P of tile x arrives in two halves; the first half's MMAs overlap the
-      // softmax of the second half.
-      auto pv_tile = [&](int x, int vs, bool first) {
-        if (!wait(&bars->p_half[x], pv_n[x] & 1)) return false;
-        tc_fence_after();
-        issue_pv(x, vs, first, 0);
-        if (!wait(&bars->p_full[x], pv_n[x] & 1)) return false;
-        tc_fence_after();
-        issue_pv(x, vs, first, 1);
-        return true;
       };
       while (ok && walk.next(p, T, seg)) {
         if (!wait(&bars->q_full, q_round & 1)) break;
@@ -761,9 +770,11 @@ __global__ void __launch_bounds__(kPairThreads, 1) attn_pair_kernel(const __grid
           const int vs = v_it % C::kStages;
           const bool more = i + 1 < nj;
           // ---- tile A
+          if (!wait(&bars->p_full[0], pv_n[0] & 1)) break;
           if (!wait(&bars->v_full[vs], (v_it / C::kStages) & 1)) break;
           if (i == 0 && seg_n > 0 && !wait(&bars->o_free[0], (seg_n & 1) ^ 1)) break;
-          if (!pv_tile(0, vs, i == 0)) break;
+          tc_fence_after();
+          issue_pv(0, vs, i == 0);
           if (i == nj - 1) mma_commit(&bars->o_final[0]);
           ++pv_n[0];
           if (more) {
@@ -773,8 +784,10 @@ __global__ void __launch_bounds__(kPairThreads, 1) attn_pair_kernel(const __grid
             issue_s(0, ks);
           }
           // ---- tile B
+          if (!wait(&bars->p_full[1], pv_n[1] & 1)) break;
           if (i == 0 && seg_n > 0 && !wait(&bars->o_free[1], (seg_n & 1) ^ 1)) break;
-          if (!pv_tile(1, vs, i == 0)) break;
+          tc_fence_after();
+          issue_pv(1, vs, i == 0);
           if (i == nj - 1) mma_commit(&bars->o_final[1]);
           ++pv_n[1];
           mma_commit(&bars->v_empty[vs]);
@@ -793,9 +806,7 @@ __global__ void __launch_bounds__(kPairThreads, 1) attn_pair_kernel(const __grid
         drain_wait(&bars->drain, 0);
       }
     }
-  }
   } else {
-    regs_increase<kSoftmaxRegs>();
     // ------------------------------------------------------ softmax warpgroups
     const int wg = warp >> 2;                  // 0: tile A, 1: tile B
     const int row = threadIdx.x - wg * 128;    // TMEM lane
@@ -847,36 +858,25 @@ __global__ void __launch_bounds__(kPairThreads, 1) attn_pair_kernel(const __grid
         l *= alpha;
         m_ref = m_new;
         const float m_use = (m_ref == -CUDART_INF_F) ? 0.f : m_ref;
-        // PV of the previous tile finished before these scores were published
-        // (same commit), so O can be rescaled without another wait; when it
-        // must be (rarely), both halves of P are published after the rescale.
-        const bool resc = i > 0 && __any_sync(0xffffffffu, need && had_mass);
         float rp[8];
 #pragma unroll
         for (int e = 0; e < 8; ++e) rp[e] = 0.f;
+        uint32_t pk[kBN / 2];
 #pragma unroll
-        for (int h = 0; h < 2; ++h) {
-          uint32_t pk[kBN / 4];
-#pragma unroll
-          for (int c = 0; c < kBN / 2; c += 2) {
-            const int cc = h * (kBN / 2) + c;
-            const float p0 = ex2_approx(fmaf(s[cc], p.scale_log2, -m_use));
-            const float p1 = ex2_approx(fmaf(s[cc + 1], p.scale_log2, -m_use));
-            rp[(c >> 1) & 7] += p0 + p1;
-            pk[c / 2] = pack_bf16x2(p0, p1);
-          }
-          tmem_st32(tmem + lane_base + s_col + h * (kBN / 4), pk);
-          if (h == 0 && !resc) {
-            tmem_st_wait();
-            tc_fence_before();
-            mbar_arrive(&bars->p_half[wg]);
-          }
+        for (int c = 0; c < kBN; c += 2) {
+          const float p0 = ex2_approx(fmaf(s[c], p.scale_log2, -m_use));
+          const float p1 = ex2_approx(fmaf(s[c + 1], p.scale_log2, -m_use));
+          rp[(c >> 1) & 7] += p0 + p1;
+          pk[c / 2] = pack_bf16x2(p0, p1);
         }
         l += ((rp[0] + rp[1]) + (rp[2] + rp[3])) + ((rp[4] + rp[5]) + (rp[6] + rp[7]));
-        if (resc) rescale_o<HD>(tmem + lane_base + o_col, alpha);
+        tmem_st64(tmem + lane_base + s_col, pk);
+        // PV of the previous tile finished before these scores were published
+        // (same commit), so O can be rescaled here without another wait.
+        if (i > 0 && __any_sync(0xffffffffu, need && had_mass))
+          rescale_o<HD>(tmem + lane_base + o_col, alpha);
         tmem_st_wait();
         tc_fence_before();
-        if (resc) mbar_arrive(&bars->p_half[wg]);
         mbar_arrive(&bars->p_full[wg]);
         ++s_it;
       }
@@ -893,8 +893,6 @@ __global__ void __launch_bounds__(kPairThreads, 1) attn_pair_kernel(const __grid
       const float lse2 = l > 0.f ? m_ref + log2f(l) : -CUDART_INF_F;
       uint32_t o[HD];
       load_o<HD>(tmem + lane_base + o_col, o);
-      tc_fence_before();
-      mbar_arrive(&bars->o_free[wg]);  // O is in registers: the next item may start
       if (seg.complete) {
         if (valid) {
           const int hq_idx = seg.head * p.group + row % p.group;
@@ -918,64 +916,9 @@ __global__ void __launch_bounds__(kPairThreads, 1) attn_pair_kernel(const __grid
           d4[c] = make_float4(__uint_as_float(o[4 * c]) * inv_l, __uint_as_float(o[4 * c + 1]) * inv_l,
                               __uint_as_float(o[4 * c + 2]) * inv_l, __uint_as_float(o[4 * c + 3]) * inv_l);
         p.part_lse[base] = lse2;
-        if (p.counters) {
-          // The CTA that finishes a unit's last key chunk merges the unit:
-          // lse = log2 sum_k 2^lse_k, O = sum_k 2^(lse_k - lse) O_k, in chunk order.
-          const int32_t n_pairs = (p.n_tiles + 1) / 2;
-          const int32_t unit = seg.head * n_pairs + seg.tile;
-          named_bar_sync(1, 256);
-          if (threadIdx.x == 0) {
-            __threadfence();
-            bars->last = atomicAdd(&p.counters[unit], 1) == seg.nk - 1;
-          }
-          named_bar_sync(1, 256);
-          if (bars->last) {
-            __threadfence();
-            const int64_t units = static_cast<int64_t>(p.hkv) * n_pairs;
-            const int64_t rin = wg * kBM + row;
-            float mx = -CUDART_INF_F;
-            for (int k = 0; k < seg.nk; ++k)
-              mx = fmaxf(mx, __ldcg(p.part_lse + (k * units + unit) * (2 * kBM) + rin));
-            float accum[HD];
-#pragma unroll
-            for (int c = 0; c < HD; ++c) accum[c] = 0.f;
-            float tot = -CUDART_INF_F;
-            if (mx != -CUDART_INF_F) {
-              float sum = 0.f;
-              for (int k = 0; k < seg.nk; ++k)
-                sum += ex2_approx(__ldcg(p.part_lse + (k * units + unit) * (2 * kBM) + rin) - mx);
-              tot = mx + log2f(sum);
-              for (int k = 0; k < seg.nk; ++k) {
-                const int64_t b = (k * units + unit) * (2 * kBM) + rin;
-                const float w = ex2_approx(__ldcg(p.part_lse + b) - tot);
-                const float4 *src = reinterpret_cast<const float4 *>(p.part_o + b * HD);
-#pragma unroll
-                for (int c = 0; c < HD / 4; ++c) {
-                  const float4 v = __ldcg(src + c);
-                  accum[4 * c] = fmaf(w, v.x, accum[4 * c]);
-                  accum[4 * c + 1] = fmaf(w, v.y, accum[4 * c + 1]);
-                  accum[4 * c + 2] = fmaf(w, v.z, accum[4 * c + 2]);
-                  accum[4 * c + 3] = fmaf(w, v.w, accum[4 * c + 3]);
-                }
-              }
-            }
-            if (valid) {
-              const int hq_idx = seg.head * p.group + row % p.group;
-              uint16_t *dst = p.out + (static_cast<int64_t>(t) * p.hq + hq_idx) * HD;
-#pragma unroll
-              for (int q8 = 0; q8 < HD / 8; ++q8) {
-                uint32_t w4[4];
-#pragma unroll
-                for (int c = 0; c < 4; ++c)
-                  w4[c] = pack_bf16x2(accum[q8 * 8 + 2 * c], accum[q8 * 8 + 2 * c + 1]);
-                reinterpret_cast<uint4 *>(dst)[q8] = make_uint4(w4[0], w4[1], w4[2], w4[3]);
-              }
-              if (p.lse) p.lse[static_cast<int64_t>(hq_idx) * p.n + t] = tot * 0.69314718055994531f;
-            }
-            if (threadIdx.x == 0) p.counters[unit] = 0;
-          }
-        }
       }
+      tc_fence_before();
+      mbar_arrive(&bars->o_free[wg]);
       ++seg_n;
     }
   }

@@ -56,9 +56,8 @@ __global__ void __launch_bounds__(256) rope_append_kernel(const __grid_constant_
     cs[i] = c;
     sn[i] = s;
   }
-  if (blockIdx.x == 0) {
+  if (blockIdx.x == 0 && p.n_ids > 0) {
     for (int i = threadIdx.x; i < p.n_ids; i += blockDim.x) p.page_table[p.first_lp + i] = p.ids[i];
-    for (int i = threadIdx.x; i < p.n_counters; i += blockDim.x) p.counters[i] = 0;
   }
   __syncthreads();
   const int64_t lp = pos / p.page_size;

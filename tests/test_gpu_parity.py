@@ -67,14 +67,11 @@ def test_ragged_sizes(libcsr, shape, chunk_tiles):
 
 @pytest.mark.parametrize("num_ctas,chunk_tiles", [(1, 0), (3, 1), (7, 2), (19, 3), (64, 5),
                                                    (152, 1), (0, 4)])
-@pytest.mark.parametrize("merge", ["fused", "separate"])
-def test_split_kv_partials_any_grid(libcsr, num_ctas, chunk_tiles, merge):
+def test_split_kv_partials_any_grid(libcsr, num_ctas, chunk_tiles):
     """Forced CTA counts and key-chunk lengths: every split into items (down to
-    one 128-key tile per item) must merge back to the oracle, whether the
-    attention kernel merges the units itself or a separate kernel does."""
-    flags = libcsr.FLAG_SEPARATE_MERGE if merge == "separate" else 0
+    one 128-key tile per item) must merge back to the oracle."""
     p = Pair(C2, pool_pages=256, max_seq=8192, max_new=1024, num_ctas=num_ctas,
-             fg_chunk_tiles=chunk_tiles, flags=flags)
+             fg_chunk_tiles=chunk_tiles)
     p.init_static(p.blk(30, 700))
     p.append(p.blk(31, 1000))
     p.append(p.blk(32, 33))
