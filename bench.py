@@ -430,7 +430,8 @@ def run_asr(args):
     pool_pages = (2 * n_max) // P + 64
     cfg = csr.make_config(HQ, HKV, D, P, BASE, max_new_tokens=PREFIX, pool_pages=pool_pages,
                           max_seq_tokens=n_max, cap_tokens=ASR_CAP,
-                          evict_tokens=ASR_EVICT, n_catchup=0)
+                          evict_tokens=ASR_EVICT, n_catchup=0,
+                          rebuild_tiles_per_cta=args.asr_rebuild_tiles)
     fg = torch.cuda.Stream(device=dev, priority=-1)     # high priority
     lo = torch.cuda.Stream(device=dev, priority=0)      # low priority (rebuild, R_2)
     gen = torch.Generator(device=dev).manual_seed(4321)
@@ -498,8 +499,6 @@ def run_asr(args):
         if not was and model.length() >= ASR_CAP:
             model.evict(ASR_EVICT)          # the library started it inside append_chunk
             rb_start = time.perf_counter()
-            lo_ev = torch.cuda.Event(enable_timing=True)
-            lo_ev.record(lo)                # after every rebuild launch
         peak_len = max(peak_len, model.length())
         during = was or model.is_reconciling
         records.append((t1 - t0, e0.elapsed_time(e1) / 1e3, during))
@@ -520,7 +519,8 @@ def run_asr(args):
         "workload": ("ASR cycle run: cap 131,072 tokens, 4,096-token prefix, 256-token chunks + "
                      "512-token suffix per step, evict oldest 32,768 tokens, rebuild on a "
                      "low-priority stream, 64 q / 4 kv heads, d 128, page 64, 1 layer"),
-        "cadence_hz": args.asr_cadence_hz, "cycles": cycles, "steps": step,
+        "cadence_hz": args.asr_cadence_hz, "rebuild_tiles_per_cta": args.asr_rebuild_tiles or 16,
+        "cycles": cycles, "steps": step,
         "steps_during_rebuild": len(dur),
         "fg_ms_host": {"p50_outside": pct(out, 50), "p99_outside": pct(out, 99),
                        "p50_during": pct(dur, 50), "p99_during": pct(dur, 99)},
@@ -535,6 +535,14 @@ def run_asr(args):
     }
     if out and dur:
         line["p99_increase_during_rebuild"] = pct(dur, 99) / pct(out, 99) - 1.0
+    # App. D viability: the rebuild (warm-up + catch-up, here eviction -> swap)
+    # must end before the cache, growing at X_dot tokens/s from tau_mem, reaches N_max
+    if rebuilds and period:
+        x_dot = CHUNK / period
+        dt_mem = (n_max - ASR_CAP) / x_dot
+        line["viability"] = {"x_dot_tokens_per_s": x_dot, "dt_mem_s": dt_mem,
+                             "dt_rebuild_max_s": max(rebuilds),
+                             "holds": max(rebuilds) <= dt_mem and peak_len <= n_max}
     print(json.dumps(line), flush=True)
     ctx.close()
     return 0 if layout_ok and flags == 0 else 1
@@ -701,6 +709,8 @@ def main(argv=None):
     ap.add_argument("--asr", action="store_true",
                     help="run the ASR cycle workload instead of the 120K step line")
     ap.add_argument("--asr-cycles", type=int, default=10)
+    ap.add_argument("--asr-rebuild-tiles", type=int, default=0,
+                    help="key tiles per rebuild CTA (0: the library default, 16)")
     ap.add_argument("--asr-cadence-hz", type=float, default=2.0,
                     help="foreground step rate; 0 runs steps back to back")
     ap.add_argument("--sweep", action="store_true",

@@ -92,7 +92,7 @@ typedef struct csr_config {
   int32_t evict_tokens;   /* tokens of the oldest chunks dropped by an automatic eviction */
   int32_t n_catchup;      /* N_catchup of Algorithm 1 */
   int32_t num_ctas;       /* CTAs of a foreground attention launch; 0 = one per SM */
-  int32_t rebuild_tiles_per_cta; /* key tiles (128 keys) per CTA in rebuild launches; 0 = 64 */
+  int32_t rebuild_tiles_per_cta; /* key tiles (128 keys) per CTA in rebuild launches; 0 = 16 */
   int32_t flags;          /* CSR_FLAG_* */
   int32_t fg_chunk_tiles; /* key tiles per split-KV item of a foreground launch; 0 = chosen
                              per launch from its shape */
@@ -177,13 +177,18 @@ csr_status csr_rewind(csr_ctx *ctx, int64_t length);
 /*
  * Source of a chunk's layer inputs for the rebuild (the "LLM(X_eps)" of
  * Algorithm 1 recomputes a retained chunk in its new context).  The callback
- * is called on the thread that drives the context, with the chunk's id and
- * length, and must set *q, *k, *v to device pointers holding that chunk's
- * pre-RoPE queries/keys/values in the layouts above, valid until the
- * reconciliation that asked for them has swapped or failed.  It may set *out
- * to a device buffer [n][num_q_heads][head_dim] that receives the chunk's
- * rebuilt attention output, or leave it NULL.  Returns 0 on success; any other
- * value aborts the reconciliation (the active version stays as it is).
+ * is called on the context's reconciliation thread (a library thread started
+ * by csr_set_reconciler; one call at a time, in rebuild order), with the
+ * chunk's id and length, and must set *q, *k, *v to device pointers holding
+ * that chunk's pre-RoPE queries/keys/values in the layouts above, valid until
+ * the reconciliation that asked for them has swapped or failed.  Their
+ * contents must be complete when the callback returns or ordered before the
+ * fg_stream position of the call that started the reconciliation (or, for a
+ * chunk appended during it, of that append).  It may set *out to a device
+ * buffer [n][num_q_heads][head_dim] that receives the chunk's rebuilt
+ * attention output, or leave it NULL.  Returns 0 on success; any other value
+ * aborts the reconciliation (the active version stays as it is), reported by
+ * the next csr_poll_swap / csr_wait_reconcile as CSR_ESTATE.
  */
 typedef int (*csr_qkv_provider)(void *user, int64_t chunk_id, int32_t n_tokens,
                                 const void **q, const void **k, const void **v,
@@ -192,8 +197,11 @@ typedef int (*csr_qkv_provider)(void *user, int64_t chunk_id, int32_t n_tokens,
 /*
  * Register the rebuild source and the low-priority stream on which the
  * rebuild runs (the secondary resource R_2 of Algorithm 1 becomes a stream of
- * the same GPU).  Create lo_stream with a lower priority than the foreground
- * stream.  CSR_EBUSY while a reconciliation runs.
+ * the same GPU, fed by a library thread that calls the provider and enqueues
+ * the rebuild's launches, so the foreground caller never waits for them).
+ * Create lo_stream with a lower priority than the foreground stream.  The
+ * thread starts at the first registration and ends in csr_destroy.
+ * CSR_EBUSY while a reconciliation runs.
  */
 csr_status csr_set_reconciler(csr_ctx *ctx, csr_qkv_provider provider,
                               void *user, csr_stream_t lo_stream);
@@ -206,10 +214,12 @@ csr_status csr_set_reconciler(csr_ctx *ctx, csr_qkv_provider provider,
  * kernel (new page table, copy of a partly filled prefix page) and a fresh
  * causal prefill of every retained chunk at its renumbered position.  Work
  * already enqueued on fg_stream is ordered before the rebuild.  Returns at
- * once; the active version keeps serving foreground calls.
+ * once, before the provider is called: the reconciliation thread enqueues the
+ * rebuild while the active version keeps serving foreground calls.
  * CSR_EBUSY if a reconciliation runs, CSR_ESTATE without a reconciler, with a
  * live suffix or with no chunk to evict, CSR_ENOMEM if the pool cannot hold
- * the second version.
+ * the second version.  A failure during the rebuild (the provider, a launch)
+ * is reported by the next csr_poll_swap / csr_wait_reconcile.
  */
 csr_status csr_evict_and_reconcile(csr_ctx *ctx, int32_t evict_tokens,
                                    csr_stream_t fg_stream);
@@ -227,7 +237,9 @@ csr_status csr_evict_and_reconcile(csr_ctx *ctx, int32_t evict_tokens,
  * their catch-up on the low-priority stream; otherwise compute the remaining
  * buffered chunks on fg_stream ("computed at next task inference") and swap
  * the active version atomically (App. D step 5).  The old version's own pages
- * return to the pool.  The swap waits while a suffix is live.
+ * return to the pool.  The swap waits while a suffix is live.  If the rebuild
+ * failed, the reconciliation is aborted (the pending version's pages return
+ * to the pool, the active version stays) and its error is returned.
  */
 csr_status csr_poll_swap(csr_ctx *ctx, csr_stream_t fg_stream, int *state);
 

@@ -12,7 +12,10 @@
 #include <atomic>
 #include <chrono>
 #include <cmath>
+#include <condition_variable>
 #include <cstring>
+#include <deque>
+#include <mutex>
 #include <string>
 #include <thread>
 #include <vector>
@@ -30,7 +33,7 @@ namespace {
 
 constexpr int kFgGridDefaultCap = 304;   // 2 x 152 SMs
 constexpr int kPartialItems = 4096;      // split partials a launch may write (per staging)
-constexpr int kDefaultRebuildTiles = 64;
+constexpr int kDefaultRebuildTiles = 16;
 constexpr size_t kAlign = 256;
 
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
@@ -185,6 +188,30 @@ Layout make_layout(const csr_config *c) {
   return L;
 }
 
+// One step of a rebuild, run in order on the low-priority stream by the
+// reconciliation worker: the compaction kernel, or the recomputation of one
+// chunk of the version being rebuilt.
+struct ReconTask {
+  EvictParams *compact = nullptr;  // compaction task (owned)
+  ChunkRec ch{};                   // chunk task: recompute ch at positions pos..
+  int64_t pos = 0;
+  std::vector<int32_t> ids;        // pages of logical pages first_lp.. (empty: read the table)
+  int32_t first_lp = 0;
+};
+
+// The secondary resource R_2 of Algorithm 1 on one GPU: a host thread that
+// calls the provider and enqueues the rebuild on the low-priority stream, so
+// the foreground caller never pays for it.
+struct Reconciler {
+  std::thread th;
+  std::mutex mu;
+  std::condition_variable cv;
+  std::deque<ReconTask> q;
+  bool busy = false, stop = false, started = false;
+  csr_status err = CSR_OK;
+  std::string err_msg;
+};
+
 }  // namespace
 
 struct csr_ctx {
@@ -204,16 +231,20 @@ struct csr_ctx {
   int64_t next_chunk_id = 0;
   // Algorithm 1 state
   bool reconciling = false;
-  std::vector<ChunkRec> buffer;      // Delta X_buffer
-  int64_t rebuilt_len = 0;           // length of the pending version computed so far
+  struct Buffered {
+    ChunkRec ch;
+    int64_t pos;
+  };
+  std::vector<Buffered> buffer;      // Delta X_buffer (N_catchup > 0): chunk and its position
   std::vector<int32_t> reserved_ids; // fresh ids the compaction kernel must produce
   bool ids_checked = false;
   csr_qkv_provider provider = nullptr;
   void *user = nullptr;
   cudaStream_t lo = nullptr;
   cudaEvent_t ev_fg = nullptr, ev_rb = nullptr;
-  int64_t launches = 0;
+  std::atomic<int64_t> launches{0};
   std::string err = "no error";
+  Reconciler rw;
   // per-kernel event timing of foreground launches
   struct Timed {
     int kind;
@@ -231,8 +262,15 @@ struct csr_ctx {
 
 namespace {
 
+// Errors raised on the reconciliation worker go to its own message, not to
+// the context's (which belongs to the caller's thread).
+thread_local std::string *t_err_sink = nullptr;
+
 csr_status fail(csr_ctx *c, csr_status s, const std::string &msg) {
-  if (c) c->err = msg;
+  if (t_err_sink)
+    *t_err_sink = msg;
+  else if (c)
+    c->err = msg;
   return s;
 }
 
@@ -292,7 +330,7 @@ cudaEvent_t take_event(csr_ctx *c) {
 // foreground launches while timing is enabled.
 template <class F>
 cudaError_t timed_launch(csr_ctx *c, int kind, bool foreground, cudaStream_t s, F fn) {
-  if (!(c->timing && foreground)) return fn();
+  if (!(foreground && c->timing)) return fn();
   cudaEvent_t a = take_event(c), b = take_event(c);
   if (!a || !b) return cudaErrorMemoryAllocation;
   cudaError_t e = cudaEventRecord(a, s);
@@ -408,7 +446,7 @@ csr_status run_block(csr_ctx *c, int slot, int ws, const void *q, const void *k,
 
 enum class Kind { Prefix, Chunk, Suffix };
 
-csr_status catch_up_now(csr_ctx *c);
+void push_chunk_task(csr_ctx *c, ChunkRec ch, int64_t pos, bool write_ids);
 
 csr_status add_block(csr_ctx *c, Kind kind, const void *q, const void *k, const void *v,
                      int32_t n, void *out, float *lse, cudaStream_t s, int64_t *chunk_id) {
@@ -456,10 +494,22 @@ csr_status add_block(csr_ctx *c, Kind kind, const void *q, const void *k, const 
     // Algorithm 1, Increment: fork the chunk into the rebuild; its pages in
     // the rebuilt version are reserved now (after the active ones).
     Version &B = c->pend();
+    const int64_t pos = B.length();
     for (int64_t i = 0; i < needB; ++i) B.pages.push_back(c->pool.take());
     B.chunks.push_back({id, n});
-    c->buffer.push_back({id, n});
-    if (c->cfg.n_catchup == 0) return catch_up_now(c);
+    if (c->cfg.n_catchup > 0) {
+      c->buffer.push_back({{id, n}, pos});
+    } else if (!c->plan_only) {
+      // N_catchup = 0: Algorithm 1's loop drains the whole buffer before the
+      // swap, so each chunk that arrives while reconciling goes to R_2 at
+      // once, in arrival order, after the foreground work that produced its
+      // inputs.  (Deferring it to the next poll would never drain the buffer
+      // while one chunk arrives per step.)
+      cudaError_t e = cudaEventRecord(c->ev_fg, s);
+      if (e == cudaSuccess) e = cudaStreamWaitEvent(c->lo, c->ev_fg, 0);
+      if (e != cudaSuccess) return cuda_fail(c, e, "ordering the catch-up after the foreground");
+      push_chunk_task(c, {id, n}, pos, true);
+    }
   }
   return CSR_OK;
 }
@@ -470,58 +520,131 @@ void drop_version(csr_ctx *c, Version &V) {
   V.clear();
 }
 
-// Abort a reconciliation: wait for its device work, give its pages back.
+// Recompute one chunk of the pending version at positions pos.. on stream s
+// (ws: staging buffers).  ids/first_lp name pages K1 writes into the device
+// table (empty: it reads the table).
+csr_status rebuild_chunk(csr_ctx *c, const ChunkRec &ch, int64_t pos,
+                         const std::vector<int32_t> &ids, int32_t first_lp, int ws,
+                         cudaStream_t s) {
+  const void *q = nullptr, *k = nullptr, *v = nullptr;
+  void *out = nullptr;
+  if (c->provider(c->user, ch.id, ch.len, &q, &k, &v, &out) != 0 || !q || !k || !v)
+    return fail(c, CSR_ESTATE, "qkv provider failed for chunk " + std::to_string(ch.id));
+  return run_block(c, 1 - c->active.load(), ws, q, k, v, ch.len, pos, ids.data(),
+                   static_cast<int32_t>(ids.size()), first_lp,
+                   out ? out : c->wsp<void>(c->lay.rb_out), nullptr, s);
+}
+
+// Worker side of Reconciler: run tasks in order, record ev_rb after each.
+void worker_main(csr_ctx *c) {
+  cudaSetDevice(c->device);
+  std::string msg;
+  t_err_sink = &msg;
+  std::unique_lock<std::mutex> lk(c->rw.mu);
+  while (true) {
+    c->rw.cv.wait(lk, [&] { return c->rw.stop || !c->rw.q.empty(); });
+    if (c->rw.q.empty()) return;  // stop requested
+    ReconTask t = std::move(c->rw.q.front());
+    c->rw.q.pop_front();
+    c->rw.busy = true;
+    const bool skip = c->rw.err != CSR_OK;  // after a failure the rest is dropped
+    lk.unlock();
+    csr_status st = CSR_OK;
+    msg.clear();
+    if (!skip) {
+      if (t.compact) {
+        const cudaError_t e = launch_evict(*t.compact, c->lo);
+        if (e != cudaSuccess) st = cuda_fail(c, e, "evict_compact launch");
+        else ++c->launches;
+      } else {
+        st = rebuild_chunk(c, t.ch, t.pos, t.ids, t.first_lp, 1, c->lo);
+      }
+      if (st == CSR_OK) {
+        const cudaError_t e = cudaEventRecord(c->ev_rb, c->lo);
+        if (e != cudaSuccess) st = cuda_fail(c, e, "recording the rebuild event");
+      }
+    }
+    delete t.compact;
+    lk.lock();
+    if (st != CSR_OK && c->rw.err == CSR_OK) {
+      c->rw.err = st;
+      c->rw.err_msg = msg;
+    }
+    c->rw.busy = false;
+    c->rw.cv.notify_all();
+  }
+}
+
+void start_worker(csr_ctx *c) {
+  if (c->rw.started || c->plan_only) return;
+  c->rw.stop = false;
+  c->rw.th = std::thread(worker_main, c);
+  c->rw.started = true;
+}
+
+void stop_worker(csr_ctx *c) {
+  if (!c->rw.started) return;
+  {
+    std::lock_guard<std::mutex> lk(c->rw.mu);
+    for (auto &t : c->rw.q) delete t.compact;
+    c->rw.q.clear();
+    c->rw.stop = true;
+  }
+  c->rw.cv.notify_all();
+  c->rw.th.join();
+  c->rw.started = false;
+}
+
+void push_task(csr_ctx *c, ReconTask t) {
+  {
+    std::lock_guard<std::mutex> lk(c->rw.mu);
+    c->rw.q.push_back(std::move(t));
+  }
+  c->rw.cv.notify_all();
+}
+
+// Enqueue the recomputation of chunk `ch` of the pending version at `pos`;
+// write_ids: K1 writes the chunk's page ids (pages reserved after the
+// compaction ran) into the device table.
+void push_chunk_task(csr_ctx *c, ChunkRec ch, int64_t pos, bool write_ids) {
+  ReconTask t;
+  t.ch = ch;
+  t.pos = pos;
+  if (write_ids) {
+    const Version &B = c->pend();
+    t.first_lp = static_cast<int32_t>(pos / c->cfg.page_size);
+    const int64_t last = pages_for(c, pos + ch.len);
+    t.ids.assign(B.pages.begin() + t.first_lp, B.pages.begin() + last);
+  }
+  push_task(c, std::move(t));
+}
+
+// Wait until the worker has nothing queued or running.
+void wait_worker_idle(csr_ctx *c) {
+  if (!c->rw.started) return;
+  std::unique_lock<std::mutex> lk(c->rw.mu);
+  c->rw.cv.wait(lk, [&] { return c->rw.q.empty() && !c->rw.busy; });
+}
+
+// Abort a reconciliation: drop queued work, wait for the device, give the
+// rebuilt version's pages back.
 void abort_reconcile(csr_ctx *c) {
+  if (c->rw.started) {
+    {
+      std::lock_guard<std::mutex> lk(c->rw.mu);
+      for (auto &t : c->rw.q) delete t.compact;
+      c->rw.q.clear();
+    }
+    wait_worker_idle(c);
+    std::lock_guard<std::mutex> lk(c->rw.mu);
+    c->rw.err = CSR_OK;
+    c->rw.err_msg.clear();
+  }
   if (!c->plan_only && c->lo) cudaStreamSynchronize(c->lo);
   drop_version(c, c->pend());
   c->reconciling = false;
   c->buffer.clear();
   c->reserved_ids.clear();
-}
-
-// Recompute `chunks` of the pending version on stream s, starting at position
-// c->rebuilt_len (the catch-up of Algorithm 1, or the remainder at the swap).
-csr_status materialise(csr_ctx *c, const std::vector<ChunkRec> &chunks, int ws, cudaStream_t s) {
-  const int slot = 1 - c->active.load();
-  Version &B = c->pend();
-  for (const ChunkRec &ch : chunks) {
-    const void *q = nullptr, *k = nullptr, *v = nullptr;
-    void *out = nullptr;
-    if (c->provider(c->user, ch.id, ch.len, &q, &k, &v, &out) != 0 || !q || !k || !v)
-      return fail(c, CSR_ESTATE, "qkv provider failed for chunk " + std::to_string(ch.id));
-    const int64_t L = c->rebuilt_len;
-    const int32_t first_lp = static_cast<int32_t>(L / c->cfg.page_size);
-    const int32_t n_ids = static_cast<int32_t>(pages_for(c, L + ch.len)) - first_lp;
-    csr_status st = run_block(c, slot, ws, q, k, v, ch.len, L, B.pages.data() + first_lp, n_ids,
-                              first_lp, out ? out : c->wsp<void>(c->lay.rb_out), nullptr, s);
-    if (st != CSR_OK) return st;
-    c->rebuilt_len += ch.len;
-  }
-  return CSR_OK;
-}
-
-// N_catchup = 0: Algorithm 1's reconcile loop drains the buffer completely
-// before the swap.  On one GPU the low-priority stream is R_2's queue, so each
-// chunk that arrives while reconciling is appended to X_eps on that stream as
-// soon as it is buffered (in arrival order); the swap happens at the first
-// poll after the stream has finished.  (Computing the buffer only when a poll
-// finds the previous round done would never drain it while one chunk arrives
-// per step.)
-csr_status catch_up_now(csr_ctx *c) {
-  std::vector<ChunkRec> batch;
-  batch.swap(c->buffer);
-  if (c->plan_only) {
-    for (const auto &ch : batch) c->rebuilt_len += ch.len;
-    return CSR_OK;
-  }
-  csr_status st = materialise(c, batch, 1, c->lo);
-  if (st != CSR_OK) {
-    abort_reconcile(c);
-    return st;
-  }
-  const cudaError_t e = cudaEventRecord(c->ev_rb, c->lo);
-  if (e != cudaSuccess) return cuda_fail(c, e, "recording the catch-up event");
-  return CSR_OK;
 }
 
 }  // namespace
@@ -609,6 +732,7 @@ csr_status csr_create(const csr_config *cfg, void *k_pool, void *v_pool, void *w
 
 void csr_destroy(csr_ctx *c) {
   if (!c) return;
+  stop_worker(c);
   if (!c->plan_only) {
     if (c->lo) cudaStreamSynchronize(c->lo);
     cudaDeviceSynchronize();
@@ -693,9 +817,11 @@ csr_status csr_set_reconciler(csr_ctx *c, csr_qkv_provider provider, void *user,
                               csr_stream_t lo_stream) {
   if (!c) return CSR_EINVAL;
   if (c->reconciling) return fail(c, CSR_EBUSY, "a reconciliation is running");
+  wait_worker_idle(c);
   c->provider = provider;
   c->user = user;
   c->lo = reinterpret_cast<cudaStream_t>(lo_stream);
+  if (provider) start_worker(c);
   return CSR_OK;
 }
 
@@ -745,11 +871,7 @@ csr_status csr_evict_and_reconcile(csr_ctx *c, int32_t evict_tokens, csr_stream_
   c->reconciling = true;
   c->buffer.clear();
   c->ids_checked = c->plan_only;
-  c->rebuilt_len = A.prefix_len;
-  if (c->plan_only) {
-    for (const auto &ch : retained) c->rebuilt_len += ch.len;
-    return CSR_OK;
-  }
+  if (c->plan_only) return CSR_OK;
   const cudaStream_t fg = reinterpret_cast<cudaStream_t>(fg_stream);
   cudaError_t e = cudaEventRecord(c->ev_fg, fg);
   if (e == cudaSuccess) e = cudaStreamWaitEvent(c->lo, c->ev_fg, 0);
@@ -771,36 +893,16 @@ csr_status csr_evict_and_reconcile(csr_ctx *c, int32_t evict_tokens, csr_stream_
   ep->page_size = P;
   ep->d = c->cfg.head_dim;
   ep->pool_pages = c->cfg.pool_pages;
-  e = launch_evict(*ep, c->lo);
-  delete ep;
-  if (e != cudaSuccess) {
-    abort_reconcile(c);
-    return cuda_fail(c, e, "evict_compact launch");
-  }
-  ++c->launches;
-  // Warm-up (LLM(X_eps) on the secondary resource): a fresh causal prefill of
-  // every retained chunk at its renumbered position, reading the page table
-  // the compaction kernel wrote.
-  const int slot = 1 - act_slot;
+  // Hand the rebuild to R_2: the compaction kernel, then the warm-up
+  // (LLM(X_eps)): a fresh causal prefill of every retained chunk at its
+  // renumbered position, reading the page table the compaction kernel wrote.
+  ReconTask t;
+  t.compact = ep;
+  push_task(c, std::move(t));
+  int64_t pos = A.prefix_len;
   for (const ChunkRec &ch : retained) {
-    const void *q = nullptr, *k2 = nullptr, *v = nullptr;
-    void *out = nullptr;
-    if (c->provider(c->user, ch.id, ch.len, &q, &k2, &v, &out) != 0 || !q || !k2 || !v) {
-      abort_reconcile(c);
-      return fail(c, CSR_ESTATE, "qkv provider failed for chunk " + std::to_string(ch.id));
-    }
-    csr_status st = run_block(c, slot, 1, q, k2, v, ch.len, c->rebuilt_len, nullptr, 0, 0,
-                              out ? out : c->wsp<void>(c->lay.rb_out), nullptr, c->lo);
-    if (st != CSR_OK) {
-      abort_reconcile(c);
-      return st;
-    }
-    c->rebuilt_len += ch.len;
-  }
-  e = cudaEventRecord(c->ev_rb, c->lo);
-  if (e != cudaSuccess) {
-    abort_reconcile(c);
-    return cuda_fail(c, e, "recording the rebuild event");
+    push_chunk_task(c, ch, pos, false);
+    pos += ch.len;
   }
   return CSR_OK;
 }
@@ -813,6 +915,22 @@ csr_status csr_poll_swap(csr_ctx *c, csr_stream_t fg_stream, int *state) {
   }
   *state = CSR_RECON_RUNNING;
   if (!c->plan_only) {
+    // R_2 is done when its queue is empty and its last launch has finished;
+    // a task that failed there aborts the reconciliation here.
+    bool idle = false;
+    csr_status werr = CSR_OK;
+    std::string wmsg;
+    {
+      std::lock_guard<std::mutex> lk(c->rw.mu);
+      idle = c->rw.q.empty() && !c->rw.busy;
+      werr = c->rw.err;
+      wmsg = c->rw.err_msg;
+    }
+    if (!idle) return CSR_OK;
+    if (werr != CSR_OK) {
+      abort_reconcile(c);
+      return fail(c, werr, wmsg);
+    }
     const cudaError_t q = cudaEventQuery(c->ev_rb);
     if (q == cudaErrorNotReady) return CSR_OK;
     if (q != cudaSuccess) return cuda_fail(c, q, "rebuild event");
@@ -834,34 +952,35 @@ csr_status csr_poll_swap(csr_ctx *c, csr_stream_t fg_stream, int *state) {
   }
   // Algorithm 1: while |buffer| > N_catchup, catch up on the secondary resource.
   if (static_cast<int64_t>(c->buffer.size()) > c->cfg.n_catchup) {
-    std::vector<ChunkRec> batch;
+    std::vector<csr_ctx::Buffered> batch;
     batch.swap(c->buffer);
     if (!c->plan_only) {
-      csr_status st = materialise(c, batch, 1, c->lo);
-      if (st != CSR_OK) {
-        abort_reconcile(c);
-        return st;
-      }
-      const cudaError_t e = cudaEventRecord(c->ev_rb, c->lo);
-      if (e != cudaSuccess) return cuda_fail(c, e, "recording the catch-up event");
-    } else {
-      for (const auto &ch : batch) c->rebuilt_len += ch.len;
+      const cudaStream_t fg = reinterpret_cast<cudaStream_t>(fg_stream);
+      cudaError_t e = cudaEventRecord(c->ev_fg, fg);
+      if (e == cudaSuccess) e = cudaStreamWaitEvent(c->lo, c->ev_fg, 0);
+      if (e != cudaSuccess) return cuda_fail(c, e, "ordering the catch-up after the foreground");
+      for (const auto &b : batch) push_chunk_task(c, b.ch, b.pos, true);
     }
     return CSR_OK;
   }
   if (c->act().suffix_len > 0) return CSR_OK;  // swap only between tasks
   // The remainder (<= N_catchup chunks) is computed now, on the foreground.
   if (!c->buffer.empty()) {
-    std::vector<ChunkRec> rest;
+    std::vector<csr_ctx::Buffered> rest;
     rest.swap(c->buffer);
     if (!c->plan_only) {
-      csr_status st = materialise(c, rest, 0, reinterpret_cast<cudaStream_t>(fg_stream));
-      if (st != CSR_OK) {
-        abort_reconcile(c);
-        return st;
+      const cudaStream_t fg = reinterpret_cast<cudaStream_t>(fg_stream);
+      const Version &B = c->pend();
+      for (const auto &b : rest) {
+        const int32_t first_lp = static_cast<int32_t>(b.pos / c->cfg.page_size);
+        const int64_t last = pages_for(c, b.pos + b.ch.len);
+        std::vector<int32_t> ids(B.pages.begin() + first_lp, B.pages.begin() + last);
+        csr_status st = rebuild_chunk(c, b.ch, b.pos, ids, first_lp, 0, fg);
+        if (st != CSR_OK) {
+          abort_reconcile(c);
+          return st;
+        }
       }
-    } else {
-      for (const auto &ch : rest) c->rebuilt_len += ch.len;
     }
   }
   // Atomic swap of the active version (App. D step 5); the old version's own
@@ -997,7 +1116,7 @@ csr_status csr_device_status(csr_ctx *c, uint32_t *flags) {
   return CSR_OK;
 }
 
-int64_t csr_kernel_launches(const csr_ctx *c) { return c ? c->launches : 0; }
+int64_t csr_kernel_launches(const csr_ctx *c) { return c ? c->launches.load() : 0; }
 
 csr_status csr_set_timing(csr_ctx *c, int enable) {
   if (!c) return CSR_EINVAL;

@@ -125,9 +125,13 @@ def test_provider_failure_keeps_old_version(libcsr):
     for i in range(4):
         p.append(p.blk(951 + i, 32))
     snap = (p.ctx.layout(), p.ctx.free_pages())
+    # the call returns before the provider runs (on the reconciliation
+    # thread); the failure surfaces at the next wait/poll, which aborts
+    p.ctx.evict_and_reconcile(32)
     with pytest.raises(csr.CsrError) as e:
-        p.ctx.evict_and_reconcile(32)
+        p.ctx.wait_reconcile(30.0)
     assert e.value.status == csr.ESTATE
+    assert "provider" in str(e.value)
     assert (p.ctx.layout(), p.ctx.free_pages()) == snap
     assert p.ctx.poll_swap() == csr.RECON_IDLE
     p.suffix(p.blk(960, 9))
