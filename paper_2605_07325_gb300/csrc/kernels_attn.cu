@@ -717,94 +717,95 @@ __global__ void __launch_bounds__(kPairThreads, 1) attn_pair_kernel(const __grid
         drain_wait(&bars->v_full[i % C::kStages], (i / C::kStages) & 1);
     }
   } else if (warp == 9) {
-    if (lane == 0) {
-      // ------------------------------------------------------ MMA issuer
-      constexpr uint32_t idesc_s = idesc_bf16_f32(kBM, kBN, false, false);
-      constexpr uint32_t idesc_pv = idesc_bf16_f32(kBM, HD, false, true);
-      const uint32_t q_base = smem_u32(smem + C::kQOff);
-      const uint32_t k_base = smem_u32(smem + C::kKOff);
-      const uint32_t v_base = smem_u32(smem + C::kVOff);
-      uint32_t q_round = 0, k_it = 0, v_it = 0, seg_n = 0;
-      uint32_t pv_n[2] = {0, 0};
-      bool ok = true;
-      auto wait = [&](uint64_t *bar, uint32_t parity) {
-        if (ok && !mbar_wait(bar, parity, abort, p.err, CSR_DEVERR_WAIT_TIMEOUT)) ok = false;
-        return ok;
-      };
-      // S_X = Q_X K^T for tile x from K stage ks
-      auto issue_s = [&](int x, int ks) {
-        const uint32_t qx = q_base + x * C::kQBytes;
-        const uint32_t kst = k_base + ks * C::kTileBytes;
+    // ------------------------------------------------------ MMA issuer
+    // The whole warp runs the issue loop (operands are warp-uniform) and an
+    // elected lane issues each MMA and commit.
+    constexpr uint32_t idesc_s = idesc_bf16_f32(kBM, kBN, false, false);
+    constexpr uint32_t idesc_pv = idesc_bf16_f32(kBM, HD, false, true);
+    const uint64_t q_desc = sdesc_sw128(smem_u32(smem + C::kQOff), 16, 1024);
+    const uint64_t k_desc = sdesc_sw128(smem_u32(smem + C::kKOff), 16, 1024);
+    const uint64_t v_desc = sdesc_sw128(smem_u32(smem + C::kVOff), kBN * 128, 1024);
+    uint32_t q_round = 0, k_it = 0, v_it = 0, seg_n = 0;
+    uint32_t pv_n[2] = {0, 0};
+    bool ok = true;
+    auto wait = [&](uint64_t *bar, uint32_t parity) {
+      if (ok)
+        ok = __all_sync(0xffffffffu, mbar_wait(bar, parity, abort, p.err, CSR_DEVERR_WAIT_TIMEOUT));
+      return ok;
+    };
+    // S_X = Q_X K^T for tile x from K stage ks
+    auto issue_s = [&](int x, int ks) {
+      const uint64_t qx = sdesc_advance(q_desc, x * C::kQBytes);
+      const uint64_t kst = sdesc_advance(k_desc, ks * C::kTileBytes);
 #pragma unroll
-        for (int kk = 0; kk < HD / 16; ++kk) {
-          const uint64_t a = sdesc_sw128(qx + (kk >> 2) * (kBM * 128) + (kk & 3) * 32, 16, 1024);
-          const uint64_t b = sdesc_sw128(kst + (kk >> 2) * (kBN * 128) + (kk & 3) * 32, 16, 1024);
-          mma_bf16_ss(tmem + x * kBN, a, b, idesc_s, kk > 0 ? 1u : 0u);
-        }
-        mma_commit(&bars->s_full[x]);
-      };
-      // O_X += P_X V for tile x from V stage vs
-      auto issue_pv = [&](int x, int vs, bool first) {
-        const uint32_t vst = v_base + vs * C::kTileBytes;
+      for (int kk = 0; kk < HD / 16; ++kk) {
+        const uint32_t off = (kk >> 2) * (kBM * 128) + (kk & 3) * 32;
+        mma_bf16_ss_warp(tmem + x * kBN, sdesc_advance(qx, off),
+                         sdesc_advance(kst, (kk >> 2) * (kBN * 128) + (kk & 3) * 32), idesc_s,
+                         kk > 0 ? 1u : 0u);
+      }
+      mma_commit_warp(&bars->s_full[x]);
+    };
+    // O_X += P_X V for tile x from V stage vs
+    auto issue_pv = [&](int x, int vs, bool first) {
+      const uint64_t vst = sdesc_advance(v_desc, vs * C::kTileBytes);
 #pragma unroll
-        for (int kk = 0; kk < kBN / 16; ++kk) {
-          const uint64_t b = sdesc_sw128(vst + kk * (16 * 128), kBN * 128, 1024);
-          mma_bf16_ts(tmem + C::kOCol + x * HD, tmem + x * kBN + kk * 8, b, idesc_pv,
-                      (!first || kk > 0) ? 1u : 0u);
-        }
-      };
-      while (ok && walk.next(p, T, seg)) {
-        if (!wait(&bars->q_full, q_round & 1)) break;
-        ++q_round;
+      for (int kk = 0; kk < kBN / 16; ++kk)
+        mma_bf16_ts_warp(tmem + C::kOCol + x * HD, tmem + x * kBN + kk * 8,
+                         sdesc_advance(vst, kk * (16 * 128)), idesc_pv,
+                         (!first || kk > 0) ? 1u : 0u);
+    };
+    while (ok && walk.next(p, T, seg)) {
+      if (!wait(&bars->q_full, q_round & 1)) break;
+      ++q_round;
+      tc_fence_after();
+      const int nj = static_cast<int>(seg.j1 - seg.j0);
+      int ks = k_it % C::kStages;
+      if (!wait(&bars->k_full[ks], (k_it / C::kStages) & 1)) break;
+      tc_fence_after();
+      issue_s(0, ks);
+      issue_s(1, ks);
+      mma_commit_warp(&bars->k_empty[ks]);
+      ++k_it;
+      if (nj == 1) mma_commit_warp(&bars->q_empty);
+      for (int i = 0; i < nj; ++i) {
+        const int vs = v_it % C::kStages;
+        const bool more = i + 1 < nj;
+        // ---- tile A
+        if (!wait(&bars->p_full[0], pv_n[0] & 1)) break;
+        if (!wait(&bars->v_full[vs], (v_it / C::kStages) & 1)) break;
+        if (i == 0 && seg_n > 0 && !wait(&bars->o_free[0], (seg_n & 1) ^ 1)) break;
         tc_fence_after();
-        const int nj = static_cast<int>(seg.j1 - seg.j0);
-        int ks = k_it % C::kStages;
-        if (!wait(&bars->k_full[ks], (k_it / C::kStages) & 1)) break;
-        tc_fence_after();
-        issue_s(0, ks);
-        issue_s(1, ks);
-        mma_commit(&bars->k_empty[ks]);
-        ++k_it;
-        if (nj == 1) mma_commit(&bars->q_empty);
-        for (int i = 0; i < nj; ++i) {
-          const int vs = v_it % C::kStages;
-          const bool more = i + 1 < nj;
-          // ---- tile A
-          if (!wait(&bars->p_full[0], pv_n[0] & 1)) break;
-          if (!wait(&bars->v_full[vs], (v_it / C::kStages) & 1)) break;
-          if (i == 0 && seg_n > 0 && !wait(&bars->o_free[0], (seg_n & 1) ^ 1)) break;
+        issue_pv(0, vs, i == 0);
+        if (i == nj - 1) mma_commit_warp(&bars->o_final[0]);
+        ++pv_n[0];
+        if (more) {
+          ks = k_it % C::kStages;
+          if (!wait(&bars->k_full[ks], (k_it / C::kStages) & 1)) break;
           tc_fence_after();
-          issue_pv(0, vs, i == 0);
-          if (i == nj - 1) mma_commit(&bars->o_final[0]);
-          ++pv_n[0];
-          if (more) {
-            ks = k_it % C::kStages;
-            if (!wait(&bars->k_full[ks], (k_it / C::kStages) & 1)) break;
-            tc_fence_after();
-            issue_s(0, ks);
-          }
-          // ---- tile B
-          if (!wait(&bars->p_full[1], pv_n[1] & 1)) break;
-          if (i == 0 && seg_n > 0 && !wait(&bars->o_free[1], (seg_n & 1) ^ 1)) break;
-          tc_fence_after();
-          issue_pv(1, vs, i == 0);
-          if (i == nj - 1) mma_commit(&bars->o_final[1]);
-          ++pv_n[1];
-          mma_commit(&bars->v_empty[vs]);
-          ++v_it;
-          if (more) {
-            issue_s(1, ks);
-            mma_commit(&bars->k_empty[ks]);
-            ++k_it;
-            if (i + 1 == nj - 1) mma_commit(&bars->q_empty);
-          }
+          issue_s(0, ks);
         }
-        ++seg_n;
+        // ---- tile B
+        if (!wait(&bars->p_full[1], pv_n[1] & 1)) break;
+        if (i == 0 && seg_n > 0 && !wait(&bars->o_free[1], (seg_n & 1) ^ 1)) break;
+        tc_fence_after();
+        issue_pv(1, vs, i == 0);
+        if (i == nj - 1) mma_commit_warp(&bars->o_final[1]);
+        ++pv_n[1];
+        mma_commit_warp(&bars->v_empty[vs]);
+        ++v_it;
+        if (more) {
+          issue_s(1, ks);
+          mma_commit_warp(&bars->k_empty[ks]);
+          ++k_it;
+          if (i + 1 == nj - 1) mma_commit_warp(&bars->q_empty);
+        }
       }
-      if (!ok) {
-        mma_commit(&bars->drain);
-        drain_wait(&bars->drain, 0);
-      }
+      ++seg_n;
+    }
+    if (!ok) {
+      mma_commit_warp(&bars->drain);
+      drain_wait(&bars->drain, 0);
     }
   } else {
     // ------------------------------------------------------ softmax warpgroups
