@@ -844,13 +844,14 @@ __global__ void __launch_bounds__(kPairThreads, 1) attn_pair_kernel(const __grid
           for (int c = 0; c < kBN; ++c)
             if (key0 + c > limit) s[c] = -CUDART_INF_F;
         }
+        // Row max: three operands per instruction, eight independent chains.
         float mp[8];
 #pragma unroll
-        for (int e = 0; e < 8; ++e) mp[e] = s[e];
+        for (int e = 0; e < 8; ++e) mp[e] = fmaxf(s[2 * e], s[2 * e + 1]);
 #pragma unroll
-        for (int c = 8; c < kBN; ++c) mp[c & 7] = fmaxf(mp[c & 7], s[c]);
-        const float mx = fmaxf(fmaxf(fmaxf(mp[0], mp[1]), fmaxf(mp[2], mp[3])),
-                               fmaxf(fmaxf(mp[4], mp[5]), fmaxf(mp[6], mp[7])));
+        for (int c = 16; c < kBN; c += 2) mp[(c >> 1) & 7] = max3f(mp[(c >> 1) & 7], s[c], s[c + 1]);
+        const float mx = max3f(max3f(mp[0], mp[1], mp[2]), max3f(mp[3], mp[4], mp[5]),
+                               fmaxf(mp[6], mp[7]));
         const float mx_s = mx * p.scale_log2;
         const bool need = mx_s > m_ref + 8.0f;
         const float m_new = need ? mx_s : m_ref;
@@ -859,18 +860,27 @@ __global__ void __launch_bounds__(kPairThreads, 1) attn_pair_kernel(const __grid
         l *= alpha;
         m_ref = m_new;
         const float m_use = (m_ref == -CUDART_INF_F) ? 0.f : m_ref;
-        float rp[8];
+        // p = 2^(s * scale_log2 - m): the scale-and-shift and the row sum run
+        // on packed fp32 pairs, the exponentials one lane at a time.
+        const uint64_t scale2 = f32x2(p.scale_log2, p.scale_log2);
+        const uint64_t shift2 = f32x2(-m_use, -m_use);
+        uint64_t rp2[4];
 #pragma unroll
-        for (int e = 0; e < 8; ++e) rp[e] = 0.f;
+        for (int e = 0; e < 4; ++e) rp2[e] = 0ull;  // (+0.0f, +0.0f)
         uint32_t pk[kBN / 2];
 #pragma unroll
         for (int c = 0; c < kBN; c += 2) {
-          const float p0 = ex2_approx(fmaf(s[c], p.scale_log2, -m_use));
-          const float p1 = ex2_approx(fmaf(s[c + 1], p.scale_log2, -m_use));
-          rp[(c >> 1) & 7] += p0 + p1;
+          float x0, x1;
+          f32x2_split(fma_f32x2(f32x2(s[c], s[c + 1]), scale2, shift2), x0, x1);
+          const float p0 = ex2_approx(x0);
+          const float p1 = ex2_approx(x1);
+          rp2[(c >> 1) & 3] = add_f32x2(rp2[(c >> 1) & 3], f32x2(p0, p1));
           pk[c / 2] = pack_bf16x2(p0, p1);
         }
-        l += ((rp[0] + rp[1]) + (rp[2] + rp[3])) + ((rp[4] + rp[5]) + (rp[6] + rp[7]));
+        float r[8];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) f32x2_split(rp2[e], r[2 * e], r[2 * e + 1]);
+        l += ((r[0] + r[1]) + (r[2] + r[3])) + ((r[4] + r[5]) + (r[6] + r[7]));
         tmem_st64(tmem + lane_base + s_col, pk);
         // PV of the previous tile finished before these scores were published
         // (same commit), so O can be rescaled here without another wait.
