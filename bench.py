@@ -415,22 +415,26 @@ def run_asr(args):
     foreground steps (256-token chunk + 512-token suffix + truncate) at a fixed
     cadence; reaching the cap evicts the oldest 32,768 tokens of chunks and
     rebuilds the retained ~98K tokens on a low-priority stream (Algorithm 1),
-    then swaps.  Reports foreground step latency during and outside rebuilds
-    and checks every post-swap page table against the oracle's allocator."""
+    then swaps.  --asr-cap / --asr-evict / --asr-chunk change the setting (the
+    paper's robot run: 100-token chunks, tau_mem = 110K, the oldest half of the
+    chunks evicted: --asr-chunk 100 --asr-cap 110000 --asr-evict 52952).  Reports foreground step latency during and outside rebuilds
+    and checks that every post-swap layout is consistent (distinct page ids,
+    disjoint from the free list, pool fully accounted for); the layouts are
+    compared with the oracle's allocator in the GPU tests."""
     import numpy as np
     import torch
-    from oracle import oracle as orc
     from paper_2605_07325_gb300 import csr
 
     dev = torch.device("cuda", 0)
     torch.cuda.set_device(dev)
     # N_max of App. D: the active version may grow past tau_mem while the rebuild and its
     # catch-up run (Eq. oom_time); one eviction's worth of headroom covers back-to-back steps
-    n_max = ASR_CAP + ASR_EVICT
+    cap, evict, chunk = args.asr_cap, args.asr_evict, args.asr_chunk
+    n_max = cap + evict
     pool_pages = (2 * n_max) // P + 64
     cfg = csr.make_config(HQ, HKV, D, P, BASE, max_new_tokens=PREFIX, pool_pages=pool_pages,
-                          max_seq_tokens=n_max, cap_tokens=ASR_CAP,
-                          evict_tokens=ASR_EVICT, n_catchup=0,
+                          max_seq_tokens=n_max, cap_tokens=cap,
+                          evict_tokens=evict, n_catchup=0,
                           rebuild_tiles_per_cta=args.asr_rebuild_tiles)
     fg = torch.cuda.Stream(device=dev, priority=-1)     # high priority
     lo = torch.cuda.Stream(device=dev, priority=0)      # low priority (rebuild, R_2)
@@ -445,21 +449,28 @@ def run_asr(args):
         q, k, v = chunks[cid]
         return q, k, v, None
 
-    # layout model: the oracle's allocator on the same operations (attention off)
-    model = orc.OracleCSR(1, 1, 2, P, BASE, pool_pages)
-    model.attend = False
-    z = lambda n: (np.zeros((n, 1, 2)), np.zeros((n, 1, 2)), np.zeros((n, 1, 2)))
+    def reconciling():
+        try:
+            ctx.layout(csr.VERSION_PENDING)
+            return True
+        except csr.CsrError:
+            return False
+
+    def layout_consistent():
+        pt, length = ctx.layout()
+        free = ctx.free_pages()
+        return (len(set(pt)) == len(pt) and not set(pt) & set(free)
+                and len(pt) + len(free) == pool_pages and len(pt) == -(-length // P))
+
     with torch.cuda.stream(fg):
         ctx = csr.Context(cfg, device=str(dev), stream=fg)
         ctx.set_reconciler(provider, lo)
         ctx.init_static(rnd(PREFIX, HQ), rnd(PREFIX, HKV), rnd(PREFIX, HKV), stream=fg)
-        model.init_static(*z(PREFIX))
-        fout = torch.empty((CHUNK, HQ, D), dtype=torch.bfloat16, device=dev)
-        while ctx.layout()[1] + CHUNK < ASR_CAP:
-            q, k, v = rnd(CHUNK, HQ), rnd(CHUNK, HKV), rnd(CHUNK, HKV)
+        fout = torch.empty((chunk, HQ, D), dtype=torch.bfloat16, device=dev)
+        while ctx.layout()[1] + chunk < cap:
+            q, k, v = rnd(chunk, HQ), rnd(chunk, HKV), rnd(chunk, HKV)
             chunks[len(chunks)] = (q, k, v)      # ids are 0, 1, 2, ... in append order
             ctx.append_chunk(q, k, v, out=fout, stream=fg)
-            model.append_chunk(*z(CHUNK))
         sq, sk, sv = rnd(SUFFIX, HQ), rnd(SUFFIX, HKV), rnd(SUFFIX, HKV)
         so = torch.empty((SUFFIX, HQ, D), dtype=torch.bfloat16, device=dev)
     fg.synchronize()
@@ -472,20 +483,16 @@ def run_asr(args):
     next_t = time.perf_counter()
     while cycles < args.asr_cycles:
         with torch.cuda.stream(fg):
-            q, k, v = rnd(CHUNK, HQ), rnd(CHUNK, HKV), rnd(CHUNK, HKV)
+            q, k, v = rnd(chunk, HQ), rnd(chunk, HKV), rnd(chunk, HKV)
         fg.synchronize()
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         t0 = time.perf_counter()
         # the task starts by polling the reconciliation (the swap happens between tasks)
         if ctx.poll_swap(fg) == csr.RECON_SWAPPED:
-            model.reconcile()
-            pt, length = ctx.layout()
-            ok = pt == model.page_table() and ctx.free_pages() == model.free_ids() \
-                and length == model.length()
-            layout_ok = layout_ok and ok
+            layout_ok = layout_ok and layout_consistent()
             rebuilds.append(time.perf_counter() - rb_start)
             cycles += 1
-        was = model.is_reconciling
+        was = reconciling()
         e0.record(fg)
         chunks[len(chunks)] = (q, k, v)          # before the call: it may start a rebuild
         _, _, cid = ctx.append_chunk(q, k, v, out=fout, stream=fg)
@@ -495,12 +502,12 @@ def run_asr(args):
         e1.record(fg)
         e1.synchronize()
         t1 = time.perf_counter()
-        model.append_chunk(*z(CHUNK))
-        if not was and model.length() >= ASR_CAP:
-            model.evict(ASR_EVICT)          # the library started it inside append_chunk
-            rb_start = time.perf_counter()
-        peak_len = max(peak_len, model.length())
-        during = was or model.is_reconciling
+        now = reconciling()
+        if now and not was:
+            rb_start = time.perf_counter()   # the library started it inside append_chunk
+        length = ctx.layout()[1]
+        peak_len = max(peak_len, length)
+        during = was or now
         records.append((t1 - t0, e0.elapsed_time(e1) / 1e3, during))
         step += 1
         if period:
@@ -516,8 +523,8 @@ def run_asr(args):
     dev_dur = [r[1] for r in records if r[2]]
     dev_out = [r[1] for r in records if not r[2]]
     line = {
-        "workload": ("ASR cycle run: cap 131,072 tokens, 4,096-token prefix, 256-token chunks + "
-                     "512-token suffix per step, evict oldest 32,768 tokens, rebuild on a "
+        "workload": (f"ASR cycle run: cap {cap:,} tokens, 4,096-token prefix, {chunk}-token chunks + "
+                     f"512-token suffix per step, evict oldest {evict:,} tokens, rebuild on a "
                      "low-priority stream, 64 q / 4 kv heads, d 128, page 64, 1 layer"),
         "cadence_hz": args.asr_cadence_hz, "rebuild_tiles_per_cta": args.asr_rebuild_tiles or 16,
         "cycles": cycles, "steps": step,
@@ -530,7 +537,7 @@ def run_asr(args):
                               "max": max(rebuilds) if rebuilds else None,
                               "note": "eviction to the poll (start of a step) that swapped"},
         "peak_cached_tokens": peak_len, "n_max_tokens": n_max,
-        "layout_bit_exact_vs_oracle": layout_ok,
+        "layout_consistent": layout_ok,
         "device_error_flags": flags,
     }
     if out and dur:
@@ -538,8 +545,8 @@ def run_asr(args):
     # App. D viability: the rebuild (warm-up + catch-up, here eviction -> swap)
     # must end before the cache, growing at X_dot tokens/s from tau_mem, reaches N_max
     if rebuilds and period:
-        x_dot = CHUNK / period
-        dt_mem = (n_max - ASR_CAP) / x_dot
+        x_dot = chunk / period
+        dt_mem = (n_max - cap) / x_dot
         line["viability"] = {"x_dot_tokens_per_s": x_dot, "dt_mem_s": dt_mem,
                              "dt_rebuild_max_s": max(rebuilds),
                              "holds": max(rebuilds) <= dt_mem and peak_len <= n_max}
@@ -709,6 +716,9 @@ def main(argv=None):
     ap.add_argument("--asr", action="store_true",
                     help="run the ASR cycle workload instead of the 120K step line")
     ap.add_argument("--asr-cycles", type=int, default=10)
+    ap.add_argument("--asr-cap", type=int, default=ASR_CAP, help="tau_mem in tokens")
+    ap.add_argument("--asr-evict", type=int, default=ASR_EVICT, help="tokens evicted per cycle")
+    ap.add_argument("--asr-chunk", type=int, default=CHUNK, help="tokens per state chunk")
     ap.add_argument("--asr-rebuild-tiles", type=int, default=0,
                     help="key tiles per rebuild CTA (0: the library default, 16)")
     ap.add_argument("--asr-cadence-hz", type=float, default=2.0,
