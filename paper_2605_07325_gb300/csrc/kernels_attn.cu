@@ -617,9 +617,9 @@ __global__ void __launch_bounds__(kPairThreads, 1) attn_pair_kernel(const __grid
     }
     for (int w = 0; w < 2; ++w) {
       mbar_init(&bars->s_full[w], 1);
-      mbar_init(&bars->p_full[w], 128);
+      mbar_init(&bars->p_full[w], 4);   // one arrival per softmax warp
       mbar_init(&bars->o_final[w], 1);
-      mbar_init(&bars->o_free[w], 128);
+      mbar_init(&bars->o_free[w], 4);
     }
     mbar_init(&bars->drain, 1);
     bars->abort = 0;
@@ -888,7 +888,10 @@ __global__ void __launch_bounds__(kPairThreads, 1) attn_pair_kernel(const __grid
           rescale_o<HD>(tmem + lane_base + o_col, alpha);
         tmem_st_wait();
         tc_fence_before();
-        mbar_arrive(&bars->p_full[wg]);
+        // One arrival per warp once all its lanes have stored P: 128 arrivals
+        // on one barrier serialise in shared memory (measured 3.5% slower).
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&bars->p_full[wg]);
         ++s_it;
       }
       if (!ok) break;
@@ -929,7 +932,8 @@ __global__ void __launch_bounds__(kPairThreads, 1) attn_pair_kernel(const __grid
         p.part_lse[base] = lse2;
       }
       tc_fence_before();
-      mbar_arrive(&bars->o_free[wg]);
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&bars->o_free[wg]);
       ++seg_n;
     }
   }
