@@ -172,6 +172,46 @@ __device__ __forceinline__ void load_kv_tile(const AttnParams &p, const CUtensor
   }
 }
 
+// Predicated forms for a converged warp: only the lane with pred != 0 acts.
+__device__ __forceinline__ uint32_t elect_lane() {
+  uint32_t e;
+  asm volatile("{\n\t.reg .pred p;\n\telect.sync _|p, 0xffffffff;\n\tselp.u32 %0, 1, 0, p;\n\t}"
+               : "=r"(e));
+  return e;
+}
+__device__ __forceinline__ void mbar_arrive_expect_tx_if(uint32_t pred, uint64_t *bar, uint32_t bytes) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %2, 0;\n\t"
+      "@p mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;\n\t}" ::"r"(smem_u32(bar)),
+      "r"(bytes), "r"(pred)
+      : "memory");
+}
+__device__ __forceinline__ void tma_load_2d_if(uint32_t pred, void *dst, const CUtensorMap *map,
+                                               uint64_t *bar, int32_t x, int32_t y) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %5, 0;\n\t"
+      "@p cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3}], [%4];\n\t}" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_u32(bar)), "r"(pred)
+      : "memory");
+}
+template <int HD>
+__device__ __forceinline__ void load_kv_tile_if(uint32_t pred, const AttnParams &p,
+                                                const CUtensorMap *map, uint8_t *dst, uint64_t *bar,
+                                                int head, const int32_t *phys) {
+  const int P = p.page_size;
+  const int ppt = kBN / P;
+  const int seg = P < 64 ? P : 64;
+  for (int pp = 0; pp < ppt; ++pp) {
+    const int32_t row0 = (phys[pp] * p.hkv + head) * P;
+    for (int r = 0; r < P; r += seg) {
+#pragma unroll
+      for (int b = 0; b < HD / 64; ++b)
+        tma_load_2d_if(pred, dst + b * (kBN * 128) + (pp * P + r) * 128, map, bar, b * 64, row0 + r);
+    }
+  }
+}
+
 // Stage the physical ids of the logical pages covering key tiles [jb, je)
 // (tiles of bn keys) into `stage`, one id per page (whole producer warp).
 // Returns the first staged logical page.
@@ -644,29 +684,28 @@ __global__ void __launch_bounds__(kPairThreads, 1) attn_pair_kernel(const __grid
 
   if (warp == 8) {
     // ------------------------------------------------------ TMA producer
+    // The whole warp runs the loop (as the MMA issuer does); the elected lane's
+    // predicate gates the expect-tx arrivals and the TMA issues.
     int32_t *stage = reinterpret_cast<int32_t *>(smem + C::kPtOff);
     const int ppt = kBN / p.page_size;
     const int tiles_per_block = C::kPtStage / ppt;
+    const uint32_t leader = elect_lane();
     uint32_t q_round = 0, k_it = 0, v_it = 0;
     bool ok = true;
     while (ok && walk.next(p, T, seg)) {
-      if (lane == 0) {
-        if (q_round > 0 && !mbar_wait(&bars->q_empty, (q_round - 1) & 1, abort, p.err,
-                                      CSR_DEVERR_WAIT_TIMEOUT)) {
-          ok = false;
-        } else {
-          mbar_arrive_expect_tx(&bars->q_full, 2 * C::kQBytes);
-          const int32_t qrow = seg.head * p.rows_cap + seg.tile * 2 * kBM;
+      if (q_round > 0)
+        ok = __all_sync(0xffffffffu, mbar_wait(&bars->q_empty, (q_round - 1) & 1, abort, p.err,
+                                               CSR_DEVERR_WAIT_TIMEOUT));
+      if (!ok) break;
+      mbar_arrive_expect_tx_if(leader, &bars->q_full, 2 * C::kQBytes);
+      const int32_t qrow = seg.head * p.rows_cap + seg.tile * 2 * kBM;
 #pragma unroll
-          for (int h = 0; h < 2; ++h)
+      for (int h = 0; h < 2; ++h)
 #pragma unroll
-            for (int b = 0; b < C::kBoxes; ++b)
-              tma_load_2d(smem + C::kQOff + h * C::kQBytes + b * (kBM * 128), &p.tm_q,
-                          &bars->q_full, b * 64, qrow + h * kBM);
-          ++q_round;
-        }
-      }
-      ok = __shfl_sync(0xffffffffu, ok, 0);
+        for (int b = 0; b < C::kBoxes; ++b)
+          tma_load_2d_if(leader, smem + C::kQOff + h * C::kQBytes + b * (kBM * 128), &p.tm_q,
+                         &bars->q_full, b * 64, qrow + h * kBM);
+      ++q_round;
       for (int64_t jb = seg.j0; ok && jb < seg.j1; jb += tiles_per_block) {
         const int64_t je = min(jb + tiles_per_block, seg.j1);
         const int npages = static_cast<int>(je - jb) * ppt;
@@ -681,32 +720,25 @@ __global__ void __launch_bounds__(kPairThreads, 1) attn_pair_kernel(const __grid
           stage[i] = phys;
         }
         __syncwarp();
-        if (lane == 0) {
-          for (int64_t j = jb; j < je; ++j) {
-            const int32_t *phys = stage + static_cast<int>(j - jb) * ppt;
-            const int ks = k_it % C::kStages;
-            if (!mbar_wait(&bars->k_empty[ks], ((k_it / C::kStages) & 1) ^ 1, abort, p.err,
-                           CSR_DEVERR_WAIT_TIMEOUT)) {
-              ok = false;
-              break;
-            }
-            mbar_arrive_expect_tx(&bars->k_full[ks], C::kTileBytes);
-            load_kv_tile<HD>(p, &p.tm_k, smem + C::kKOff + ks * C::kTileBytes, &bars->k_full[ks],
-                             seg.head, phys);
-            ++k_it;
-            const int vs = v_it % C::kStages;
-            if (!mbar_wait(&bars->v_empty[vs], ((v_it / C::kStages) & 1) ^ 1, abort, p.err,
-                           CSR_DEVERR_WAIT_TIMEOUT)) {
-              ok = false;
-              break;
-            }
-            mbar_arrive_expect_tx(&bars->v_full[vs], C::kTileBytes);
-            load_kv_tile<HD>(p, &p.tm_v, smem + C::kVOff + vs * C::kTileBytes, &bars->v_full[vs],
-                             seg.head, phys);
-            ++v_it;
-          }
+        for (int64_t j = jb; j < je; ++j) {
+          const int32_t *phys = stage + static_cast<int>(j - jb) * ppt;
+          const int ks = k_it % C::kStages;
+          ok = __all_sync(0xffffffffu, mbar_wait(&bars->k_empty[ks], ((k_it / C::kStages) & 1) ^ 1,
+                                                 abort, p.err, CSR_DEVERR_WAIT_TIMEOUT));
+          if (!ok) break;
+          mbar_arrive_expect_tx_if(leader, &bars->k_full[ks], C::kTileBytes);
+          load_kv_tile_if<HD>(leader, p, &p.tm_k, smem + C::kKOff + ks * C::kTileBytes,
+                              &bars->k_full[ks], seg.head, phys);
+          ++k_it;
+          const int vs = v_it % C::kStages;
+          ok = __all_sync(0xffffffffu, mbar_wait(&bars->v_empty[vs], ((v_it / C::kStages) & 1) ^ 1,
+                                                 abort, p.err, CSR_DEVERR_WAIT_TIMEOUT));
+          if (!ok) break;
+          mbar_arrive_expect_tx_if(leader, &bars->v_full[vs], C::kTileBytes);
+          load_kv_tile_if<HD>(leader, p, &p.tm_v, smem + C::kVOff + vs * C::kTileBytes,
+                              &bars->v_full[vs], seg.head, phys);
+          ++v_it;
         }
-        ok = __shfl_sync(0xffffffffu, ok, 0);
       }
     }
     if (!ok && lane == 0) {
