@@ -6,7 +6,9 @@ bf16, RoPE base 1e6, page size 64.  The cache holds a 4,096-token static
 prefix plus 256-token chunks; the first timed step starts at 122,880 cached
 tokens.  A step appends a 256-token state chunk, attends a 512-token task
 suffix over the whole cache and truncates the suffix (section III-D), through
-the C-ABI library; the chunk is then invalidated again (csr_rewind, host-only)
+the C-ABI library: by default in one pass (csr_append_chunk_attend_suffix, then
+csr_truncate_suffix; --step separate issues csr_append_chunk and
+csr_attend_suffix instead); the chunk is then invalidated again (csr_rewind, host-only)
 so that every step sees exactly 122,880 cached tokens.  Inputs are seeded synthetic N(0,1) bf16 tensors already
 resident in HBM; the KV cache (about 252 MB) is larger than the 129 MB L2, so
 no flush is needed between steps.
@@ -65,16 +67,19 @@ def _attention_source_hash() -> str:
         return hashlib.sha256(f.read()).hexdigest()[:16]
 
 
-def _traffic_per_launch_step():
-    """DRAM bytes per step of the attention kernel from the committed ncu
-    summary, if it was taken on the current kernel source; else None."""
+def _traffic_per_launch(fused: bool):
+    """DRAM bytes per attention launch of the step from the committed ncu
+    summary (the fused step's single launch, or the mean of the separate
+    step's two), if it was taken on the current kernel source; else None."""
     try:
         with open(TRAFFIC_FILE) as f:
             kv = dict(line.strip().split("=", 1) for line in f
                       if "=" in line and not line.startswith("#"))
         if kv.get("kernel_source_sha256_16") != _attention_source_hash():
             return None
-        return float(kv["dram_bytes_per_step"])
+        if fused:
+            return float(kv["dram_bytes_per_launch_fused"])
+        return float(kv["dram_bytes_per_step"]) / 2
     except (OSError, KeyError, ValueError):
         return None
 
@@ -264,23 +269,29 @@ def run_ours(args):
         for _ in range(fill_chunks):
             ctx.append_chunk(fq, rnd(fill, HKV), rnd(fill, HKV), out=fout, stream=stream)
         sets = []
-        for _ in range(4):
-            sets.append(dict(cq=rnd(CHUNK, HQ), ck=rnd(CHUNK, HKV), cv=rnd(CHUNK, HKV),
-                             sq=rnd(SUFFIX, HQ), sk=rnd(SUFFIX, HKV), sv=rnd(SUFFIX, HKV),
-                             co=torch.empty((CHUNK, HQ, D), dtype=torch.bfloat16, device=dev),
-                             so=torch.empty((SUFFIX, HQ, D), dtype=torch.bfloat16, device=dev)))
+        for _ in range(4):   # the step's tokens: the chunk (first 256), then the suffix
+            sets.append(dict(q=rnd(CHUNK + SUFFIX, HQ), k=rnd(CHUNK + SUFFIX, HKV),
+                             v=rnd(CHUNK + SUFFIX, HKV),
+                             o=torch.empty((CHUNK + SUFFIX, HQ, D), dtype=torch.bfloat16, device=dev)))
     stream.synchronize()
     assert ctx.layout()[1] == L0, ctx.layout()[1]
+    fused = args.step == "fused"
 
-    def step(i):
+    def run_step(s):
         # one step of the robot loop: state chunk, task suffix, drop the suffix;
         # then invalidate the cache after L0 (host-only) so every step sees 122,880
         # cached tokens
-        s = sets[i % len(sets)]
-        ctx.append_chunk(s["cq"], s["ck"], s["cv"], out=s["co"], stream=stream)
-        ctx.attend_suffix(s["sq"], s["sk"], s["sv"], out=s["so"], stream=stream)
+        if fused:
+            ctx.append_chunk_attend_suffix(s["q"], s["k"], s["v"], CHUNK, out=s["o"], stream=stream)
+        else:
+            c, x = slice(0, CHUNK), slice(CHUNK, CHUNK + SUFFIX)
+            ctx.append_chunk(s["q"][c], s["k"][c], s["v"][c], out=s["o"][c], stream=stream)
+            ctx.attend_suffix(s["q"][x], s["k"][x], s["v"][x], out=s["o"][x], stream=stream)
         ctx.truncate_suffix()
         ctx.rewind(L0)
+
+    def step(i):
+        run_step(sets[i % len(sets)])
 
     for i in range(W):
         step(i)
@@ -316,24 +327,19 @@ def run_ours(args):
     # ------------------------------------------------ end to end, host buffers
     host = []
     for s in sets:
-        host.append({k: v.cpu().pin_memory() for k, v in s.items() if k[1] in "qkv"})
-        host[-1]["co"] = torch.empty((CHUNK, HQ, D), dtype=torch.bfloat16).pin_memory()
-        host[-1]["so"] = torch.empty((SUFFIX, HQ, D), dtype=torch.bfloat16).pin_memory()
+        host.append({k: s[k].cpu().pin_memory() for k in ("q", "k", "v")})
+        host[-1]["o"] = torch.empty((CHUNK + SUFFIX, HQ, D), dtype=torch.bfloat16).pin_memory()
     stage = {k: torch.empty_like(v) for k, v in sets[0].items()}
-    h2d = sum(v.numel() * 2 for k, v in sets[0].items() if k[1] in "qkv")
+    h2d = sum(sets[0][k].numel() * 2 for k in ("q", "k", "v"))
     d2h = (CHUNK + SUFFIX) * HQ * D * 2
 
     def step_e2e(i):
         h = host[i % len(host)]
         with torch.cuda.stream(stream):
-            for k in ("cq", "ck", "cv", "sq", "sk", "sv"):
+            for k in ("q", "k", "v"):
                 stage[k].copy_(h[k], non_blocking=True)
-            ctx.append_chunk(stage["cq"], stage["ck"], stage["cv"], out=stage["co"], stream=stream)
-            ctx.attend_suffix(stage["sq"], stage["sk"], stage["sv"], out=stage["so"], stream=stream)
-            ctx.truncate_suffix()
-            ctx.rewind(L0)
-            h["co"].copy_(stage["co"], non_blocking=True)
-            h["so"].copy_(stage["so"], non_blocking=True)
+            run_step(stage)
+            h["o"].copy_(stage["o"], non_blocking=True)
 
     for i in range(W):
         step_e2e(i)
@@ -361,7 +367,7 @@ def run_ours(args):
     flops = step_flops * K
     att_ms, att_n = ktimes["attention"]
     achieved = flops / (att_ms * 1e-3) / 1e12 if att_ms > 0 else None
-    traffic_step = _traffic_per_launch_step()
+    traffic = _traffic_per_launch(fused)
     step_floor = (costmodel.floor_seconds(costmodel.attention_flops(HQ, D, L0, CHUNK),
                                           costmodel.call_bytes(HQ, HKV, D, L0, CHUNK), peak_burst, hbm) +
                   costmodel.floor_seconds(costmodel.attention_flops(HQ, D, L0 + CHUNK, SUFFIX),
@@ -374,12 +380,14 @@ def run_ours(args):
         "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic: seeded N(0,1) bf16 Q/K/V (torch CUDA generator), resident in HBM",
         "config": {"workload": WORKLOAD_NAME, "cached_tokens": L0,
+                   "step_calls": ("csr_append_chunk_attend_suffix + csr_truncate_suffix" if fused else
+                                  "csr_append_chunk + csr_attend_suffix + csr_truncate_suffix"),
                    "step_flops": step_flops,
                    "l2": "inputs larger than L2: the 252 MB KV cache is streamed every step",
                    "replicas": world, "foreground_ctas": ctx.cfg.num_ctas or props.multi_processor_count},
         "roofline": {"bound": "tensor", "achieved": achieved, "peak": peak_burst, "unit": "TFLOP/s",
                      "frac": (achieved / peak_burst) if achieved else None,
-                     "traffic": (traffic_step / 2) if traffic_step else None,
+                     "traffic": traffic,
                      "kernel": {"pipe": "attn_pipe_kernel<128>", "pair": "attn_pair_kernel<128>",
                                 "single": "attn_kernel<128>"}[args.kernel] +
                                " (tcgen05 QK^T and PV, TMA paged K/V)",
@@ -706,6 +714,9 @@ def main(argv=None):
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--step", choices=["fused", "separate"], default="fused",
+                    help="how a step calls the library: separate (csr_append_chunk then "
+                         "csr_attend_suffix) or fused (csr_append_chunk_attend_suffix, one pass)")
     ap.add_argument("--kernel", choices=["pair", "pipe", "single"], default="pair",
                     help="attention kernel: pair (default: two query tiles per CTA, 128-key "
                          "tiles), pipe (two query tiles, 64-key tiles, two score buffers each), "

@@ -157,8 +157,29 @@ csr_status csr_attend_suffix(csr_ctx *ctx, const void *q, const void *k,
                              csr_stream_t stream);
 
 /*
+ * One task step in one pass: csr_append_chunk of the first n_chunk tokens
+ * followed by csr_attend_suffix of the next n_suffix, computed as a single
+ * causal block of n_chunk + n_suffix tokens (the chunk's tokens see the cache
+ * and the chunk, the suffix's see the cache, the chunk and the suffix: the
+ * same results as the two calls, with one RoPE/append launch, one pass of the
+ * attention over the cache and at most one merge).  q, k, v, out and lse hold
+ * the n_chunk + n_suffix tokens, chunk first.  The chunk joins X_static
+ * (*chunk_id as for csr_append_chunk) and the suffix stays live until
+ * csr_truncate_suffix.  When the chunk brings the static length to cap_tokens,
+ * the eviction of Algorithm 1 starts at that truncation (ordered after the
+ * work enqueued on `stream`).  CSR_EINVAL if either count is < 1 or their sum
+ * exceeds max_new_tokens; CSR_ESTATE as for csr_append_chunk.
+ */
+csr_status csr_append_chunk_attend_suffix(csr_ctx *ctx, const void *q, const void *k,
+                                          const void *v, int32_t n_chunk, int32_t n_suffix,
+                                          void *out, float *lse, csr_stream_t stream,
+                                          int64_t *chunk_id);
+
+/*
  * Drop the live suffix: the length returns to |X_static| and the pages that
- * hold only suffix slots go back to the pool.  Host-only (no kernel).
+ * hold only suffix slots go back to the pool.  Host-only (no kernel), unless a
+ * fused csr_append_chunk_attend_suffix reached cap_tokens: then the eviction
+ * starts here (as csr_evict_and_reconcile would) and its status is returned.
  * CSR_ESTATE when no suffix is live.
  */
 csr_status csr_truncate_suffix(csr_ctx *ctx);

@@ -77,6 +77,8 @@ _SIGS = {
     "csr_destroy": ([_vp], None),
     "csr_init_static": ([_vp, _vp, _vp, _vp, _i32, _vp, _vp, _vp], ctypes.c_int),
     "csr_append_chunk": ([_vp, _vp, _vp, _vp, _i32, _vp, _vp, _vp, _P64], ctypes.c_int),
+    "csr_append_chunk_attend_suffix": ([_vp, _vp, _vp, _vp, _i32, _i32, _vp, _vp, _vp, _P64],
+                                       ctypes.c_int),
     "csr_attend_suffix": ([_vp, _vp, _vp, _vp, _i32, _vp, _vp, _vp], ctypes.c_int),
     "csr_truncate_suffix": ([_vp], ctypes.c_int),
     "csr_rewind": ([_vp, _i64], ctypes.c_int),
@@ -207,6 +209,18 @@ class Context:
         self._check(_lib.csr_append_chunk(self._h, _ptr(q), _ptr(k), _ptr(v), n, _ptr(out),
                                           _ptr(lse), _stream_ptr_opt(self, stream),
                                           ctypes.byref(cid)))
+        return out, lse, cid.value
+
+    def append_chunk_attend_suffix(self, q, k, v, n_chunk, out=None, lse=None, stream=None,
+                                   n=None):
+        """One step: the first n_chunk tokens join the cache as a chunk, the rest
+        are a live suffix (truncate it with truncate_suffix)."""
+        q, out, lse = self._io(q, k, v, out, lse)
+        n = q.shape[0] if n is None else n
+        cid = ctypes.c_int64(-1)
+        self._check(_lib.csr_append_chunk_attend_suffix(
+            self._h, _ptr(q), _ptr(k), _ptr(v), int(n_chunk), int(n - n_chunk), _ptr(out),
+            _ptr(lse), _stream_ptr_opt(self, stream), ctypes.byref(cid)))
         return out, lse, cid.value
 
     def attend_suffix(self, q, k, v, out=None, lse=None, stream=None, n=None):

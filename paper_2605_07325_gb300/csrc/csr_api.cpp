@@ -238,6 +238,8 @@ struct csr_ctx {
   std::vector<Buffered> buffer;      // Delta X_buffer (N_catchup > 0): chunk and its position
   std::vector<int32_t> reserved_ids; // fresh ids the compaction kernel must produce
   bool ids_checked = false;
+  bool deferred_evict = false;        // a fused call reached tau_mem: evict at the truncation
+  csr_stream_t deferred_stream = nullptr;
   csr_qkv_provider provider = nullptr;
   void *user = nullptr;
   cudaStream_t lo = nullptr;
@@ -444,12 +446,17 @@ csr_status run_block(csr_ctx *c, int slot, int ws, const void *q, const void *k,
   return CSR_OK;
 }
 
-enum class Kind { Prefix, Chunk, Suffix };
+// ChunkSuffix: one block of n tokens whose first n_chunk are a chunk and the
+// rest a suffix (the fused step).
+enum class Kind { Prefix, Chunk, Suffix, ChunkSuffix };
 
 void push_chunk_task(csr_ctx *c, ChunkRec ch, int64_t pos, bool write_ids);
 
 csr_status add_block(csr_ctx *c, Kind kind, const void *q, const void *k, const void *v,
-                     int32_t n, void *out, float *lse, cudaStream_t s, int64_t *chunk_id) {
+                     int32_t n, void *out, float *lse, cudaStream_t s, int64_t *chunk_id,
+                     int32_t n_chunk = 0) {
+  const bool is_chunk = kind == Kind::Chunk || kind == Kind::ChunkSuffix;
+  const int32_t chunk_len = kind == Kind::ChunkSuffix ? n_chunk : n;
   if (n < 1 || n > c->cfg.max_new_tokens)
     return fail(c, CSR_EINVAL, "n must be in [1, max_new_tokens]");
   if (!c->plan_only && (!q || !k || !v || !out))
@@ -464,20 +471,34 @@ csr_status add_block(csr_ctx *c, Kind kind, const void *q, const void *k, const 
   const int64_t new_len = L + n;
   if (new_len > c->cfg.max_seq_tokens) return fail(c, CSR_ENOMEM, "max_seq_tokens exceeded");
   const int64_t needA = pages_for(c, new_len) - static_cast<int64_t>(A.pages.size());
-  const bool fork = kind == Kind::Chunk && c->reconciling;
+  const bool fork = is_chunk && c->reconciling;
   int64_t needB = 0;
   if (fork) {
     Version &B = c->pend();
-    if (B.length() + n > c->cfg.max_seq_tokens)
+    if (B.length() + chunk_len > c->cfg.max_seq_tokens)
       return fail(c, CSR_ENOMEM, "max_seq_tokens exceeded in the rebuilt version");
-    needB = pages_for(c, B.length() + n) - static_cast<int64_t>(B.pages.size());
+    needB = pages_for(c, B.length() + chunk_len) - static_cast<int64_t>(B.pages.size());
   }
   if (needA + needB > c->pool.n_free) return fail(c, CSR_ENOMEM, "page pool exhausted");
-  for (int64_t i = 0; i < needA; ++i) A.pages.push_back(c->pool.take());
+  // Reservation order (reading R4): the active version's pages for the chunk,
+  // then the rebuilt version's for the forked chunk, then the active version's
+  // for a fused suffix -- the order of csr_append_chunk + csr_attend_suffix.
+  const int64_t needA_chunk =
+      kind == Kind::ChunkSuffix
+          ? std::max<int64_t>(0, pages_for(c, L + chunk_len) - static_cast<int64_t>(A.pages.size()))
+          : needA;
+  for (int64_t i = 0; i < needA_chunk; ++i) A.pages.push_back(c->pool.take());
+  int64_t fork_pos = 0;
+  if (fork) {
+    Version &B = c->pend();
+    fork_pos = B.length();
+    for (int64_t i = 0; i < needB; ++i) B.pages.push_back(c->pool.take());
+  }
+  for (int64_t i = needA_chunk; i < needA; ++i) A.pages.push_back(c->pool.take());
   const int32_t first_lp = static_cast<int32_t>(L / c->cfg.page_size);
   const int32_t n_ids = static_cast<int32_t>(pages_for(c, new_len)) - first_lp;
   int64_t id = -1;
-  if (kind == Kind::Chunk) id = c->next_chunk_id++;
+  if (is_chunk) id = c->next_chunk_id++;
   if (!c->plan_only) {
     const int slot = c->active.load();
     csr_status st = run_block(c, slot, 0, q, k, v, n, L, A.pages.data() + first_lp, n_ids,
@@ -488,17 +509,20 @@ csr_status add_block(csr_ctx *c, Kind kind, const void *q, const void *k, const 
     case Kind::Prefix: A.prefix_len = n; break;
     case Kind::Chunk: A.chunks.push_back({id, n}); break;
     case Kind::Suffix: A.suffix_len = n; break;
+    case Kind::ChunkSuffix:
+      A.chunks.push_back({id, n_chunk});
+      A.suffix_len = n - n_chunk;
+      break;
   }
   if (chunk_id) *chunk_id = id;
   if (fork) {
-    // Algorithm 1, Increment: fork the chunk into the rebuild; its pages in
-    // the rebuilt version are reserved now (after the active ones).
+    // Algorithm 1, Increment: fork the chunk into the rebuild (its pages in
+    // the rebuilt version were reserved above).
     Version &B = c->pend();
-    const int64_t pos = B.length();
-    for (int64_t i = 0; i < needB; ++i) B.pages.push_back(c->pool.take());
-    B.chunks.push_back({id, n});
+    const int64_t pos = fork_pos;
+    B.chunks.push_back({id, chunk_len});
     if (c->cfg.n_catchup > 0) {
-      c->buffer.push_back({{id, n}, pos});
+      c->buffer.push_back({{id, chunk_len}, pos});
     } else if (!c->plan_only) {
       // N_catchup = 0: Algorithm 1's loop drains the whole buffer before the
       // swap, so each chunk that arrives while reconciling goes to R_2 at
@@ -508,7 +532,7 @@ csr_status add_block(csr_ctx *c, Kind kind, const void *q, const void *k, const 
       cudaError_t e = cudaEventRecord(c->ev_fg, s);
       if (e == cudaSuccess) e = cudaStreamWaitEvent(c->lo, c->ev_fg, 0);
       if (e != cudaSuccess) return cuda_fail(c, e, "ordering the catch-up after the foreground");
-      push_chunk_task(c, {id, n}, pos, true);
+      push_chunk_task(c, {id, chunk_len}, pos, true);
     }
   }
   return CSR_OK;
@@ -772,6 +796,28 @@ csr_status csr_append_chunk(csr_ctx *c, const void *q, const void *k, const void
   return CSR_OK;
 }
 
+csr_status csr_append_chunk_attend_suffix(csr_ctx *c, const void *q, const void *k, const void *v,
+                                          int32_t n_chunk, int32_t n_suffix, void *out, float *lse,
+                                          csr_stream_t stream, int64_t *chunk_id) {
+  if (!c) return CSR_EINVAL;
+  if (!c->has_static) return fail(c, CSR_ESTATE, "csr_init_static must come first");
+  if (c->act().suffix_len > 0) return fail(c, CSR_ESTATE, "a suffix is live: truncate it first");
+  if (n_chunk < 1 || n_suffix < 1) return fail(c, CSR_EINVAL, "n_chunk and n_suffix must be >= 1");
+  if (static_cast<int64_t>(n_chunk) + n_suffix > c->cfg.max_new_tokens)
+    return fail(c, CSR_EINVAL, "n_chunk + n_suffix must be <= max_new_tokens");
+  csr_status st = add_block(c, Kind::ChunkSuffix, q, k, v, n_chunk + n_suffix, out, lse,
+                            reinterpret_cast<cudaStream_t>(stream), chunk_id, n_chunk);
+  if (st != CSR_OK) return st;
+  // Algorithm 1, Increment: tau_mem reached; the eviction waits for the
+  // truncation that ends this task (it needs no live suffix).
+  if (c->provider && c->cfg.cap_tokens > 0 && !c->reconciling &&
+      c->act().length() - c->act().suffix_len >= c->cfg.cap_tokens) {
+    c->deferred_evict = true;
+    c->deferred_stream = stream;
+  }
+  return CSR_OK;
+}
+
 csr_status csr_attend_suffix(csr_ctx *c, const void *q, const void *k, const void *v, int32_t n,
                              void *out, float *lse, csr_stream_t stream) {
   if (!c) return CSR_EINVAL;
@@ -790,6 +836,11 @@ csr_status csr_truncate_suffix(csr_ctx *c) {
   while (static_cast<int64_t>(A.pages.size()) > keep) {
     c->pool.release(A.pages.back());
     A.pages.pop_back();
+  }
+  if (c->deferred_evict) {  // tau_mem was reached by a fused chunk + suffix call
+    c->deferred_evict = false;
+    if (c->provider && !c->reconciling)
+      return csr_evict_and_reconcile(c, c->cfg.evict_tokens, c->deferred_stream);
   }
   return CSR_OK;
 }

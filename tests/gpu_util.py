@@ -124,6 +124,29 @@ class Pair:
         self._check(f"chunk {cid}", out, lse, exp, compare)
         return out, lse, cid
 
+    def fused(self, b: synth.Block, n_chunk: int, compare=True):
+        """csr_append_chunk_attend_suffix of b (chunk = its first n_chunk
+        tokens) against the oracle's append_chunk + attend_suffix."""
+        q, k, v = self._dev(b)
+        lse = self._lse(b.n)
+        chunk = synth.Block(b.q[:n_chunk], b.k[:n_chunk], b.v[:n_chunk])
+        suffix = synth.Block(b.q[n_chunk:], b.k[n_chunk:], b.v[n_chunk:])
+        self.orc.attend = compare
+        exp_c = self.orc.append_chunk(*chunk.f64())
+        self.orc.attend = True
+        exp_s = self.orc.attend_suffix(*suffix.f64()) if compare else (None, None)
+        if not compare:
+            self.orc.attend = False
+            self.orc.attend_suffix(*suffix.f64())
+            self.orc.attend = True
+        self.blocks[exp_c[2]] = chunk     # before the call: it may start a rebuild
+        out, _, cid = self.ctx.append_chunk_attend_suffix(q, k, v, n_chunk, lse=lse)
+        assert cid == exp_c[2]
+        torch.cuda.synchronize()
+        self._check(f"fused chunk {cid}", out[:n_chunk], lse[:, :n_chunk], exp_c, compare)
+        self._check("fused suffix", out[n_chunk:], lse[:, n_chunk:], exp_s, compare)
+        return out, lse, cid
+
     def suffix(self, b: synth.Block, compare=True):
         q, k, v = self._dev(b)
         lse = self._lse(b.n)

@@ -176,3 +176,21 @@ def test_other_kernel_designs_match_oracle(libcsr, shape, chunk_tiles, kernel):
     p.suffix(p.blk(20, 70))
     p.truncate()
     p.device_clean()
+
+
+@pytest.mark.parametrize("shape", [C1, C2], ids=["d64_p16_g4", "d128_p64_g16"])
+@pytest.mark.parametrize("chunk_tiles", [0, 2])
+def test_fused_step_matches_oracle(libcsr, shape, chunk_tiles):
+    """csr_append_chunk_attend_suffix: the chunk's outputs equal those of
+    append_chunk and the suffix's those of attend_suffix on the same cache;
+    the layout after the truncation equals the two-call layout."""
+    p = Pair(shape, pool_pages=160, max_seq=4096, max_new=1024, fg_chunk_tiles=chunk_tiles)
+    p.init_static(p.blk(40, 77))
+    for i, (nc, ns) in enumerate([(1, 1), (37, 100), (129, 300), (256, 512)]):
+        p.fused(p.blk(41 + i, nc + ns), nc)
+        p.check_layout()
+        p.truncate()
+        p.check_layout()
+    p.append(p.blk(60, 50))
+    p.check_cache()
+    p.device_clean()

@@ -112,6 +112,38 @@ def test_automatic_eviction_and_repeated_cycles(libcsr):
     p.device_clean()
 
 
+def test_fused_steps_through_eviction_cycles(libcsr):
+    """Fused chunk + suffix steps: tau_mem reached by a fused step starts the
+    eviction at its truncation; fused steps during the reconciliation fork
+    only their chunk; two cycles against the oracle."""
+    csr = csr_mod()
+    p = Pair(C1, pool_pages=256, max_seq=4096, max_new=256, cap_tokens=400, evict_tokens=128)
+    lo = torch.cuda.Stream(priority=0)
+    outs = {}
+    p.ctx.set_reconciler(_provider(p, outs), lo)
+    p.init_static(p.blk(950, 70))
+    seed, cycles, steps = 951, 0, 0
+    while cycles < 2:
+        assert steps < 100
+        if p.orc.is_reconciling and p.ctx.poll_swap() == csr.RECON_SWAPPED:
+            expect = p.orc.reconcile()
+            torch.cuda.synchronize()
+            for cid, (eo, _) in expect.items():
+                assert_close(to_f64(outs[cid]), eo, f"cycle {cycles} chunk {cid}")
+            p.check_layout()
+            p.check_cache()
+            cycles += 1
+        p.fused(p.blk(seed, 45), 30)
+        trigger = not p.orc.is_reconciling and p.orc.length() - 15 >= 400
+        p.truncate()
+        if trigger:
+            p.orc.evict(128)            # the library started it at the truncation
+            assert p.ctx.layout(csr.VERSION_PENDING)[0] == p.orc.page_table("pending")
+        seed += 1
+        steps += 1
+    p.device_clean()
+
+
 def test_provider_failure_keeps_old_version(libcsr):
     csr = csr_mod()
     p = Pair(C1, pool_pages=128, max_seq=4096, max_new=256)

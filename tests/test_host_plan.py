@@ -206,3 +206,73 @@ def test_rewind_matches_oracle(libcsr):
     _same(ctx, m, libcsr)
     ctx.attend_suffix(None, None, None, n=3)
     _err(libcsr, lambda: ctx.rewind(40), libcsr.ESTATE)
+
+
+def test_fused_step_layout_matches_separate_calls(libcsr):
+    """csr_append_chunk_attend_suffix = csr_append_chunk + csr_attend_suffix:
+    the same page tables, free lists and chunk ids, against the oracle."""
+    fused, sep, m = _plan(libcsr, pool=128), _plan(libcsr, pool=128), _Model(128)
+    for c in (fused, sep):
+        c.init_static(None, None, None, n=37)
+    m.o.init_static(*m.blk(37))
+    for n_chunk, n_suffix in [(5, 40), (16, 16), (27, 1), (100, 29), (1, 63), (64, 64)]:
+        _, _, cid = fused.append_chunk_attend_suffix(None, None, None, n_chunk, n=n_chunk + n_suffix)
+        _, _, cid2 = sep.append_chunk(None, None, None, n=n_chunk)
+        sep.attend_suffix(None, None, None, n=n_suffix)
+        _, _, cid3 = m.o.append_chunk(*m.blk(n_chunk))
+        m.o.attend_suffix(*m.blk(n_suffix))
+        assert cid == cid2 == cid3
+        _same(fused, m, libcsr)
+        assert fused.layout() == sep.layout() and fused.free_pages() == sep.free_pages()
+        for c in (fused, sep):
+            c.truncate_suffix()
+        m.o.truncate_suffix()
+        _same(fused, m, libcsr)
+    assert fused.chunks() == sep.chunks()
+
+
+def test_fused_step_eviction_starts_at_truncate(libcsr):
+    """tau_mem reached by a fused step: the eviction waits for the truncation
+    (it needs no live suffix), then matches the oracle; a fused step during the
+    reconciliation forks only its chunk into the rebuilt version."""
+    ctx = _plan(libcsr, pool=128, cap_tokens=100, evict_tokens=40)
+    m = _Model(128)
+    ctx.set_reconciler(lambda cid, n: None)
+    ctx.init_static(None, None, None, n=20)
+    m.o.init_static(*m.blk(20))
+    for i in range(4):
+        ctx.append_chunk_attend_suffix(None, None, None, 20, n=33)
+        m.o.append_chunk(*m.blk(20))
+        m.o.attend_suffix(*m.blk(13))
+        if i == 3:                                  # 100 = tau_mem, suffix still live
+            assert ctx.poll_swap() == libcsr.RECON_IDLE
+        ctx.truncate_suffix()
+        m.o.truncate_suffix()
+    m.o.evict(40)
+    _same(ctx, m, libcsr, "pending")
+    ctx.append_chunk_attend_suffix(None, None, None, 12, n=30)   # forked: 12 tokens
+    m.o.append_chunk(*m.blk(12))
+    m.o.attend_suffix(*m.blk(18))
+    _same(ctx, m, libcsr, "pending")
+    assert ctx.poll_swap() == libcsr.RECON_RUNNING  # swap waits for the live suffix
+    ctx.truncate_suffix()
+    m.o.truncate_suffix()
+    assert ctx.wait_reconcile(5.0) == libcsr.RECON_SWAPPED
+    m.o.reconcile()
+    _same(ctx, m, libcsr)
+
+
+def test_fused_step_errors(libcsr):
+    ctx = _plan(libcsr, pool=64, max_new=64)
+    _err(libcsr, lambda: ctx.append_chunk_attend_suffix(None, None, None, 4, n=8), libcsr.ESTATE)
+    ctx.init_static(None, None, None, n=16)
+    before = (ctx.layout(), ctx.free_pages())
+    _err(libcsr, lambda: ctx.append_chunk_attend_suffix(None, None, None, 0, n=8), libcsr.EINVAL)
+    _err(libcsr, lambda: ctx.append_chunk_attend_suffix(None, None, None, 8, n=8), libcsr.EINVAL)
+    _err(libcsr, lambda: ctx.append_chunk_attend_suffix(None, None, None, 40, n=65), libcsr.EINVAL)
+    assert (ctx.layout(), ctx.free_pages()) == before
+    ctx.append_chunk_attend_suffix(None, None, None, 4, n=8)
+    _err(libcsr, lambda: ctx.append_chunk_attend_suffix(None, None, None, 4, n=8), libcsr.ESTATE)
+    _err(libcsr, lambda: ctx.append_chunk(None, None, None, n=4), libcsr.ESTATE)
+    ctx.truncate_suffix()
+    assert ctx.layout()[1] == 20
