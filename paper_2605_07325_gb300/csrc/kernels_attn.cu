@@ -1387,6 +1387,21 @@ __global__ void __launch_bounds__(320, 1) attn_pipe_kernel(const __grid_constant
 // Merge the key-chunk pieces of one row: lse = log2 sum_k 2^lse_k and
 // O = sum_k 2^(lse_k - lse) O_k (each O_k already normalised by its own sum).
 // One warp per packed row; lanes own head_dim/32 output columns.
+// kPer consecutive floats of a partial row (16-byte loads for kPer = 4).
+template <int kPer>
+__device__ __forceinline__ void load_row_part(const float *src, float (&v)[kPer]) {
+  if constexpr (kPer == 4) {
+    const float4 x = *reinterpret_cast<const float4 *>(src);
+    v[0] = x.x; v[1] = x.y; v[2] = x.z; v[3] = x.w;
+  } else {
+#pragma unroll
+    for (int e = 0; e < kPer; e += 2) {
+      const float2 x = *reinterpret_cast<const float2 *>(src + e);
+      v[e] = x.x; v[e + 1] = x.y;
+    }
+  }
+}
+
 template <int HD>
 __global__ void __launch_bounds__(256) merge_kernel(const __grid_constant__ MergeParams p) {
   const int head = blockIdx.x / p.n_tiles;
@@ -1425,17 +1440,31 @@ __global__ void __launch_bounds__(256) merge_kernel(const __grid_constant__ Merg
 #pragma unroll
     for (int off = 16; off > 0; off >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, off);
     lse2 = mx + log2f(sum);
-    for (int k = 0; k < nk; ++k) {
+    // Four chunks' rows in flight per lane before any is consumed: the merge
+    // is bound by HBM latency, not by arithmetic.
+    constexpr int kU = 4;
+    int k = 0;
+    for (; k + kU <= nk; k += kU) {
+      float lw[kU];
+      float v[kU][kPer];
+#pragma unroll
+      for (int u = 0; u < kU; ++u) {
+        const int64_t base = prow(k + u);
+        lw[u] = p.part_lse[base];
+        load_row_part<kPer>(p.part_o + base * HD + lane * kPer, v[u]);
+      }
+#pragma unroll
+      for (int u = 0; u < kU; ++u) {
+        const float w = ex2_approx(lw[u] - lse2);
+#pragma unroll
+        for (int e = 0; e < kPer; ++e) acc[e] = fmaf(w, v[u][e], acc[e]);
+      }
+    }
+    for (; k < nk; ++k) {
       const int64_t base = prow(k);
       const float w = ex2_approx(p.part_lse[base] - lse2);
-      const float *src = p.part_o + base * HD + lane * kPer;
       float v[kPer];
-#pragma unroll
-      for (int e = 0; e < kPer; e += 2) {
-        const float2 x = *reinterpret_cast<const float2 *>(src + e);
-        v[e] = x.x;
-        v[e + 1] = x.y;
-      }
+      load_row_part<kPer>(p.part_o + base * HD + lane * kPer, v);
 #pragma unroll
       for (int e = 0; e < kPer; ++e) acc[e] = fmaf(w, v[e], acc[e]);
     }
