@@ -650,7 +650,7 @@ def run_sweep(args):
     dev = torch.device("cuda", 0)
     torch.cuda.set_device(dev)
     hbm, peak, _, kind = _peaks()
-    max_L = max(SWEEP_L)
+    max_L = max(args.sweep_l or SWEEP_L)
     cfg = csr.make_config(HQ, HKV, D, P, BASE, max_new_tokens=4096,
                           pool_pages=(max_L + 4096) // P + 16, max_seq_tokens=max_L + 4096 + P)
     stream = torch.cuda.Stream(device=dev, priority=-1)
@@ -668,7 +668,7 @@ def run_sweep(args):
         fill_o = torch.empty((4096, HQ, D), dtype=torch.bfloat16, device=dev)
         blocks = {n: (rnd(n, HQ), rnd(n, HKV), rnd(n, HKV),
                       torch.empty((n, HQ, D), dtype=torch.bfloat16, device=dev)) for n in SWEEP_N}
-        for L in SWEEP_L:
+        for L in (args.sweep_l or SWEEP_L):
             while ctx.layout()[1] < L:
                 ctx.append_chunk(fill_q, rnd(4096, HKV), rnd(4096, HKV), out=fill_o, stream=stream)
             assert ctx.layout()[1] == L
@@ -694,6 +694,7 @@ def run_sweep(args):
                 floor = costmodel.floor_seconds(f, b, peak, hbm) * 1e6
                 att_us = t["attention"][0] / max(1, t["attention"][1]) * 1e3
                 pt = {"L": L, "n": n, "us_per_call": us, "attention_us": att_us,
+                      "rope_append_us": t["rope_append"][0] / K * 1e3, "merge_us": t["merge"][0] / K * 1e3,
                       "tflops": f / (us * 1e-6) / 1e12, "gbs": b / (us * 1e-6) / 1e9,
                       "floor_us": floor, "bound": "tensor" if f / (peak * 1e12) > b / (hbm * 1e9) else "hbm",
                       "roofline_frac": floor / us}
@@ -736,6 +737,8 @@ def main(argv=None):
                     help="foreground step rate; 0 runs steps back to back")
     ap.add_argument("--sweep", action="store_true",
                     help="run the L x n sweep instead of the 120K step line")
+    ap.add_argument("--sweep-l", type=int, nargs="*", default=None,
+                    help="cached lengths of the sweep (default: 16K 32K 64K 96K 128K)")
     ap.add_argument("--unordered", action="store_true",
                     help="time the unordered baseline (full recompute per step) beside CSR")
     args = ap.parse_args(argv)

@@ -1403,7 +1403,7 @@ __device__ __forceinline__ void load_row_part(const float *src, float (&v)[kPer]
 }
 
 template <int HD>
-__global__ void __launch_bounds__(256) merge_kernel(const __grid_constant__ MergeParams p) {
+__global__ void __launch_bounds__(256, 4) merge_kernel(const __grid_constant__ MergeParams p) {
   const int head = blockIdx.x / p.n_tiles;
   const int tile = blockIdx.x - head * p.n_tiles;
   const int T = kBM / p.group;
@@ -1425,48 +1425,72 @@ __global__ void __launch_bounds__(256) merge_kernel(const __grid_constant__ Merg
     return (static_cast<int64_t>(k) * units + static_cast<int64_t>(head) * uph + unit) * rows_per_item +
            row_in_item;
   };
-  float mx = -CUDART_INF_F;
-  for (int k = lane; k < nk; k += 32) mx = fmaxf(mx, p.part_lse[prow(k)]);
-#pragma unroll
-  for (int off = 16; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
   constexpr int kPer = HD / 32;  // floats per lane
   float acc[kPer];
 #pragma unroll
   for (int e = 0; e < kPer; ++e) acc[e] = 0.f;
   float lse2 = -CUDART_INF_F;
-  if (mx != -CUDART_INF_F) {
-    float sum = 0.f;
-    for (int k = lane; k < nk; k += 32) sum += ex2_approx(p.part_lse[prow(k)] - mx);
+  if (nk <= 64) {
+    // Every chunk's LSE sits in a register of lane k % 32 (loaded once), so
+    // the maximum, the sum and each chunk's weight (broadcast by shuffle)
+    // need no second pass over memory; the rows are then read four chunks
+    // at a time (more in flight costs registers, hence occupancy).
+    const float l0 = lane < nk ? p.part_lse[prow(lane)] : -CUDART_INF_F;
+    const float l1 = lane + 32 < nk ? p.part_lse[prow(lane + 32)] : -CUDART_INF_F;
+    float mx = fmaxf(l0, l1);
 #pragma unroll
-    for (int off = 16; off > 0; off >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, off);
-    lse2 = mx + log2f(sum);
-    // Four chunks' rows in flight per lane before any is consumed: the merge
-    // is bound by HBM latency, not by arithmetic.
-    constexpr int kU = 4;
-    int k = 0;
-    for (; k + kU <= nk; k += kU) {
-      float lw[kU];
-      float v[kU][kPer];
+    for (int off = 16; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
+    if (mx != -CUDART_INF_F) {
+      const float e0 = lane < nk ? ex2_approx(l0 - mx) : 0.f;
+      const float e1 = lane + 32 < nk ? ex2_approx(l1 - mx) : 0.f;
+      float sum = e0 + e1;
 #pragma unroll
-      for (int u = 0; u < kU; ++u) {
-        const int64_t base = prow(k + u);
-        lw[u] = p.part_lse[base];
-        load_row_part<kPer>(p.part_o + base * HD + lane * kPer, v[u]);
-      }
+      for (int off = 16; off > 0; off >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, off);
+      lse2 = mx + log2f(sum);
+      const float inv = 1.0f / sum;
+      const float w0 = e0 * inv, w1 = e1 * inv;
+      constexpr int kU = 4;
+      for (int k0 = 0; k0 < nk; k0 += kU) {
+        float v[kU][kPer];
 #pragma unroll
-      for (int u = 0; u < kU; ++u) {
-        const float w = ex2_approx(lw[u] - lse2);
+        for (int u = 0; u < kU; ++u) {
+          if (k0 + u < nk) {
+            load_row_part<kPer>(p.part_o + prow(k0 + u) * HD + lane * kPer, v[u]);
+          } else {
 #pragma unroll
-        for (int e = 0; e < kPer; ++e) acc[e] = fmaf(w, v[u][e], acc[e]);
+            for (int e = 0; e < kPer; ++e) v[u][e] = 0.f;
+          }
+        }
+#pragma unroll
+        for (int u = 0; u < kU; ++u) {
+          const int k = k0 + u;
+          const float w = __shfl_sync(0xffffffffu, k < 32 ? w0 : w1, k & 31);
+          if (k < nk) {
+#pragma unroll
+            for (int e = 0; e < kPer; ++e) acc[e] = fmaf(w, v[u][e], acc[e]);
+          }
+        }
       }
     }
-    for (; k < nk; ++k) {
-      const int64_t base = prow(k);
-      const float w = ex2_approx(p.part_lse[base] - lse2);
-      float v[kPer];
-      load_row_part<kPer>(p.part_o + base * HD + lane * kPer, v);
+  } else {
+    float mx = -CUDART_INF_F;
+    for (int k = lane; k < nk; k += 32) mx = fmaxf(mx, p.part_lse[prow(k)]);
 #pragma unroll
-      for (int e = 0; e < kPer; ++e) acc[e] = fmaf(w, v[e], acc[e]);
+    for (int off = 16; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
+    if (mx != -CUDART_INF_F) {
+      float sum = 0.f;
+      for (int k = lane; k < nk; k += 32) sum += ex2_approx(p.part_lse[prow(k)] - mx);
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, off);
+      lse2 = mx + log2f(sum);
+      for (int k = 0; k < nk; ++k) {
+        const int64_t base = prow(k);
+        const float w = ex2_approx(p.part_lse[base] - lse2);
+        float v[kPer];
+        load_row_part<kPer>(p.part_o + base * HD + lane * kPer, v);
+#pragma unroll
+        for (int e = 0; e < kPer; ++e) acc[e] = fmaf(w, v[e], acc[e]);
+      }
     }
   }
   const int hq_idx = head * p.group + r % p.group;
