@@ -39,10 +39,12 @@ __device__ __forceinline__ void rotate8(const uint4 &a, const uint4 &b, const fl
   yb = make_uint4(rb[0], rb[1], rb[2], rb[3]);
 }
 
-// One block per new token.  Angles: theta_i = pos * base^(-2i/d); the turn
-// count pos * base^(-2i/d) / (2 pi) is formed in fp64 and reduced to
-// [-1/2, 1/2] before the fp32 sincospi, so positions past 10^5 keep full
-// fp32 angle accuracy.
+// Block (token t, part y): the token's 16-byte work items (rotated query
+// pairs, rotated key pairs, value vectors) y, y + gridDim.y, ... in units of
+// 256.  Angles: theta_i =
+// pos * base^(-2i/d); the turn count pos * base^(-2i/d) / (2 pi) is formed in
+// fp64 and reduced to [-1/2, 1/2] before the fp32 sincospi, so positions past
+// 10^5 keep full fp32 angle accuracy.
 __global__ void __launch_bounds__(256) rope_append_kernel(const __grid_constant__ RopeAppendParams p) {
   __shared__ float cs[kMaxHalfDim], sn[kMaxHalfDim];
   const int t = blockIdx.x;
@@ -56,7 +58,7 @@ __global__ void __launch_bounds__(256) rope_append_kernel(const __grid_constant_
     cs[i] = c;
     sn[i] = s;
   }
-  if (blockIdx.x == 0 && p.n_ids > 0) {
+  if (blockIdx.x == 0 && blockIdx.y == 0 && p.n_ids > 0) {
     for (int i = threadIdx.x; i < p.n_ids; i += blockDim.x) p.page_table[p.first_lp + i] = p.ids[i];
   }
   __syncthreads();
@@ -70,7 +72,7 @@ __global__ void __launch_bounds__(256) rope_append_kernel(const __grid_constant_
   const int c16 = p.d / 16;  // 8-pair chunks per head
   const int c8 = p.d / 8;    // 16-byte vectors per head
   const int nq = p.hq * c16, nk = p.hkv * c16, nv = p.hkv * c8;
-  for (int w = threadIdx.x; w < nq + nk + nv; w += blockDim.x) {
+  for (int w = blockIdx.y * blockDim.x + threadIdx.x; w < nq + nk + nv; w += gridDim.y * blockDim.x) {
     if (w < nq + nk) {
       const bool is_q = w < nq;
       const int ww = is_q ? w : w - nq;
@@ -103,7 +105,12 @@ __global__ void __launch_bounds__(256) rope_append_kernel(const __grid_constant_
 }
 
 cudaError_t launch_rope_append(const RopeAppendParams &p, cudaStream_t s) {
-  rope_append_kernel<<<p.n, 256, 0, s>>>(p);
+  // Short blocks split each token over several CTAs (one work item per
+  // thread: latency-bound otherwise); long blocks already fill the GPU with
+  // one CTA per token and would only recompute the angle table.
+  const int items = (p.hq + p.hkv) * (p.d / 16) + p.hkv * (p.d / 8);
+  const dim3 grid(p.n, p.n < 128 ? (items + 255) / 256 : 1);
+  rope_append_kernel<<<grid, 256, 0, s>>>(p);
   return cudaGetLastError();
 }
 
