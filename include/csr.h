@@ -271,6 +271,33 @@ csr_status csr_poll_swap(csr_ctx *ctx, csr_stream_t fg_stream, int *state);
 csr_status csr_wait_reconcile(csr_ctx *ctx, csr_stream_t fg_stream,
                               int64_t timeout_us, int *state);
 
+/*
+ * Sequence versions of Algorithm 2: *k is the active version (0 at creation,
+ * +1 at every swap); *k_ready is k + 1 once the running reconciliation's
+ * rebuild and catch-up are complete up to at most n_catchup buffered chunks
+ * (as of the last csr_poll_swap / csr_route), else k.  Host-only.
+ */
+csr_status csr_get_versions(csr_ctx *ctx, int64_t *k, int64_t *k_ready);
+
+/* Values of *route from csr_route. */
+#define CSR_ROUTE_CONTINUE 0  /* k_t = k: serve on the active version (case 1) */
+#define CSR_ROUTE_BRIDGE 1    /* k_t = k + 1 before k_ready: serve on the active version;
+                                 chunks appended now are forked into the rebuild (case 2) */
+#define CSR_ROUTE_SWAPPED 2   /* k_t = k + 1 = k_ready: this call swapped the versions;
+                                 serve on the new active version (case 2) */
+#define CSR_ROUTE_STRAGGLER 3 /* k_t < k: served on the active version; the paper's
+                                 secondary copy of the old sequence is not retained (case 3) */
+
+/*
+ * Per-query routing of Algorithm 2 (concurrent request routing): classify a
+ * query built on sequence version k_t against the context's versions, and
+ * perform the resource swap when the query is the first of the rebuilt
+ * version and the rebuild is ready (as csr_poll_swap would; never while a
+ * suffix is live).  Progresses the reconciliation like csr_poll_swap.
+ * CSR_EINVAL if k_t > k + 1, or k_t = k + 1 without a running reconciliation.
+ */
+csr_status csr_route(csr_ctx *ctx, int64_t k_t, csr_stream_t fg_stream, int *route);
+
 /* Which version an inspection call reads. */
 #define CSR_VERSION_ACTIVE 0
 #define CSR_VERSION_PENDING 1

@@ -11,6 +11,8 @@ Contents
   causal softmax attention, Eq. causal_attention_1..3 of section III-A).
 * ``PageAllocatorModel``: a set of free physical page ids; every page request
   takes the smallest free id.  Independent of the library's allocator.
+* ``Alg2Router``: the per-query routing state machine of Algorithm 2
+  (sequence versions k, k_ready; continuation, bridging, swap, stragglers).
 * ``OracleCSR``: the CSR cache lifecycle as a list of cached segments
   (section III-D: X_static = (X_pre, X_chunks), X_dyn = (X_suff, X_task)) with
   the operations of Algorithm 1: Increment (append a chunk, buffer it while a
@@ -397,3 +399,68 @@ class OracleCSR:
     def slot_of(self, position: int, which: str = "active") -> int:
         ver = self.active if which == "active" else self.pending
         return ver.pages[position // self.P] * self.P + position % self.P
+
+
+# --------------------------------------------------------------------------
+# Algorithm 2: asynchronous state reconciliation with concurrent request routing
+# --------------------------------------------------------------------------
+class Alg2Router:
+    """The routing procedure of Algorithm 2, step by step in the paper's order
+    and notation, over sequence metadata only (the states are represented by
+    their static lengths j, and the caches by the resource names R1, R2).
+
+    ``inference(j_t, k_t, j_eps_t)`` classifies one query and returns
+    (case, resource): "continue" (case 1, k_t = k), "bridge" (case 2,
+    k_t > k_ready), "swap" (case 2, k_t = k_ready), "straggler_primary"
+    (case 3 while reconciling) or "straggler_secondary" (case 3 otherwise).
+    ``reconcile_start`` / ``reconcile_done`` are the first and last steps of
+    procedure Reconcile (lock R2 from stragglers, empty the buffer; authorise
+    the swap with k_ready <- k_target)."""
+
+    def __init__(self):
+        self.j = 0                 # current active sequence static length
+        self.k = 0                 # current active sequence version
+        self.k_ready = 0           # highest version fully precomputed on the secondary
+        self.j_eps = None          # evicted sequence static length (the eviction cursor)
+        self.x_recon = None        # reconciliation state: (start, end) of the bridged chunks
+        self.buffer = []           # Delta X_eps: (start, end) ranges of bridged chunks
+        self.primary, self.secondary = "R1", "R2"
+        self.is_reconciling = False
+
+    def reconcile_start(self, k_target: int) -> None:
+        self.is_reconciling = True
+        self.buffer = []
+
+    def reconcile_done(self, k_target: int) -> None:
+        self.buffer = []
+        self.k_ready = k_target
+
+    def inference(self, j_t: int, k_t: int, j_eps_t: int):
+        if self.j_eps is None:
+            self.j_eps = j_eps_t
+        # case 1: sequence continuation
+        if k_t == self.k:
+            if j_t > self.j:
+                self.x_recon = (0, j_t)
+                self.j = j_t
+            return "continue", self.primary
+        # case 2: reconciliation
+        if k_t > self.k:
+            if k_t > self.k_ready:
+                # the secondary has not finished: bridge the new chunks on the primary
+                delta = (self.j_eps, j_t)
+                self.buffer.append(delta)
+                self.j_eps = j_t
+                return "bridge", self.primary
+            if k_t == self.k_ready:
+                # the secondary has finished: resource swap
+                self.primary, self.secondary = self.secondary, self.primary
+                self.is_reconciling = False
+                self.x_recon = (0, j_t)
+                self.j, self.k, self.j_eps = j_t, k_t, None
+                return "swap", self.primary
+        # case 3: straggler queries
+        if self.is_reconciling:
+            return "straggler_primary", self.primary
+        return "straggler_secondary", self.secondary
+

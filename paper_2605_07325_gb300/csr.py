@@ -32,6 +32,7 @@ FLAG_PLAN_ONLY = 0x1
 FLAG_SINGLE_TILE = 0x2
 FLAG_PIPE_64 = 0x4
 RECON_IDLE, RECON_RUNNING, RECON_SWAPPED = 0, 1, 2
+ROUTE_CONTINUE, ROUTE_BRIDGE, ROUTE_SWAPPED, ROUTE_STRAGGLER = 0, 1, 2, 3
 VERSION_ACTIVE, VERSION_PENDING = 0, 1
 
 
@@ -79,6 +80,8 @@ _SIGS = {
     "csr_append_chunk": ([_vp, _vp, _vp, _vp, _i32, _vp, _vp, _vp, _P64], ctypes.c_int),
     "csr_append_chunk_attend_suffix": ([_vp, _vp, _vp, _vp, _i32, _i32, _vp, _vp, _vp, _P64],
                                        ctypes.c_int),
+    "csr_get_versions": ([_vp, _P64, _P64], ctypes.c_int),
+    "csr_route": ([_vp, ctypes.c_int64, _vp, ctypes.POINTER(ctypes.c_int)], ctypes.c_int),
     "csr_attend_suffix": ([_vp, _vp, _vp, _vp, _i32, _vp, _vp, _vp], ctypes.c_int),
     "csr_truncate_suffix": ([_vp], ctypes.c_int),
     "csr_rewind": ([_vp, _i64], ctypes.c_int),
@@ -276,6 +279,20 @@ class Context:
         if st.value == RECON_SWAPPED:
             self._keep.clear()
         return st.value
+
+    def versions(self) -> Tuple[int, int]:
+        """(k, k_ready) of Algorithm 2."""
+        k, kr = ctypes.c_int64(0), ctypes.c_int64(0)
+        self._check(_lib.csr_get_versions(self._h, ctypes.byref(k), ctypes.byref(kr)))
+        return k.value, kr.value
+
+    def route(self, k_t: int, stream=None) -> int:
+        """Algorithm 2's routing of a query built on version k_t (ROUTE_*)."""
+        r = ctypes.c_int(0)
+        self._check(_lib.csr_route(self._h, int(k_t), _stream_ptr_opt(self, stream), ctypes.byref(r)))
+        if r.value == ROUTE_SWAPPED:
+            self._keep.clear()
+        return r.value
 
     # ------------------------------------------------------------ inspection
     def layout(self, which: int = VERSION_ACTIVE) -> Tuple[List[int], int]:

@@ -238,6 +238,8 @@ struct csr_ctx {
   std::vector<Buffered> buffer;      // Delta X_buffer (N_catchup > 0): chunk and its position
   std::vector<int32_t> reserved_ids; // fresh ids the compaction kernel must produce
   bool ids_checked = false;
+  bool ready = false;                 // the rebuild is complete (Algorithm 2's k_ready = k + 1)
+  int64_t version = 0;                // active sequence version k (swaps so far)
   bool deferred_evict = false;        // a fused call reached tau_mem: evict at the truncation
   csr_stream_t deferred_stream = nullptr;
   csr_qkv_provider provider = nullptr;
@@ -667,6 +669,7 @@ void abort_reconcile(csr_ctx *c) {
   if (!c->plan_only && c->lo) cudaStreamSynchronize(c->lo);
   drop_version(c, c->pend());
   c->reconciling = false;
+  c->ready = false;
   c->buffer.clear();
   c->reserved_ids.clear();
 }
@@ -958,13 +961,15 @@ csr_status csr_evict_and_reconcile(csr_ctx *c, int32_t evict_tokens, csr_stream_
   return CSR_OK;
 }
 
-csr_status csr_poll_swap(csr_ctx *c, csr_stream_t fg_stream, int *state) {
-  if (!c || !state) return CSR_EINVAL;
-  if (!c->reconciling) {
-    *state = CSR_RECON_IDLE;
-    return CSR_OK;
-  }
-  *state = CSR_RECON_RUNNING;
+namespace {
+
+// One step of Algorithm 1's Reconcile loop without the swap: surface a
+// failure of R_2, check the compaction kernel's pages once the rebuild has
+// finished, and while more than N_catchup chunks are buffered hand them to
+// R_2.  *ready: the rebuilt version (k + 1) is complete up to at most
+// N_catchup buffered chunks (Algorithm 2's k_ready = k + 1).
+csr_status reconcile_progress(csr_ctx *c, csr_stream_t fg_stream, bool *ready) {
+  *ready = false;
   if (!c->plan_only) {
     // R_2 is done when its queue is empty and its last launch has finished;
     // a task that failed there aborts the reconciliation here.
@@ -1014,7 +1019,14 @@ csr_status csr_poll_swap(csr_ctx *c, csr_stream_t fg_stream, int *state) {
     }
     return CSR_OK;
   }
-  if (c->act().suffix_len > 0) return CSR_OK;  // swap only between tasks
+  *ready = true;
+  return CSR_OK;
+}
+
+// App. D step 5: compute the remaining buffered chunks on the foreground and
+// swap the active version atomically; the old version's own pages return to
+// the pool (the shared prefix pages stay referenced).
+csr_status reconcile_swap(csr_ctx *c, csr_stream_t fg_stream) {
   // The remainder (<= N_catchup chunks) is computed now, on the foreground.
   if (!c->buffer.empty()) {
     std::vector<csr_ctx::Buffered> rest;
@@ -1034,14 +1046,67 @@ csr_status csr_poll_swap(csr_ctx *c, csr_stream_t fg_stream, int *state) {
       }
     }
   }
-  // Atomic swap of the active version (App. D step 5); the old version's own
-  // pages return to the pool (the shared prefix pages stay referenced).
   const int old = c->active.load();
   c->active.store(1 - old);
   drop_version(c, c->ver[old]);
   c->reconciling = false;
   c->reserved_ids.clear();
-  *state = CSR_RECON_SWAPPED;
+  c->ready = false;
+  ++c->version;
+  return CSR_OK;
+}
+
+}  // namespace
+
+csr_status csr_poll_swap(csr_ctx *c, csr_stream_t fg_stream, int *state) {
+  if (!c || !state) return CSR_EINVAL;
+  if (!c->reconciling) {
+    *state = CSR_RECON_IDLE;
+    return CSR_OK;
+  }
+  *state = CSR_RECON_RUNNING;
+  bool ready = false;
+  csr_status st = reconcile_progress(c, fg_stream, &ready);
+  c->ready = ready;
+  if (st != CSR_OK || !ready) return st;
+  if (c->act().suffix_len > 0) return CSR_OK;  // swap only between tasks
+  st = reconcile_swap(c, fg_stream);
+  if (st == CSR_OK) *state = CSR_RECON_SWAPPED;
+  return st;
+}
+
+csr_status csr_get_versions(csr_ctx *c, int64_t *k, int64_t *k_ready) {
+  if (!c) return CSR_EINVAL;
+  if (k) *k = c->version;
+  if (k_ready) *k_ready = c->version + ((c->reconciling && c->ready) ? 1 : 0);
+  return CSR_OK;
+}
+
+csr_status csr_route(csr_ctx *c, int64_t k_t, csr_stream_t fg_stream, int *route) {
+  if (!c || !route) return CSR_EINVAL;
+  const int64_t k = c->version;
+  if (k_t == k) {                       // Algorithm 2, case 1: sequence continuation
+    *route = CSR_ROUTE_CONTINUE;
+    return CSR_OK;
+  }
+  if (k_t < k) {                        // case 3: straggler
+    *route = CSR_ROUTE_STRAGGLER;
+    return CSR_OK;
+  }
+  if (k_t != k + 1 || !c->reconciling)
+    return fail(c, CSR_EINVAL, "k_t names no version of this context");
+  // case 2: the query is built on the evicted sequence k + 1
+  bool ready = false;
+  csr_status st = reconcile_progress(c, fg_stream, &ready);
+  c->ready = ready;
+  if (st != CSR_OK) return st;
+  if (ready && c->act().suffix_len == 0) {   // k_t = k_ready: resource swap
+    st = reconcile_swap(c, fg_stream);
+    if (st != CSR_OK) return st;
+    *route = CSR_ROUTE_SWAPPED;
+    return CSR_OK;
+  }
+  *route = CSR_ROUTE_BRIDGE;            // k_t > k_ready: bridge on the active version
   return CSR_OK;
 }
 

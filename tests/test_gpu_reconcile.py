@@ -144,6 +144,44 @@ def test_fused_steps_through_eviction_cycles(libcsr):
     p.device_clean()
 
 
+def test_routing_swaps_on_first_query_of_rebuilt_version(libcsr):
+    """Algorithm 2 on the GPU: queries of the evicted sequence (k_t = k + 1)
+    are bridged on the active version until the rebuild is ready, and the
+    first one after that swaps; the swapped cache matches the oracle."""
+    csr = csr_mod()
+    p = Pair(C2, pool_pages=256, max_seq=8192, max_new=512)
+    lo = torch.cuda.Stream(priority=0)
+    outs = {}
+    p.ctx.set_reconciler(_provider(p, outs), lo)
+    p.init_static(p.blk(970, 300))
+    for i in range(12):
+        p.append(p.blk(971 + i, 200))
+    assert p.ctx.route(0) == csr.ROUTE_CONTINUE
+    p.ctx.evict_and_reconcile(600)
+    p.orc.evict(600)
+    routes, seed = [], 990
+    while True:
+        r = p.ctx.route(1)
+        routes.append(r)
+        if r == csr.ROUTE_SWAPPED:
+            break
+        assert r == csr.ROUTE_BRIDGE and len(routes) < 10000
+        if len(routes) <= 3:            # bridged tasks: their chunks join the rebuild
+            p.append(p.blk(seed, 64))
+            p.suffix(p.blk(seed + 100, 16))
+            p.truncate()
+            seed += 1
+    assert p.ctx.versions() == (1, 1)
+    p.orc.reconcile()
+    torch.cuda.synchronize()
+    p.check_layout()
+    p.check_cache()
+    assert p.ctx.route(0) == csr.ROUTE_STRAGGLER
+    p.suffix(p.blk(999, 33))
+    p.truncate()
+    p.device_clean()
+
+
 def test_provider_failure_keeps_old_version(libcsr):
     csr = csr_mod()
     p = Pair(C1, pool_pages=128, max_seq=4096, max_new=256)
