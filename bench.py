@@ -678,7 +678,8 @@ def run_sweep(args):
                     ctx.attend_suffix(q, k, v, out=o, stream=stream)
                     ctx.truncate_suffix()
                 stream.synchronize()
-                ctx.set_timing(True)
+                # whole calls, untimed inside (the library's per-kernel events
+                # would add their own cost to short calls) ...
                 e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
                 e0.record(stream)
                 for _ in range(K):
@@ -686,9 +687,15 @@ def run_sweep(args):
                     ctx.truncate_suffix()
                 e1.record(stream)
                 stream.synchronize()
+                us = e0.elapsed_time(e1) / K * 1e3
+                # ... then the per-kernel split from a second, event-timed pass
+                ctx.set_timing(True)
+                for _ in range(K):
+                    ctx.attend_suffix(q, k, v, out=o, stream=stream)
+                    ctx.truncate_suffix()
+                stream.synchronize()
                 t = ctx.get_timing()
                 ctx.set_timing(False)
-                us = e0.elapsed_time(e1) / K * 1e3
                 f = costmodel.attention_flops(HQ, D, L, n)
                 b = costmodel.call_bytes(HQ, HKV, D, L, n)
                 floor = costmodel.floor_seconds(f, b, peak, hbm) * 1e6

@@ -273,6 +273,7 @@ __global__ void __launch_bounds__(192, 1) attn_kernel(const __grid_constant__ At
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  pdl_wait();   // the block's queries, keys and page table come from the previous kernel
   const uint32_t tmem = bars->tmem_base;
   volatile int *abort = &bars->abort;
   ItemWalker walk{static_cast<int32_t>(blockIdx.x)};
@@ -553,6 +554,7 @@ __global__ void __launch_bounds__(192, 1) attn_kernel(const __grid_constant__ At
     }
   }
 
+  pdl_launch_dependents();
   tc_fence_before();
   __syncthreads();
   if (warp == 5) {
@@ -677,6 +679,7 @@ __global__ void __launch_bounds__(kPairThreads, 1) attn_pair_kernel(const __grid
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  pdl_wait();   // the block's queries, keys and page table come from the previous kernel
   const uint32_t tmem = bars->tmem_base;
   volatile int *abort = &bars->abort;
   PairWalker walk{static_cast<int32_t>(blockIdx.x)};
@@ -970,6 +973,7 @@ __global__ void __launch_bounds__(kPairThreads, 1) attn_pair_kernel(const __grid
     }
   }
 
+  pdl_launch_dependents();
   tc_fence_before();
   __syncthreads();
   if (warp == 9) {
@@ -1065,6 +1069,7 @@ __global__ void __launch_bounds__(320, 1) attn_pipe_kernel(const __grid_constant
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  pdl_wait();   // the block's queries, keys and page table come from the previous kernel
   const uint32_t tmem = bars->tmem_base;
   volatile int *abort = &bars->abort;
   PairWalker walk{static_cast<int32_t>(blockIdx.x)};
@@ -1374,6 +1379,7 @@ __global__ void __launch_bounds__(320, 1) attn_pipe_kernel(const __grid_constant
     }
   }
 
+  pdl_launch_dependents();
   tc_fence_before();
   __syncthreads();
   if (warp == 9) {
@@ -1404,6 +1410,7 @@ __device__ __forceinline__ void load_row_part(const float *src, float (&v)[kPer]
 
 template <int HD>
 __global__ void __launch_bounds__(256, 4) merge_kernel(const __grid_constant__ MergeParams p) {
+  pdl_wait();   // the partials come from the attention kernel
   const int head = blockIdx.x / p.n_tiles;
   const int tile = blockIdx.x - head * p.n_tiles;
   const int T = kBM / p.group;
@@ -1517,33 +1524,43 @@ cudaError_t attn_configure(int head_dim) {
   return e;
 }
 
+// Launch with programmatic stream serialisation (see pdl_wait).
+template <typename... Args>
+cudaError_t launch_pdl(void (*kernel)(Args...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                       const Args &...args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, args...);
+}
+
 cudaError_t launch_attention(const AttnParams &p, int head_dim, cudaStream_t s) {
   if (p.unit_tiles == 2 && p.kv_tile == kBN64) {
     if (head_dim == 64)
-      attn_pipe_kernel<64><<<p.grid, 320, PipeCfg<64>::kSmem, s>>>(p);
-    else
-      attn_pipe_kernel<128><<<p.grid, 320, PipeCfg<128>::kSmem, s>>>(p);
-  } else if (p.unit_tiles == 2) {
-    if (head_dim == 64)
-      attn_pair_kernel<64><<<p.grid, kPairThreads, PairCfg<64>::kSmem, s>>>(p);
-    else
-      attn_pair_kernel<128><<<p.grid, kPairThreads, PairCfg<128>::kSmem, s>>>(p);
-  } else {
-    if (head_dim == 64)
-      attn_kernel<64><<<p.grid, 192, AttnCfg<64>::kSmem, s>>>(p);
-    else
-      attn_kernel<128><<<p.grid, 192, AttnCfg<128>::kSmem, s>>>(p);
+      return launch_pdl(attn_pipe_kernel<64>, dim3(p.grid), dim3(320), PipeCfg<64>::kSmem, s, p);
+    return launch_pdl(attn_pipe_kernel<128>, dim3(p.grid), dim3(320), PipeCfg<128>::kSmem, s, p);
   }
-  return cudaGetLastError();
+  if (p.unit_tiles == 2) {
+    if (head_dim == 64)
+      return launch_pdl(attn_pair_kernel<64>, dim3(p.grid), dim3(kPairThreads), PairCfg<64>::kSmem, s, p);
+    return launch_pdl(attn_pair_kernel<128>, dim3(p.grid), dim3(kPairThreads), PairCfg<128>::kSmem, s, p);
+  }
+  if (head_dim == 64)
+    return launch_pdl(attn_kernel<64>, dim3(p.grid), dim3(192), AttnCfg<64>::kSmem, s, p);
+  return launch_pdl(attn_kernel<128>, dim3(p.grid), dim3(192), AttnCfg<128>::kSmem, s, p);
 }
 
 cudaError_t launch_merge(const MergeParams &p, cudaStream_t s) {
   const dim3 grid(p.hkv * p.n_tiles, kBM / 8);
-  if (p.d == 64)
-    merge_kernel<64><<<grid, 256, 0, s>>>(p);
-  else
-    merge_kernel<128><<<grid, 256, 0, s>>>(p);
-  return cudaGetLastError();
+  if (p.d == 64) return launch_pdl(merge_kernel<64>, grid, dim3(256), 0, s, p);
+  return launch_pdl(merge_kernel<128>, grid, dim3(256), 0, s, p);
 }
 
 }  // namespace csr

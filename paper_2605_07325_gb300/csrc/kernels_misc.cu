@@ -10,6 +10,7 @@
 
 #include "../../include/csr.h"
 #include "internal.h"
+#include "ptx.cuh"
 
 namespace csr {
 
@@ -58,6 +59,9 @@ __global__ void __launch_bounds__(256) rope_append_kernel(const __grid_constant_
     cs[i] = c;
     sn[i] = s;
   }
+  // The previous kernel of the stream may still read the packed queries and
+  // cache pages this block overwrites.
+  pdl_wait();
   if (blockIdx.x == 0 && blockIdx.y == 0 && p.n_ids > 0) {
     for (int i = threadIdx.x; i < p.n_ids; i += blockDim.x) p.page_table[p.first_lp + i] = p.ids[i];
   }
@@ -102,6 +106,7 @@ __global__ void __launch_bounds__(256) rope_append_kernel(const __grid_constant_
       *reinterpret_cast<uint4 *>(dst) = *reinterpret_cast<const uint4 *>(src);
     }
   }
+  pdl_launch_dependents();
 }
 
 cudaError_t launch_rope_append(const RopeAppendParams &p, cudaStream_t s) {
@@ -110,8 +115,16 @@ cudaError_t launch_rope_append(const RopeAppendParams &p, cudaStream_t s) {
   // one CTA per token and would only recompute the angle table.
   const int items = (p.hq + p.hkv) * (p.d / 16) + p.hkv * (p.d / 8);
   const dim3 grid(p.n, p.n < 128 ? (items + 255) / 256 : 1);
-  rope_append_kernel<<<grid, 256, 0, s>>>(p);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = dim3(256);
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, rope_append_kernel, p);
 }
 
 // K4: one block.  Copies the shared prefix entries, takes the n_new smallest

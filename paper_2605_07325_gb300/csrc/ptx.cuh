@@ -72,6 +72,17 @@ __device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, volati
   }
 }
 
+// ---------------------------------------------------- programmatic dependent launch
+// Kernels of a call are launched with programmatic stream serialisation: a
+// kernel may start while its predecessor in the stream finishes, runs its
+// setup, and waits here before its first global-memory access (returns at
+// once when the launch did not allow the overlap).
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+// This CTA's results are written: the dependent kernel may begin launching.
+__device__ __forceinline__ void pdl_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 // ---------------------------------------------------------------- TMA
 __device__ __forceinline__ void tma_prefetch_desc(const CUtensorMap *map) {
   asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
