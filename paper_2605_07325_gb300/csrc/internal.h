@@ -64,7 +64,14 @@ struct MergeParams {
   float *lse;
   int64_t L;
   int32_t n, hq, hkv, group, n_tiles, chunk_tiles, unit_tiles, kv_tile, d;
+  int32_t warps_per_row;   // 1, 2, 4 or 8 warps share one row's chunks
 };
+
+// Warps per merged row for rows of up to max_chunks partials.  Rows of many
+// chunks (short blocks over long contexts) are split over eight warps; below
+// 33 chunks the extra blocks and the shared-memory sum cost more than the
+// parallel loads save (measured at 10-20 chunks on the 64/4/128 head shape).
+inline int32_t merge_warps_per_row(int64_t max_chunks) { return max_chunks > 32 ? 8 : 1; }
 
 // K4: eviction / compaction: new version's page table from the free bitmap.
 struct EvictParams {

@@ -1408,8 +1408,15 @@ __device__ __forceinline__ void load_row_part(const float *src, float (&v)[kPer]
   }
 }
 
+// K3: one block of 8 warps merges `8 / wpr` rows of one query tile, wpr
+// warps per row (wpr = p.warps_per_row, from the chunk count: many chunks per
+// row are split over several warps so their loads run in parallel).  Each
+// warp of a row computes the row's LSE statistics, accumulates its share of
+// the chunks' normalised partial rows weighted by exp2(lse_k - lse), and the
+// shares are summed through shared memory.
 template <int HD>
 __global__ void __launch_bounds__(256, 4) merge_kernel(const __grid_constant__ MergeParams p) {
+  __shared__ float red[8][HD];
   pdl_wait();   // the partials come from the attention kernel
   const int head = blockIdx.x / p.n_tiles;
   const int tile = blockIdx.x - head * p.n_tiles;
@@ -1420,10 +1427,13 @@ __global__ void __launch_bounds__(256, 4) merge_kernel(const __grid_constant__ M
   const int half = tile - unit * p.unit_tiles;
   const int64_t kv = unit_iters(p.L, p.n, T, unit * p.unit_tiles + p.unit_tiles - 1, p.kv_tile);
   const int nk = static_cast<int>((kv + p.chunk_tiles - 1) / p.chunk_tiles);
-  if (nk <= 1) return;  // written whole by the attention kernel
-  const int r = blockIdx.y * 8 + warp;
+  if (nk <= 1) return;  // the whole block: written whole by the attention kernel
+  const int wpr = p.warps_per_row;
+  const int rows_pb = 8 / wpr;
+  const int sub = warp % wpr;
+  const int r = blockIdx.y * rows_pb + warp / wpr;
   const int64_t t = static_cast<int64_t>(tile) * T + r / p.group;
-  if (r >= kBM || t >= p.n) return;
+  const bool valid = r < kBM && t < p.n;
   const int64_t units = static_cast<int64_t>(p.hkv) * uph;
   const int64_t rows_per_item = static_cast<int64_t>(p.unit_tiles) * kBM;
   const int64_t row_in_item = static_cast<int64_t>(half) * kBM + r;
@@ -1437,11 +1447,11 @@ __global__ void __launch_bounds__(256, 4) merge_kernel(const __grid_constant__ M
 #pragma unroll
   for (int e = 0; e < kPer; ++e) acc[e] = 0.f;
   float lse2 = -CUDART_INF_F;
-  if (nk <= 64) {
+  if (valid && nk <= 64) {
     // Every chunk's LSE sits in a register of lane k % 32 (loaded once), so
     // the maximum, the sum and each chunk's weight (broadcast by shuffle)
-    // need no second pass over memory; the rows are then read four chunks
-    // at a time (more in flight costs registers, hence occupancy).
+    // need no second pass over memory; this warp then reads chunks sub,
+    // sub + wpr, ... four at a time.
     const float l0 = lane < nk ? p.part_lse[prow(lane)] : -CUDART_INF_F;
     const float l1 = lane + 32 < nk ? p.part_lse[prow(lane + 32)] : -CUDART_INF_F;
     float mx = fmaxf(l0, l1);
@@ -1457,12 +1467,13 @@ __global__ void __launch_bounds__(256, 4) merge_kernel(const __grid_constant__ M
       const float inv = 1.0f / sum;
       const float w0 = e0 * inv, w1 = e1 * inv;
       constexpr int kU = 4;
-      for (int k0 = 0; k0 < nk; k0 += kU) {
+      for (int k0 = sub; k0 < nk; k0 += kU * wpr) {
         float v[kU][kPer];
 #pragma unroll
         for (int u = 0; u < kU; ++u) {
-          if (k0 + u < nk) {
-            load_row_part<kPer>(p.part_o + prow(k0 + u) * HD + lane * kPer, v[u]);
+          const int k = k0 + u * wpr;
+          if (k < nk) {
+            load_row_part<kPer>(p.part_o + prow(k) * HD + lane * kPer, v[u]);
           } else {
 #pragma unroll
             for (int e = 0; e < kPer; ++e) v[u][e] = 0.f;
@@ -1470,7 +1481,7 @@ __global__ void __launch_bounds__(256, 4) merge_kernel(const __grid_constant__ M
         }
 #pragma unroll
         for (int u = 0; u < kU; ++u) {
-          const int k = k0 + u;
+          const int k = k0 + u * wpr;
           const float w = __shfl_sync(0xffffffffu, k < 32 ? w0 : w1, k & 31);
           if (k < nk) {
 #pragma unroll
@@ -1479,7 +1490,7 @@ __global__ void __launch_bounds__(256, 4) merge_kernel(const __grid_constant__ M
         }
       }
     }
-  } else {
+  } else if (valid) {
     float mx = -CUDART_INF_F;
     for (int k = lane; k < nk; k += 32) mx = fmaxf(mx, p.part_lse[prow(k)]);
 #pragma unroll
@@ -1490,7 +1501,7 @@ __global__ void __launch_bounds__(256, 4) merge_kernel(const __grid_constant__ M
 #pragma unroll
       for (int off = 16; off > 0; off >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, off);
       lse2 = mx + log2f(sum);
-      for (int k = 0; k < nk; ++k) {
+      for (int k = sub; k < nk; k += wpr) {
         const int64_t base = prow(k);
         const float w = ex2_approx(p.part_lse[base] - lse2);
         float v[kPer];
@@ -1500,6 +1511,17 @@ __global__ void __launch_bounds__(256, 4) merge_kernel(const __grid_constant__ M
       }
     }
   }
+  if (wpr > 1) {   // sum the row's shares
+#pragma unroll
+    for (int e = 0; e < kPer; ++e) red[warp][lane * kPer + e] = acc[e];
+    __syncthreads();
+    if (sub == 0) {
+      for (int w = 1; w < wpr; ++w)
+#pragma unroll
+        for (int e = 0; e < kPer; ++e) acc[e] += red[warp + w][lane * kPer + e];
+    }
+  }
+  if (!valid || sub != 0) return;
   const int hq_idx = head * p.group + r % p.group;
   uint16_t *dst = p.out + (t * p.hq + hq_idx) * HD + lane * kPer;
 #pragma unroll
@@ -1558,7 +1580,7 @@ cudaError_t launch_attention(const AttnParams &p, int head_dim, cudaStream_t s) 
 }
 
 cudaError_t launch_merge(const MergeParams &p, cudaStream_t s) {
-  const dim3 grid(p.hkv * p.n_tiles, kBM / 8);
+  const dim3 grid(p.hkv * p.n_tiles, kBM / (8 / p.warps_per_row));
   if (p.d == 64) return launch_pdl(merge_kernel<64>, grid, dim3(256), 0, s, p);
   return launch_pdl(merge_kernel<128>, grid, dim3(256), 0, s, p);
 }

@@ -106,7 +106,9 @@ class Pair:
         q, k, v = self._dev(b)
         lse = self._lse(b.n)
         out, _ = self.ctx.init_static(q, k, v, lse=lse)
+        self.orc.attend = compare
         exp = self.orc.init_static(*b.f64())
+        self.orc.attend = True
         torch.cuda.synchronize()
         self._check("init_static", out, lse, exp, compare)
         return out, lse
