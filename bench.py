@@ -253,7 +253,8 @@ def run_ours(args):
     cfg = csr.make_config(HQ, HKV, D, P, BASE, max_new_tokens=PREFIX, pool_pages=pool_pages,
                           max_seq_tokens=max_tokens + P,
                           flags={"pair": 0, "pipe": csr.FLAG_PIPE_64,
-                                 "single": csr.FLAG_SINGLE_TILE}[args.kernel])
+                                 "single": csr.FLAG_SINGLE_TILE}[args.kernel],
+                          fg_chunk_tiles=args.fg_chunk_tiles)
     stream = torch.cuda.Stream(device=dev, priority=-1)
     gen = torch.Generator(device=dev).manual_seed(1234 + rank)
 
@@ -725,6 +726,8 @@ def main(argv=None):
     ap.add_argument("--step", choices=["fused", "separate"], default="fused",
                     help="how a step calls the library: separate (csr_append_chunk then "
                          "csr_attend_suffix) or fused (csr_append_chunk_attend_suffix, one pass)")
+    ap.add_argument("--fg-chunk-tiles", type=int, default=0,
+                    help="key tiles per attention work item (0: the library's cost model)")
     ap.add_argument("--kernel", choices=["pair", "pipe", "single"], default="pair",
                     help="attention kernel: pair (default: two query tiles per CTA, 128-key "
                          "tiles), pipe (two query tiles, 64-key tiles, two score buffers each), "
