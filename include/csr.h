@@ -298,6 +298,15 @@ csr_status csr_get_versions(csr_ctx *ctx, int64_t *k, int64_t *k_ready);
  */
 csr_status csr_route(csr_ctx *ctx, int64_t k_t, csr_stream_t fg_stream, int *route);
 
+/*
+ * Abandon the running reconciliation (App. D: the swap never happens on a
+ * rebuild that did not finish): rebuild work not yet enqueued is dropped, work
+ * already on the low-priority stream runs to completion (this call waits for
+ * it), and the rebuilt version's pages return to the pool.  The active
+ * version is untouched.  CSR_ESTATE when no reconciliation runs.
+ */
+csr_status csr_cancel_reconcile(csr_ctx *ctx);
+
 /* Which version an inspection call reads. */
 #define CSR_VERSION_ACTIVE 0
 #define CSR_VERSION_PENDING 1

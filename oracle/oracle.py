@@ -372,6 +372,17 @@ class OracleCSR:
         self._swap()
         return outs
 
+    def cancel(self) -> None:
+        """Abandon the reconciliation (App. D: the swap never follows an
+        unfinished rebuild): the rebuilt version's page references are
+        released; the active version, including the chunks appended while
+        reconciling, stays as it is."""
+        assert self.pending is not None
+        for pid in self.pending.pages:
+            self.alloc.release(pid)
+        self.pending = None
+        self.buffer = []
+
     def _swap(self):
         old = self.active
         for pid in old.pages:

@@ -81,6 +81,7 @@ _SIGS = {
     "csr_append_chunk_attend_suffix": ([_vp, _vp, _vp, _vp, _i32, _i32, _vp, _vp, _vp, _P64],
                                        ctypes.c_int),
     "csr_get_versions": ([_vp, _P64, _P64], ctypes.c_int),
+    "csr_cancel_reconcile": ([_vp], ctypes.c_int),
     "csr_route": ([_vp, ctypes.c_int64, _vp, ctypes.POINTER(ctypes.c_int)], ctypes.c_int),
     "csr_attend_suffix": ([_vp, _vp, _vp, _vp, _i32, _vp, _vp, _vp], ctypes.c_int),
     "csr_truncate_suffix": ([_vp], ctypes.c_int),
@@ -279,6 +280,11 @@ class Context:
         if st.value == RECON_SWAPPED:
             self._keep.clear()
         return st.value
+
+    def cancel_reconcile(self) -> None:
+        """Abandon the running reconciliation; the active version stays."""
+        self._check(_lib.csr_cancel_reconcile(self._h))
+        self._keep.clear()
 
     def versions(self) -> Tuple[int, int]:
         """(k, k_ready) of Algorithm 2."""

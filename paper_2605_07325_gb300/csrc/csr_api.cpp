@@ -23,6 +23,7 @@
 #include <cuda.h>
 #include <cudaTypedefs.h>
 #include <cuda_runtime.h>
+#include <nvtx3/nvToolsExt.h>
 
 #include "../../include/csr.h"
 #include "internal.h"
@@ -30,6 +31,15 @@
 using namespace csr;
 
 namespace {
+
+// NVTX range around an entry point or a rebuild task (visible in profilers;
+// no cost beyond a call when no tool is attached).
+struct Range {
+  explicit Range(const char *name) { nvtxRangePushA(name); }
+  ~Range() { nvtxRangePop(); }
+  Range(const Range &) = delete;
+  Range &operator=(const Range &) = delete;
+};
 
 constexpr int kFgGridDefaultCap = 304;   // 2 x 152 SMs
 constexpr int kPartialItems = 4096;      // split partials a launch may write (per staging)
@@ -579,6 +589,7 @@ void worker_main(csr_ctx *c) {
     csr_status st = CSR_OK;
     msg.clear();
     if (!skip) {
+      Range range(t.compact ? "csr_rebuild_compact" : "csr_rebuild_chunk");
       if (t.compact) {
         const cudaError_t e = launch_evict(*t.compact, c->lo);
         if (e != cudaSuccess) st = cuda_fail(c, e, "evict_compact launch");
@@ -777,6 +788,7 @@ void csr_destroy(csr_ctx *c) {
 
 csr_status csr_init_static(csr_ctx *c, const void *q, const void *k, const void *v, int32_t n,
                            void *out, float *lse, csr_stream_t stream) {
+  Range range("csr_init_static");
   if (!c) return CSR_EINVAL;
   if (c->has_static) return fail(c, CSR_ESTATE, "static prefix already initialised");
   csr_status st = add_block(c, Kind::Prefix, q, k, v, n, out, lse,
@@ -787,6 +799,7 @@ csr_status csr_init_static(csr_ctx *c, const void *q, const void *k, const void 
 
 csr_status csr_append_chunk(csr_ctx *c, const void *q, const void *k, const void *v, int32_t n,
                             void *out, float *lse, csr_stream_t stream, int64_t *chunk_id) {
+  Range range("csr_append_chunk");
   if (!c) return CSR_EINVAL;
   if (!c->has_static) return fail(c, CSR_ESTATE, "csr_init_static must come first");
   if (c->act().suffix_len > 0) return fail(c, CSR_ESTATE, "a suffix is live: truncate it first");
@@ -803,6 +816,7 @@ csr_status csr_append_chunk(csr_ctx *c, const void *q, const void *k, const void
 csr_status csr_append_chunk_attend_suffix(csr_ctx *c, const void *q, const void *k, const void *v,
                                           int32_t n_chunk, int32_t n_suffix, void *out, float *lse,
                                           csr_stream_t stream, int64_t *chunk_id) {
+  Range range("csr_append_chunk_attend_suffix");
   if (!c) return CSR_EINVAL;
   if (!c->has_static) return fail(c, CSR_ESTATE, "csr_init_static must come first");
   if (c->act().suffix_len > 0) return fail(c, CSR_ESTATE, "a suffix is live: truncate it first");
@@ -824,6 +838,7 @@ csr_status csr_append_chunk_attend_suffix(csr_ctx *c, const void *q, const void 
 
 csr_status csr_attend_suffix(csr_ctx *c, const void *q, const void *k, const void *v, int32_t n,
                              void *out, float *lse, csr_stream_t stream) {
+  Range range("csr_attend_suffix");
   if (!c) return CSR_EINVAL;
   if (!c->has_static) return fail(c, CSR_ESTATE, "csr_init_static must come first");
   if (c->act().suffix_len > 0) return fail(c, CSR_ESTATE, "a suffix is already live");
@@ -881,6 +896,7 @@ csr_status csr_set_reconciler(csr_ctx *c, csr_qkv_provider provider, void *user,
 }
 
 csr_status csr_evict_and_reconcile(csr_ctx *c, int32_t evict_tokens, csr_stream_t fg_stream) {
+  Range range("csr_evict_and_reconcile");
   if (!c) return CSR_EINVAL;
   if (c->reconciling) return fail(c, CSR_EBUSY, "a reconciliation is already running");
   if (!c->provider) return fail(c, CSR_ESTATE, "no reconciler registered");
@@ -1060,6 +1076,7 @@ csr_status reconcile_swap(csr_ctx *c, csr_stream_t fg_stream) {
 }  // namespace
 
 csr_status csr_poll_swap(csr_ctx *c, csr_stream_t fg_stream, int *state) {
+  Range range("csr_poll_swap");
   if (!c || !state) return CSR_EINVAL;
   if (!c->reconciling) {
     *state = CSR_RECON_IDLE;
@@ -1084,6 +1101,7 @@ csr_status csr_get_versions(csr_ctx *c, int64_t *k, int64_t *k_ready) {
 }
 
 csr_status csr_route(csr_ctx *c, int64_t k_t, csr_stream_t fg_stream, int *route) {
+  Range range("csr_route");
   if (!c || !route) return CSR_EINVAL;
   const int64_t k = c->version;
   if (k_t == k) {                       // Algorithm 2, case 1: sequence continuation
@@ -1108,6 +1126,13 @@ csr_status csr_route(csr_ctx *c, int64_t k_t, csr_stream_t fg_stream, int *route
     return CSR_OK;
   }
   *route = CSR_ROUTE_BRIDGE;            // k_t > k_ready: bridge on the active version
+  return CSR_OK;
+}
+
+csr_status csr_cancel_reconcile(csr_ctx *c) {
+  if (!c) return CSR_EINVAL;
+  if (!c->reconciling) return fail(c, CSR_ESTATE, "no reconciliation running");
+  abort_reconcile(c);
   return CSR_OK;
 }
 

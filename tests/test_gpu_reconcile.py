@@ -182,6 +182,40 @@ def test_routing_swaps_on_first_query_of_rebuilt_version(libcsr):
     p.device_clean()
 
 
+def test_deadline_and_cancel(libcsr):
+    """csr_wait_reconcile with a deadline the rebuild cannot meet returns
+    CSR_ETIMEOUT and leaves it running; csr_cancel_reconcile abandons it (the
+    active version keeps serving, the pending pages return to the pool); a
+    second eviction then runs to the swap and matches the oracle."""
+    csr = csr_mod()
+    p = Pair(C2, pool_pages=256, max_seq=8192, max_new=1024)
+    lo = torch.cuda.Stream(priority=0)
+    outs = {}
+    p.ctx.set_reconciler(_provider(p, outs), lo)
+    p.init_static(p.blk(1100, 300))
+    for i in range(6):
+        p.append(p.blk(1101 + i, 300))
+    free_before = p.ctx.free_pages()
+    p.ctx.evict_and_reconcile(600)
+    with pytest.raises(csr.CsrError) as e:
+        p.ctx.wait_reconcile(1e-6)
+    assert e.value.status == csr.ETIMEOUT
+    p.ctx.cancel_reconcile()
+    assert p.ctx.free_pages() == free_before
+    assert p.ctx.poll_swap() == csr.RECON_IDLE
+    p.check_layout()
+    p.suffix(p.blk(1120, 40))               # the active version still serves
+    p.truncate()
+    p.ctx.evict_and_reconcile(600)
+    p.orc.evict(600)
+    assert p.ctx.wait_reconcile(60.0) == csr.RECON_SWAPPED
+    p.orc.reconcile()
+    torch.cuda.synchronize()
+    p.check_layout()
+    p.check_cache()
+    p.device_clean()
+
+
 def test_provider_failure_keeps_old_version(libcsr):
     csr = csr_mod()
     p = Pair(C1, pool_pages=128, max_seq=4096, max_new=256)

@@ -276,3 +276,33 @@ def test_fused_step_errors(libcsr):
     _err(libcsr, lambda: ctx.append_chunk(None, None, None, n=4), libcsr.ESTATE)
     ctx.truncate_suffix()
     assert ctx.layout()[1] == 20
+
+
+def test_cancel_reconcile_restores_layout(libcsr):
+    """csr_cancel_reconcile: the rebuilt version's pages return to the pool and
+    the active version keeps every chunk appended meanwhile (its page ids as
+    reserved while the rebuild ran); a later eviction runs normally."""
+    ctx = _plan(libcsr, pool=128)
+    m = _Model(128)
+    ctx.set_reconciler(lambda cid, n: None)
+    ctx.init_static(None, None, None, n=37)
+    m.o.init_static(*m.blk(37))
+    for _ in range(5):
+        ctx.append_chunk(None, None, None, n=21)
+        m.o.append_chunk(*m.blk(21))
+    ctx.evict_and_reconcile(40)
+    m.o.evict(40)
+    for _ in range(2):                       # forked into the rebuild, then abandoned
+        ctx.append_chunk(None, None, None, n=13)
+        m.o.append_chunk(*m.blk(13))
+    ctx.cancel_reconcile()
+    m.o.cancel()
+    _same(ctx, m, libcsr)
+    assert ctx.poll_swap() == libcsr.RECON_IDLE
+    _err(libcsr, lambda: ctx.cancel_reconcile(), libcsr.ESTATE)
+    ctx.evict_and_reconcile(40)
+    m.o.evict(40)
+    _same(ctx, m, libcsr, "pending")
+    assert ctx.wait_reconcile(5.0) == libcsr.RECON_SWAPPED
+    m.o.reconcile()
+    _same(ctx, m, libcsr)
