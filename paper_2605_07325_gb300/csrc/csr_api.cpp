@@ -4,10 +4,11 @@
 // the transient X_dyn suffix), the physical page pool (smallest free id
 // first), two cache versions (the active one and the one a reconciliation
 // rebuilds, Algorithm 1 / App. D), and the launch of the kernels:
-//   K1 rope_append  -> K2 attention (stream-K split) -> K3 merge   per block
-//   K4 evict_compact                                                per eviction
+//   K1 rope_append  -> K2 attention (split over key chunks) -> K3 merge   per block
+//   K4 evict_compact                                                       per eviction
 // The foreground runs on the caller's stream; the rebuild and its catch-up
-// run on the low-priority stream registered with csr_set_reconciler.
+// run on the low-priority stream registered with csr_set_reconciler, fed by
+// the context's reconciliation thread (the host side of R_2).
 #include <algorithm>
 #include <atomic>
 #include <chrono>

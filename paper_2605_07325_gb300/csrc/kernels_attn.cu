@@ -14,18 +14,27 @@
 // written directly; otherwise each item writes a normalised partial output
 // with its log-sum-exp and K3 merges them.
 //
-// CTA roles (192 threads):
-//   warp 4 lane 0  TMA producer: the Q tile, then K and V tiles page by page
-//                  (page table lookup per 64/16-token page), into 128-byte
-//                  swizzled shared memory rings;
-//   warp 5 lane 0  MMA issuer: S = Q K^T into one of two TMEM score buffers
-//                  (tcgen05.mma, both operands in shared memory), then
-//                  O += P V with P read from TMEM and V from shared memory;
-//   warps 0-3      softmax: one thread per query row (its TMEM lane); masks
-//                  keys past the row's position, keeps a running max with a
-//                  lazy rescale of O (only when the max grows by more than
-//                  2^8), writes P as bf16 over its own score columns, and
-//                  finally normalises O and stores it.
+// Kernels.  attn_pair_kernel (the default) gives each CTA two consecutive
+// query tiles of one KV head, so every K/V tile staged in shared memory feeds
+// both; attn_kernel (one query tile per CTA, two score buffers) and
+// attn_pipe_kernel (two query tiles, 64-key tiles, two score buffers each) are
+// earlier designs kept behind flags.  Roles of the default (320 threads):
+//   warp 8    TMA producer: the two Q tiles, then K and V tiles page by page
+//             (page ids staged in shared memory), into 128-byte-swizzled
+//             shared-memory stages; the whole warp runs the loop and an
+//             elected lane issues the copies;
+//   warp 9    MMA issuer: S_X = Q_X K^T (both operands in shared memory) and
+//             O_X += P_X V (P from TMEM) for X = A, B, ordered PV_A(i),
+//             S_A(i+1), PV_B(i), S_B(i+1); the whole warp runs the loop and
+//             elect.sync picks the issuing lane;
+//   warps 0-7 softmax, one warpgroup per query tile: one thread per query row
+//             (its TMEM lane); masks keys past the row's position, keeps a
+//             running max with a lazy rescale of O (only when the max grows
+//             by more than 2^8), writes P as bf16 over its own score columns,
+//             and finally normalises O and stores it.
+// The kernels of a call (K1 rope/append, K2 attention, K3 merge) are chained
+// by programmatic dependent launch: each runs its setup while its predecessor
+// finishes and waits (griddepcontrol) before its first global access.
 // Every wait on an mbarrier is bounded (CSR_DEVERR_WAIT_TIMEOUT).
 #include <cuda_bf16.h>
 #include <math_constants.h>
