@@ -22,8 +22,10 @@ inside the timed region.  `roofline` is the attention kernel's achieved
 TFLOP/s (algorithmic FLOPs / its CUDA-event time) against the measured bf16
 peak; `cpu_baseline` times the fp64 CPU oracle on a bounded sample of the
 same step.  With N > 1 (torchrun) every rank runs an independent replica
-(the path does not shard: one layer's cache lives on one GPU); the slowest
-rank's time is reported.  `--impl reference` times the fp64 oracle alone.
+(the path does not shard: one layer's cache lives on one GPU); `value` is the
+whole job's time per layer-step, the slowest replica's step time divided by N
+(N layer-steps per step time), and config.replica_us_per_step the step time
+itself.  `--impl reference` times the fp64 oracle alone.
 """
 from __future__ import annotations
 
@@ -375,8 +377,10 @@ def run_ours(args):
                                           costmodel.call_bytes(HQ, HKV, D, L0 + CHUNK, SUFFIX),
                                           peak_burst, hbm)) * 1e6
     us_step = ms_total / K * 1e3
+    # the whole job: `world` replicas each process one layer-step per step time
+    us_job = us_step / world
     line = {
-        "metric": METRIC, "value": us_step, "unit": UNIT, "n_gpus": world, "steps": K,
+        "metric": METRIC, "value": us_job, "unit": UNIT, "n_gpus": world, "steps": K,
         "warmup": W, "ms_per_step": ms_total / K, "higher_is_better": False, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic: seeded N(0,1) bf16 Q/K/V (torch CUDA generator), resident in HBM",
@@ -385,7 +389,8 @@ def run_ours(args):
                                   "csr_append_chunk + csr_attend_suffix + csr_truncate_suffix"),
                    "step_flops": step_flops,
                    "l2": "inputs larger than L2: the 252 MB KV cache is streamed every step",
-                   "replicas": world, "foreground_ctas": ctx.cfg.num_ctas or props.multi_processor_count},
+                   "replicas": world, "replica_us_per_step": us_step,
+                   "foreground_ctas": ctx.cfg.num_ctas or props.multi_processor_count},
         "roofline": {"bound": "tensor", "achieved": achieved, "peak": peak_burst, "unit": "TFLOP/s",
                      "frac": (achieved / peak_burst) if achieved else None,
                      "traffic": traffic,
@@ -399,7 +404,7 @@ def run_ours(args):
                           "note": "max(FLOPs / bf16 peak, bytes / HBM peak) per call, summed over the step"},
         "ttft_proxy_94_layers_ms": us_step * LAYERS_PROXY / 1e3,
         "kernels": {k: {"ms_total": v[0], "launches": v[1]} for k, v in ktimes.items() if v[1]},
-        "e2e": {"value": ms_e2e / K * 1e3, "unit": UNIT, "h2d_bytes_per_step": h2d,
+        "e2e": {"value": ms_e2e / K * 1e3 / world, "unit": UNIT, "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h},
         "gpu_launches": launches,
         "clocks": clocks,
