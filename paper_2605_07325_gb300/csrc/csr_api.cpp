@@ -452,7 +452,7 @@ csr_status run_block(csr_ctx *c, int slot, int ws, const void *q, const void *k,
     mp.unit_tiles = ap.unit_tiles;
     mp.kv_tile = ap.kv_tile;
     mp.d = cf.head_dim;
-    mp.warps_per_row = merge_warps_per_row(n_chunks);
+    mp.slots_per_row = merge_slots_per_row(n_chunks, mp.d);
     e = timed_launch(c, CSR_KERNEL_MERGE, fg, s, [&] { return launch_merge(mp, s); });
     if (e != cudaSuccess) return cuda_fail(c, e, "merge launch");
     ++c->launches;

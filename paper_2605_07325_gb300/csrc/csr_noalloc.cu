@@ -216,7 +216,7 @@ extern "C" csr_status csr_attend_block_noalloc(const csr_block_args *a, csr_stre
     mp.unit_tiles = 2;
     mp.kv_tile = kBN;
     mp.d = d;
-    mp.warps_per_row = merge_warps_per_row(n_chunks);
+    mp.slots_per_row = merge_slots_per_row(n_chunks, mp.d);
     if (launch_merge(mp, s) != cudaSuccess) return CSR_ECUDA;
   }
   return CSR_OK;

@@ -64,14 +64,20 @@ struct MergeParams {
   float *lse;
   int64_t L;
   int32_t n, hq, hkv, group, n_tiles, chunk_tiles, unit_tiles, kv_tile, d;
-  int32_t warps_per_row;   // 1, 2, 4 or 8 warps share one row's chunks
+  int32_t slots_per_row;   // lane groups sharing one row's chunks (a power of two)
 };
 
-// Warps per merged row for rows of up to max_chunks partials.  Rows of many
-// chunks (short blocks over long contexts) are split over eight warps; below
-// 33 chunks the extra blocks and the shared-memory sum cost more than the
-// parallel loads save (measured at 10-20 chunks on the 64/4/128 head shape).
-inline int32_t merge_warps_per_row(int64_t max_chunks) { return max_chunks > 32 ? 8 : 1; }
+// K3 merge: a row's partials are read by slots of head_dim / 8 lanes, each
+// with at most kMergeChunksPerSlot partial rows in flight; rows of more
+// chunks are spread over 2, 4, ... slots (up to a whole block of
+// 256 / (head_dim / 8) slots, which then loops over its chunks).
+constexpr int kMergeChunksPerSlot = 4;
+inline int32_t merge_slots_per_row(int64_t max_chunks, int head_dim) {
+  const int32_t block_slots = 256 / (head_dim / 8);
+  int32_t spr = 1;
+  while (spr < block_slots && spr * kMergeChunksPerSlot < max_chunks) spr *= 2;
+  return spr;
+}
 
 // K4: eviction / compaction: new version's page table from the free bitmap.
 struct EvictParams {

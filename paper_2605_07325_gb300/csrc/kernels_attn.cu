@@ -968,11 +968,15 @@ __global__ void __launch_bounds__(kPairThreads, 1) attn_pair_kernel(const __grid
         }
       } else {
         const int64_t base = static_cast<int64_t>(seg.item) * (2 * kBM) + wg * kBM + row;
-        float4 *d4 = reinterpret_cast<float4 *>(p.part_o + base * HD);
+        // the partial buffer is 256-byte aligned and rows are HD floats: 32-byte stores
+        float *dst = p.part_o + base * HD;
 #pragma unroll
-        for (int c = 0; c < HD / 4; ++c)
-          d4[c] = make_float4(__uint_as_float(o[4 * c]) * inv_l, __uint_as_float(o[4 * c + 1]) * inv_l,
-                              __uint_as_float(o[4 * c + 2]) * inv_l, __uint_as_float(o[4 * c + 3]) * inv_l);
+        for (int c = 0; c < HD / 8; ++c) {
+          uint32_t w[8];
+#pragma unroll
+          for (int e = 0; e < 8; ++e) w[e] = __float_as_uint(__uint_as_float(o[8 * c + e]) * inv_l);
+          st_global_v8(dst + 8 * c, w);
+        }
         p.part_lse[base] = lse2;
       }
       tc_fence_before();
@@ -1402,45 +1406,46 @@ __global__ void __launch_bounds__(320, 1) attn_pipe_kernel(const __grid_constant
 // Merge the key-chunk pieces of one row: lse = log2 sum_k 2^lse_k and
 // O = sum_k 2^(lse_k - lse) O_k (each O_k already normalised by its own sum).
 // One warp per packed row; lanes own head_dim/32 output columns.
-// kPer consecutive floats of a partial row (16-byte loads for kPer = 4).
-template <int kPer>
-__device__ __forceinline__ void load_row_part(const float *src, float (&v)[kPer]) {
-  if constexpr (kPer == 4) {
-    const float4 x = *reinterpret_cast<const float4 *>(src);
-    v[0] = x.x; v[1] = x.y; v[2] = x.z; v[3] = x.w;
-  } else {
-#pragma unroll
-    for (int e = 0; e < kPer; e += 2) {
-      const float2 x = *reinterpret_cast<const float2 *>(src + e);
-      v[e] = x.x; v[e + 1] = x.y;
-    }
-  }
+// 32-byte global loads (the partial buffer is 256-byte aligned and its rows
+// are HD floats, so every lane's eight floats start on a 32-byte boundary).
+__device__ __forceinline__ void ld_global_v8f(const float *ptr, float (&v)[8]) {
+  asm volatile("ld.global.v8.f32 {%0, %1, %2, %3, %4, %5, %6, %7}, [%8];"
+               : "=f"(v[0]), "=f"(v[1]), "=f"(v[2]), "=f"(v[3]), "=f"(v[4]), "=f"(v[5]), "=f"(v[6]),
+                 "=f"(v[7])
+               : "l"(ptr));
 }
 
-// K3: one block of 8 warps merges `8 / wpr` rows of one query tile, wpr
-// warps per row (wpr = p.warps_per_row, from the chunk count: many chunks per
-// row are split over several warps so their loads run in parallel).  Each
-// warp of a row computes the row's LSE statistics, accumulates its share of
-// the chunks' normalised partial rows weighted by exp2(lse_k - lse), and the
-// shares are summed through shared memory.
+// K3: combine the split-KV partials of every row: lse = log2(sum_k 2^lse_k),
+// out = sum_k 2^(lse_k - lse) * O_k (each O_k already normalised by its own
+// row sum).  A row is read by a group of HD / 8 lanes (eight floats, one
+// 32-byte load per lane per chunk); a block of 256 threads holds 256 / (HD/8)
+// such slots.  The merge is bound by how many bytes are in flight, so every
+// load of a slot -- the LSEs of all chunks and up to kMergeChunksPerSlot
+// partial rows -- is issued before any is used; rows with more chunks are
+// spread over p.slots_per_row slots whose shares are summed in shared memory.
+// Rows with more than 64 chunks loop over their chunks.
 template <int HD>
 __global__ void __launch_bounds__(256, 4) merge_kernel(const __grid_constant__ MergeParams p) {
-  __shared__ float red[8][HD];
+  constexpr int kLanes = HD / 8;            // lanes per slot (16 or 8)
+  constexpr int kSlots = 256 / kLanes;      // slots per block (16 or 32)
+  constexpr int kLse = 64 / kLanes;         // LSE registers per lane for up to 64 chunks
+  constexpr int kC = kMergeChunksPerSlot;
+  __shared__ float red[kSlots][HD];
   pdl_wait();   // the partials come from the attention kernel
   const int head = blockIdx.x / p.n_tiles;
   const int tile = blockIdx.x - head * p.n_tiles;
   const int T = kBM / p.group;
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int uph = (p.n_tiles + p.unit_tiles - 1) / p.unit_tiles;  // units per head
   const int unit = tile / p.unit_tiles;
   const int half = tile - unit * p.unit_tiles;
   const int64_t kv = unit_iters(p.L, p.n, T, unit * p.unit_tiles + p.unit_tiles - 1, p.kv_tile);
   const int nk = static_cast<int>((kv + p.chunk_tiles - 1) / p.chunk_tiles);
   if (nk <= 1) return;  // the whole block: written whole by the attention kernel
-  const int wpr = p.warps_per_row;
-  const int rows_pb = 8 / wpr;
-  const int sub = warp % wpr;
-  const int r = blockIdx.y * rows_pb + warp / wpr;
+  const int spr = p.slots_per_row;
+  const int slot = threadIdx.x / kLanes;
+  const int sl = threadIdx.x % kLanes;
+  const int sub = slot % spr;
+  const int r = blockIdx.y * (kSlots / spr) + slot / spr;
   const int64_t t = static_cast<int64_t>(tile) * T + r / p.group;
   const bool valid = r < kBM && t < p.n;
   const int64_t units = static_cast<int64_t>(p.hkv) * uph;
@@ -1451,93 +1456,98 @@ __global__ void __launch_bounds__(256, 4) merge_kernel(const __grid_constant__ M
     return (static_cast<int64_t>(k) * units + static_cast<int64_t>(head) * uph + unit) * rows_per_item +
            row_in_item;
   };
-  constexpr int kPer = HD / 32;  // floats per lane
-  float acc[kPer];
+  float acc[8];
 #pragma unroll
-  for (int e = 0; e < kPer; ++e) acc[e] = 0.f;
+  for (int e = 0; e < 8; ++e) acc[e] = 0.f;
   float lse2 = -CUDART_INF_F;
-  if (valid && nk <= 64) {
-    // Every chunk's LSE sits in a register of lane k % 32 (loaded once), so
-    // the maximum, the sum and each chunk's weight (broadcast by shuffle)
-    // need no second pass over memory; this warp then reads chunks sub,
-    // sub + wpr, ... four at a time.
-    const float l0 = lane < nk ? p.part_lse[prow(lane)] : -CUDART_INF_F;
-    const float l1 = lane + 32 < nk ? p.part_lse[prow(lane + 32)] : -CUDART_INF_F;
-    float mx = fmaxf(l0, l1);
+  // Shuffles run on every lane (rows past n included) and stay within a slot.
+  auto slot_max = [&](float x) {
 #pragma unroll
-    for (int off = 16; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
-    if (mx != -CUDART_INF_F) {
-      const float e0 = lane < nk ? ex2_approx(l0 - mx) : 0.f;
-      const float e1 = lane + 32 < nk ? ex2_approx(l1 - mx) : 0.f;
-      float sum = e0 + e1;
+    for (int off = kLanes / 2; off > 0; off >>= 1) x = fmaxf(x, __shfl_xor_sync(0xffffffffu, x, off, kLanes));
+    return x;
+  };
+  auto slot_sum = [&](float x) {
 #pragma unroll
-      for (int off = 16; off > 0; off >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, off);
-      lse2 = mx + log2f(sum);
-      const float inv = 1.0f / sum;
-      const float w0 = e0 * inv, w1 = e1 * inv;
-      constexpr int kU = 4;
-      for (int k0 = sub; k0 < nk; k0 += kU * wpr) {
-        float v[kU][kPer];
+    for (int off = kLanes / 2; off > 0; off >>= 1) x += __shfl_xor_sync(0xffffffffu, x, off, kLanes);
+    return x;
+  };
+  if (nk <= 64 && nk <= kC * spr) {
+    // lane sl holds the LSEs of chunks sl, sl + kLanes, ...
+    float l[kLse];
 #pragma unroll
-        for (int u = 0; u < kU; ++u) {
-          const int k = k0 + u * wpr;
-          if (k < nk) {
-            load_row_part<kPer>(p.part_o + prow(k) * HD + lane * kPer, v[u]);
-          } else {
+    for (int i = 0; i < kLse; ++i) {
+      const int k = sl + i * kLanes;
+      l[i] = (valid && k < nk) ? p.part_lse[prow(k)] : -CUDART_INF_F;
+    }
+    // this slot's chunks: their partial rows and (the same address on every
+    // lane of the slot) their LSEs
+    float v[kC][8], lk[kC];
 #pragma unroll
-            for (int e = 0; e < kPer; ++e) v[u][e] = 0.f;
-          }
-        }
+    for (int u = 0; u < kC; ++u) {
+      const int k = sub + u * spr;
+      if (valid && k < nk) {
+        lk[u] = p.part_lse[prow(k)];
+        ld_global_v8f(p.part_o + prow(k) * HD + sl * 8, v[u]);
+      } else {
+        lk[u] = -CUDART_INF_F;
 #pragma unroll
-        for (int u = 0; u < kU; ++u) {
-          const int k = k0 + u * wpr;
-          const float w = __shfl_sync(0xffffffffu, k < 32 ? w0 : w1, k & 31);
-          if (k < nk) {
-#pragma unroll
-            for (int e = 0; e < kPer; ++e) acc[e] = fmaf(w, v[u][e], acc[e]);
-          }
-        }
+        for (int e = 0; e < 8; ++e) v[u][e] = 0.f;
       }
     }
-  } else if (valid) {
+    float mx = l[0];
+#pragma unroll
+    for (int i = 1; i < kLse; ++i) mx = fmaxf(mx, l[i]);
+    mx = slot_max(mx);
+    const float m_use = mx == -CUDART_INF_F ? 0.f : mx;
+    float sum = 0.f;
+#pragma unroll
+    for (int i = 0; i < kLse; ++i) sum += ex2_approx(l[i] - m_use);   // 0 for absent chunks
+    sum = slot_sum(sum);
+    lse2 = sum > 0.f ? m_use + log2f(sum) : -CUDART_INF_F;
+    if (sum > 0.f) {
+#pragma unroll
+      for (int u = 0; u < kC; ++u) {
+        const float w = ex2_approx(lk[u] - lse2);
+#pragma unroll
+        for (int x = 0; x < 8; ++x) acc[x] = fmaf(w, v[u][x], acc[x]);
+      }
+    }
+  } else {
     float mx = -CUDART_INF_F;
-    for (int k = lane; k < nk; k += 32) mx = fmaxf(mx, p.part_lse[prow(k)]);
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
-    if (mx != -CUDART_INF_F) {
-      float sum = 0.f;
-      for (int k = lane; k < nk; k += 32) sum += ex2_approx(p.part_lse[prow(k)] - mx);
-#pragma unroll
-      for (int off = 16; off > 0; off >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, off);
-      lse2 = mx + log2f(sum);
-      for (int k = sub; k < nk; k += wpr) {
+    for (int k = sl; k < nk; k += kLanes) mx = fmaxf(mx, valid ? p.part_lse[prow(k)] : -CUDART_INF_F);
+    mx = slot_max(mx);
+    const float m_use = mx == -CUDART_INF_F ? 0.f : mx;
+    float sum = 0.f;
+    for (int k = sl; k < nk; k += kLanes) sum += valid ? ex2_approx(p.part_lse[prow(k)] - m_use) : 0.f;
+    sum = slot_sum(sum);
+    lse2 = sum > 0.f ? m_use + log2f(sum) : -CUDART_INF_F;
+    if (valid && sum > 0.f) {
+      for (int k = sub; k < nk; k += spr) {
         const int64_t base = prow(k);
         const float w = ex2_approx(p.part_lse[base] - lse2);
-        float v[kPer];
-        load_row_part<kPer>(p.part_o + base * HD + lane * kPer, v);
+        float v[8];
+        ld_global_v8f(p.part_o + base * HD + sl * 8, v);
 #pragma unroll
-        for (int e = 0; e < kPer; ++e) acc[e] = fmaf(w, v[e], acc[e]);
+        for (int x = 0; x < 8; ++x) acc[x] = fmaf(w, v[x], acc[x]);
       }
     }
   }
-  if (wpr > 1) {   // sum the row's shares
+  if (spr > 1) {   // sum the row's shares
 #pragma unroll
-    for (int e = 0; e < kPer; ++e) red[warp][lane * kPer + e] = acc[e];
+    for (int x = 0; x < 8; ++x) red[slot][sl * 8 + x] = acc[x];
     __syncthreads();
     if (sub == 0) {
-      for (int w = 1; w < wpr; ++w)
+      for (int w = 1; w < spr; ++w)
 #pragma unroll
-        for (int e = 0; e < kPer; ++e) acc[e] += red[warp + w][lane * kPer + e];
+        for (int x = 0; x < 8; ++x) acc[x] += red[slot + w][sl * 8 + x];
     }
   }
   if (!valid || sub != 0) return;
   const int hq_idx = head * p.group + r % p.group;
-  uint16_t *dst = p.out + (t * p.hq + hq_idx) * HD + lane * kPer;
-#pragma unroll
-  for (int e = 0; e < kPer; e += 2) {
-    *reinterpret_cast<uint32_t *>(dst + e) = pack_bf16x2(acc[e], acc[e + 1]);
-  }
-  if (lane == 0 && p.lse) p.lse[static_cast<int64_t>(hq_idx) * p.n + t] = lse2 * 0.69314718055994531f;
+  uint16_t *dst = p.out + (t * p.hq + hq_idx) * HD + sl * 8;
+  *reinterpret_cast<uint4 *>(dst) = make_uint4(pack_bf16x2(acc[0], acc[1]), pack_bf16x2(acc[2], acc[3]),
+                                               pack_bf16x2(acc[4], acc[5]), pack_bf16x2(acc[6], acc[7]));
+  if (sl == 0 && p.lse) p.lse[static_cast<int64_t>(hq_idx) * p.n + t] = lse2 * 0.69314718055994531f;
 }
 
 cudaError_t attn_configure(int head_dim) {
@@ -1589,7 +1599,8 @@ cudaError_t launch_attention(const AttnParams &p, int head_dim, cudaStream_t s) 
 }
 
 cudaError_t launch_merge(const MergeParams &p, cudaStream_t s) {
-  const dim3 grid(p.hkv * p.n_tiles, kBM / (8 / p.warps_per_row));
+  const int slots = 256 / (p.d / 8);
+  const dim3 grid(p.hkv * p.n_tiles, kBM * p.slots_per_row / slots);
   if (p.d == 64) return launch_pdl(merge_kernel<64>, grid, dim3(256), 0, s, p);
   return launch_pdl(merge_kernel<128>, grid, dim3(256), 0, s, p);
 }

@@ -48,6 +48,10 @@ __device__ __forceinline__ void rotate8(const uint4 &a, const uint4 &b, const fl
 // 10^5 keep full fp32 angle accuracy.
 __global__ void __launch_bounds__(256) rope_append_kernel(const __grid_constant__ RopeAppendParams p) {
   __shared__ float cs[kMaxHalfDim], sn[kMaxHalfDim];
+  // The attention kernel may launch now: its setup (barriers, TMEM, tensor
+  // maps) overlaps this kernel, and it waits for this grid's writes before
+  // touching queries, keys or the page table.
+  pdl_launch_dependents();
   const int t = blockIdx.x;
   const int64_t pos = p.pos0 + t;
   const int half = p.d / 2;
@@ -106,7 +110,6 @@ __global__ void __launch_bounds__(256) rope_append_kernel(const __grid_constant_
       *reinterpret_cast<uint4 *>(dst) = *reinterpret_cast<const uint4 *>(src);
     }
   }
-  pdl_launch_dependents();
 }
 
 cudaError_t launch_rope_append(const RopeAppendParams &p, cudaStream_t s) {

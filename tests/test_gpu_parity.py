@@ -196,12 +196,14 @@ def test_fused_step_matches_oracle(libcsr, shape, chunk_tiles):
     p.device_clean()
 
 
+@pytest.mark.parametrize("shape", [C1, C2], ids=["d64_p16_g4", "d128_p64_g16"])
 @pytest.mark.parametrize("chunk_tiles", [1, 2, 3, 9])
-def test_merge_many_chunks_per_row(libcsr, chunk_tiles):
+def test_merge_many_chunks_per_row(libcsr, shape, chunk_tiles):
     """Long context, short blocks, short key chunks: rows merged from up to 67
-    partials (the merge splits such rows over several warps, and above 64
-    partials takes its general path)."""
-    p = Pair(C2, pool_pages=256, max_seq=16384, max_new=4096, fg_chunk_tiles=chunk_tiles)
+    partials (the merge spreads such rows over several lane groups, and above
+    64 partials takes its general path)."""
+    pages = 16384 // shape["P"] + 64
+    p = Pair(shape, pool_pages=pages, max_seq=16384, max_new=4096, fg_chunk_tiles=chunk_tiles)
     p.init_static(p.blk(70, 4000), compare=False)
     p.append(p.blk(71, 4000), compare=False)
     p.append(p.blk(72, 500))
