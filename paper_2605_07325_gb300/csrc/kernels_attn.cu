@@ -28,7 +28,9 @@
 //             S_A(i+1), PV_B(i), S_B(i+1); the whole warp runs the loop and
 //             elect.sync picks the issuing lane;
 //   warps 0-7 softmax, one warpgroup per query tile: one thread per query row
-//             (its TMEM lane); masks keys past the row's position, keeps a
+//             (its TMEM lane); reads its scores with the row maximum reduced
+//             by the TMEM load (tcgen05.ld.red, sm_103a), masks keys past the
+//             row's position, keeps a
 //             running max with a lazy rescale of O (only when the max grows
 //             by more than 2^8), writes P as bf16 over its own score columns,
 //             and finally normalises O and stores it.
@@ -877,8 +879,11 @@ __global__ void __launch_bounds__(kPairThreads, 1) attn_pair_kernel(const __grid
           break;
         }
         tc_fence_after();
+        // The scores and their row maximum in one load (the TMEM load path
+        // reduces); tiles that reach past the row's causal limit mask the
+        // later keys and take the maximum of what is left.
         uint32_t sr[kBN];
-        tmem_ld128_wait(tmem + lane_base + s_col, sr);
+        float mx = tmem_ld128_rowmax_wait(tmem + lane_base + s_col, sr);
         float s[kBN];
 #pragma unroll
         for (int c = 0; c < kBN; ++c) s[c] = __uint_as_float(sr[c]);
@@ -887,15 +892,14 @@ __global__ void __launch_bounds__(kPairThreads, 1) attn_pair_kernel(const __grid
 #pragma unroll
           for (int c = 0; c < kBN; ++c)
             if (key0 + c > limit) s[c] = -CUDART_INF_F;
+          // three operands per instruction, eight independent chains
+          float mp[8];
+#pragma unroll
+          for (int e = 0; e < 8; ++e) mp[e] = fmaxf(s[2 * e], s[2 * e + 1]);
+#pragma unroll
+          for (int c = 16; c < kBN; c += 2) mp[(c >> 1) & 7] = max3f(mp[(c >> 1) & 7], s[c], s[c + 1]);
+          mx = max3f(max3f(mp[0], mp[1], mp[2]), max3f(mp[3], mp[4], mp[5]), fmaxf(mp[6], mp[7]));
         }
-        // Row max: three operands per instruction, eight independent chains.
-        float mp[8];
-#pragma unroll
-        for (int e = 0; e < 8; ++e) mp[e] = fmaxf(s[2 * e], s[2 * e + 1]);
-#pragma unroll
-        for (int c = 16; c < kBN; c += 2) mp[(c >> 1) & 7] = max3f(mp[(c >> 1) & 7], s[c], s[c + 1]);
-        const float mx = max3f(max3f(mp[0], mp[1], mp[2]), max3f(mp[3], mp[4], mp[5]),
-                               fmaxf(mp[6], mp[7]));
         const float mx_s = mx * p.scale_log2;
         const bool need = mx_s > m_ref + 8.0f;
         const float m_new = need ? mx_s : m_ref;

@@ -48,9 +48,11 @@ class Block:
 
 def block(seed: int, n: int, hq: int, hkv: int, d: int, kind: str = "normal") -> Block:
     """Draw one block.  ``kind``: "normal" (N(0,1)), "ones_v" (V = 1),
-    "zero_k" (K = 0), "const_q" (every query row equal), "kv_only" (K then V
-    are drawn from the seed and Q is all zero: fill-phase chunks of long
-    caches whose outputs are not compared)."""
+    "zero_k" (K = 0), "const_q" (every query row equal), "peaked" (Q and K
+    scaled by 12: scores spread over hundreds of units, so a softmax that
+    used a wrong row maximum would overflow or lose every weight),
+    "kv_only" (K then V are drawn from the seed and Q is all zero:
+    fill-phase chunks of long caches whose outputs are not compared)."""
     rng = np.random.default_rng(seed)
     if kind == "kv_only":
         k = rng.standard_normal((n, hkv, d), dtype=np.float32)
@@ -65,6 +67,9 @@ def block(seed: int, n: int, hq: int, hkv: int, d: int, kind: str = "normal") ->
         k[...] = 0.0
     elif kind == "const_q":
         q[...] = q[:1]
+    elif kind == "peaked":
+        q *= 12.0
+        k *= 12.0
     elif kind != "normal":
         raise ValueError(kind)
     return Block(bf16_bits(q), bf16_bits(k), bf16_bits(v))

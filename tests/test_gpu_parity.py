@@ -2,8 +2,8 @@
 
 Covers the tiny correctness configuration in full, the 64/4/128 head shape
 with ragged sizes, split-KV partial merging under forced CTA counts, edge
-cases (one token, n = max_new_tokens, special inputs) and run-to-run bitwise
-determinism.
+cases (one token, n = max_new_tokens, special inputs, scores spread over
+hundreds of units) and run-to-run bitwise determinism.
 """
 import math
 
@@ -11,7 +11,10 @@ import numpy as np
 import pytest
 import torch
 
-from gpu_util import C1, C2, Pair, assert_close, bits_of, to_f64
+from gpu_util import (C1, C2, TOL_LSE, TOL_MAX_ABS, TOL_REL_FRO, Pair, assert_close, bits_of,
+                      csr_mod, err_stats, to_dev, to_f64)
+from oracle import oracle as orc
+from paper_2605_07325_gb300 import synth
 
 pytestmark = pytest.mark.gpu
 
@@ -100,6 +103,56 @@ def test_special_inputs(libcsr):
     p2.append(p2.blk(52, 100, "zero_k"))
     p.device_clean()
     p2.device_clean()
+
+
+@pytest.mark.parametrize("shape", [C1, C2], ids=["d64_p16_g4", "d128_p64_g16"])
+def test_large_scores_match_oracle(libcsr, shape):
+    """Scores spread over hundreds of units (Q and K scaled by 12): the softmax
+    must take each row's true maximum -- from the reducing TMEM load on whole
+    key tiles, recomputed after masking on a row's diagonal tile -- and rescale
+    O when it jumps; a wrong maximum overflows (non-finite outputs) or flushes
+    every weight (zero rows).  At this scale the bf16 rounding of the rotated
+    queries and keys alone moves scores by ~0.2 and near-ties by as much, so
+    the bound is three times the difference the oracle itself shows between
+    exact and bf16-rounded rotated operands on the same inputs."""
+    csr = csr_mod()
+    hq, hkv, d, P, base = shape["hq"], shape["hkv"], shape["d"], shape["P"], shape["base"]
+    ctx = csr.Context(csr.make_config(hq, hkv, d, P, base, max_new_tokens=512, pool_pages=128,
+                                      max_seq_tokens=4096))
+    blocks = [synth.block(90 + i, n, hq, hkv, d, "peaked") for i, n in enumerate((300, 200, 50))]
+    ctx.init_static(*(to_dev(x) for x in (blocks[0].q, blocks[0].k, blocks[0].v)))
+    lse_c = torch.empty((hq, 200), dtype=torch.float32, device="cuda")
+    lse_s = torch.empty((hq, 50), dtype=torch.float32, device="cuda")
+    out_c, _, _ = ctx.append_chunk(*(to_dev(x) for x in (blocks[1].q, blocks[1].k, blocks[1].v)), lse=lse_c)
+    out_s, _ = ctx.attend_suffix(*(to_dev(x) for x in (blocks[2].q, blocks[2].k, blocks[2].v)), lse=lse_s)
+    torch.cuda.synchronize()
+    f64 = [b.f64() for b in blocks]
+    k = np.concatenate([x[1] for x in f64])
+    v = np.concatenate([x[2] for x in f64])
+    pos = np.arange(len(k))
+    k_rot = orc.rope(k, pos, base)
+
+    def rounded(x):
+        return synth.bf16_to_f64(synth.bf16_bits(x.astype(np.float32)))
+
+    scale = 1.0 / math.sqrt(d)
+    for (q, _, _), p0, out, lse in ((f64[1], 300, out_c, lse_c), (f64[2], 500, out_s, lse_s)):
+        qp = pos[p0:p0 + len(q)]
+        q_rot = orc.rope(q, qp, base)
+        exp_o, exp_l = orc.attention(q_rot, qp, k_rot[:qp[-1] + 1], v[:qp[-1] + 1], pos[:qp[-1] + 1], scale)
+        rnd_o, rnd_l = orc.attention(rounded(q_rot), qp, rounded(k_rot[:qp[-1] + 1]), v[:qp[-1] + 1],
+                                     pos[:qp[-1] + 1], scale)
+        got_o = to_f64(out)
+        got_l = lse.cpu().numpy().astype(np.float64)
+        assert np.all(np.isfinite(got_o)) and np.all(np.isfinite(got_l))
+        assert np.all(np.abs(got_o).reshape(len(q), -1).max(axis=1) > 0), "a row lost every weight"
+        base_abs, base_rel = err_stats(rnd_o, exp_o)
+        got_abs, got_rel = err_stats(got_o, exp_o)
+        assert got_rel <= 3 * base_rel + TOL_REL_FRO, (got_rel, base_rel)
+        assert got_abs <= 3 * base_abs + TOL_MAX_ABS, (got_abs, base_abs)
+        assert np.max(np.abs(got_l - exp_l)) <= 3 * np.max(np.abs(rnd_l - exp_l)) + TOL_LSE
+    assert ctx.device_status() == 0
+    ctx.close()
 
 
 def test_bitwise_deterministic(libcsr):
