@@ -682,8 +682,9 @@ SWEEP_N = (16, 64, 256, 1024, 4096)
 
 def run_sweep(args):
     """One attend call of n new tokens over L cached tokens for every sweep
-    point: device time per call, the attention kernel's time, achieved
-    TFLOP/s and GB/s, and the fraction of the roofline floor
+    point: device time per call (mean over K >= 20 back-to-back calls, and
+    the median and p99 of K single calls), the attention kernel's time,
+    achieved TFLOP/s and GB/s, and the fraction of the roofline floor
     max(FLOPs / bf16 peak, bytes / HBM peak)."""
     import torch
     from paper_2605_07325_gb300 import costmodel, csr
@@ -700,7 +701,8 @@ def run_sweep(args):
     def rnd(n, h):
         return torch.randn((n, h, D), generator=gen, device=dev, dtype=torch.float32).to(torch.bfloat16)
 
-    K, W = max(3, args.steps // 10), args.warmup
+    K, W = max(20, args.steps // 10), args.warmup
+    sweep_n = args.sweep_n or SWEEP_N
     points = []
     with torch.cuda.stream(stream):
         ctx = csr.Context(cfg, device=str(dev), stream=stream)
@@ -708,17 +710,24 @@ def run_sweep(args):
         fill_q = rnd(4096, HQ)
         fill_o = torch.empty((4096, HQ, D), dtype=torch.bfloat16, device=dev)
         blocks = {n: (rnd(n, HQ), rnd(n, HKV), rnd(n, HKV),
-                      torch.empty((n, HQ, D), dtype=torch.bfloat16, device=dev)) for n in SWEEP_N}
+                      torch.empty((n, HQ, D), dtype=torch.bfloat16, device=dev)) for n in sweep_n}
         for L in (args.sweep_l or SWEEP_L):
             while ctx.layout()[1] < L:
                 ctx.append_chunk(fill_q, rnd(4096, HKV), rnd(4096, HKV), out=fill_o, stream=stream)
             assert ctx.layout()[1] == L
-            for n in SWEEP_N:
+            for n in sweep_n:
                 q, k, v, o = blocks[n]
                 for _ in range(W):
                     ctx.attend_suffix(q, k, v, out=o, stream=stream)
                     ctx.truncate_suffix()
+                # one call inside an NVTX range "probe": what an ncu capture of a
+                # sweep point selects (--nvtx --nvtx-include probe/)
                 stream.synchronize()
+                torch.cuda.nvtx.range_push("probe")
+                ctx.attend_suffix(q, k, v, out=o, stream=stream)
+                ctx.truncate_suffix()
+                stream.synchronize()
+                torch.cuda.nvtx.range_pop()
                 # whole calls, untimed inside (the library's per-kernel events
                 # would add their own cost to short calls) ...
                 e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -729,7 +738,18 @@ def run_sweep(args):
                 e1.record(stream)
                 stream.synchronize()
                 us = e0.elapsed_time(e1) / K * 1e3
-                # ... then the per-kernel split from a second, event-timed pass
+                # ... the latency of single calls (an event pair around each:
+                # consecutive calls no longer overlap) ...
+                ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                      for _ in range(K)]
+                for a, b_ in ev:
+                    a.record(stream)
+                    ctx.attend_suffix(q, k, v, out=o, stream=stream)
+                    ctx.truncate_suffix()
+                    b_.record(stream)
+                stream.synchronize()
+                lat = sorted(a.elapsed_time(b_) * 1e3 for a, b_ in ev)
+                # ... then the per-kernel split from a third, event-timed pass
                 ctx.set_timing(True)
                 for _ in range(K):
                     ctx.attend_suffix(q, k, v, out=o, stream=stream)
@@ -741,7 +761,9 @@ def run_sweep(args):
                 b = costmodel.call_bytes(HQ, HKV, D, L, n)
                 floor = costmodel.floor_seconds(f, b, peak, hbm) * 1e6
                 att_us = t["attention"][0] / max(1, t["attention"][1]) * 1e3
-                pt = {"L": L, "n": n, "us_per_call": us, "attention_us": att_us,
+                pt = {"L": L, "n": n, "us_per_call": us, "calls": K,
+                      "us_median": lat[len(lat) // 2], "us_p99": lat[min(len(lat) - 1, int(0.99 * len(lat)))],
+                      "attention_us": att_us,
                       "rope_append_us": t["rope_append"][0] / K * 1e3, "merge_us": t["merge"][0] / K * 1e3,
                       "tflops": f / (us * 1e-6) / 1e12, "gbs": b / (us * 1e-6) / 1e9,
                       "floor_us": floor, "bound": "tensor" if f / (peak * 1e12) > b / (hbm * 1e9) else "hbm",
@@ -789,6 +811,8 @@ def main(argv=None):
                     help="run the L x n sweep instead of the 120K step line")
     ap.add_argument("--sweep-l", type=int, nargs="*", default=None,
                     help="cached lengths of the sweep (default: 16K 32K 64K 96K 128K)")
+    ap.add_argument("--sweep-n", type=int, nargs="*", default=None,
+                    help="new-token counts of the sweep (default: 16 64 256 1024 4096)")
     ap.add_argument("--unordered", action="store_true",
                     help="time the unordered baseline (full recompute per step) beside CSR")
     args = ap.parse_args(argv)
