@@ -35,8 +35,9 @@
 //             by more than 2^8), writes P as bf16 over its own score columns,
 //             and finally normalises O and stores it.
 // The kernels of a call (K1 rope/append, K2 attention, K3 merge) are chained
-// by programmatic dependent launch: each runs its setup while its predecessor
-// finishes and waits (griddepcontrol) before its first global access.
+// by programmatic dependent launch: K1 releases K2 at its entry and K2
+// releases K3 at its end; each runs its setup while its predecessor works and
+// waits (griddepcontrol) before its first global access.
 // Every wait on an mbarrier is bounded (CSR_DEVERR_WAIT_TIMEOUT).
 #include <cuda_bf16.h>
 #include <math_constants.h>

@@ -78,7 +78,8 @@ __device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, volati
 // setup, and waits here before its first global-memory access (returns at
 // once when the launch did not allow the overlap).
 __device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
-// This CTA's results are written: the dependent kernel may begin launching.
+// Let the dependent kernel begin launching (its pdl_wait still waits for this
+// grid to complete and its writes to be visible).
 __device__ __forceinline__ void pdl_launch_dependents() {
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 }
