@@ -461,8 +461,9 @@ ASR_CAP, ASR_EVICT = 131072, 32768
 
 def run_asr(args):
     """The ASR cycle run: cache capped at 131,072 tokens (4,096-token prefix),
-    foreground steps (256-token chunk + 512-token suffix + truncate) at a fixed
-    cadence; reaching the cap evicts the oldest 32,768 tokens of chunks and
+    foreground steps (256-token chunk + 512-token suffix + truncate; one fused
+    call, or two with --step separate) at a fixed cadence; reaching the cap
+    evicts the oldest 32,768 tokens of chunks and
     rebuilds the retained ~98K tokens on a low-priority stream (Algorithm 1),
     then swaps.  --asr-cap / --asr-evict / --asr-chunk change the setting (the
     paper's robot run: 100-token chunks, tau_mem = 110K, the oldest half of the
@@ -522,7 +523,9 @@ def run_asr(args):
             ctx.append_chunk(q, k, v, out=fout, stream=fg)
         sq, sk, sv = rnd(SUFFIX, HQ), rnd(SUFFIX, HKV), rnd(SUFFIX, HKV)
         so = torch.empty((SUFFIX, HQ, D), dtype=torch.bfloat16, device=dev)
+        step_out = torch.empty((chunk + SUFFIX, HQ, D), dtype=torch.bfloat16, device=dev)
     fg.synchronize()
+    fused = args.step == "fused"
 
     period = 1.0 / args.asr_cadence_hz if args.asr_cadence_hz > 0 else 0.0
     records, rebuilds, layout_ok = [], [], True
@@ -533,6 +536,8 @@ def run_asr(args):
     while cycles < args.asr_cycles:
         with torch.cuda.stream(fg):
             q, k, v = rnd(chunk, HQ), rnd(chunk, HKV), rnd(chunk, HKV)
+            if fused:   # the task's tokens as one block: the chunk, then the suffix
+                qs, ks, vs = torch.cat([q, sq]), torch.cat([k, sk]), torch.cat([v, sv])
         fg.synchronize()
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         t0 = time.perf_counter()
@@ -544,10 +549,13 @@ def run_asr(args):
         was = reconciling()
         e0.record(fg)
         chunks[len(chunks)] = (q, k, v)          # before the call: it may start a rebuild
-        _, _, cid = ctx.append_chunk(q, k, v, out=fout, stream=fg)
+        if fused:
+            _, _, cid = ctx.append_chunk_attend_suffix(qs, ks, vs, chunk, out=step_out, stream=fg)
+        else:
+            _, _, cid = ctx.append_chunk(q, k, v, out=fout, stream=fg)
+            ctx.attend_suffix(sq, sk, sv, out=so, stream=fg)
         assert cid == len(chunks) - 1
-        ctx.attend_suffix(sq, sk, sv, out=so, stream=fg)
-        ctx.truncate_suffix()
+        ctx.truncate_suffix()   # with the fused call, an eviction due starts here
         e1.record(fg)
         e1.synchronize()
         t1 = time.perf_counter()
@@ -575,6 +583,8 @@ def run_asr(args):
         "workload": (f"ASR cycle run: cap {cap:,} tokens, 4,096-token prefix, {chunk}-token chunks + "
                      f"512-token suffix per step, evict oldest {evict:,} tokens, rebuild on a "
                      "low-priority stream, 64 q / 4 kv heads, d 128, page 64, 1 layer"),
+        "step_calls": ("csr_append_chunk_attend_suffix + csr_truncate_suffix" if fused else
+                       "csr_append_chunk + csr_attend_suffix + csr_truncate_suffix"),
         "cadence_hz": args.asr_cadence_hz, "rebuild_tiles_per_cta": args.asr_rebuild_tiles or 16,
         "cycles": cycles, "steps": step,
         "steps_during_rebuild": len(dur),
