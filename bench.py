@@ -359,6 +359,10 @@ def run_ours(args):
     def run_e2e(n, start=None, end=None):
         if start is not None:
             start.record(stream)
+        if n == 0:
+            if end is not None:
+                end.record(stream)
+            return
         copy_stream.wait_stream(stream)
         upload(0)
         for i in range(n):
