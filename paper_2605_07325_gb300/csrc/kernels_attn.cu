@@ -1091,7 +1091,7 @@ __global__ void __launch_bounds__(320, 1) attn_pipe_kernel(const __grid_constant
   const uint32_t tmem = bars->tmem_base;
   volatile int *abort = &bars->abort;
   PairWalker walk{static_cast<int32_t>(blockIdx.x)};
-  Seg seg;
+  Seg seg{};
 
   if (warp == 8) {
     // ------------------------------------------------------ TMA producer
