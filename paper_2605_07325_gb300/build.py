@@ -2,9 +2,9 @@
 
     python -m paper_2605_07325_gb300.build [--force] [--verbose]
 
-Three translation units compile in parallel: the host API (g++), the
-attention kernels and the memory-bound kernels (nvcc, one -gencode for
-sm_103a).  The CUDA runtime is linked statically; the driver's libcuda is
+Four translation units compile in parallel: the host API (g++), the
+attention kernels, the memory-bound kernels and the no-allocation block
+entry (nvcc, one -gencode for sm_103a).  The CUDA runtime is linked statically; the driver's libcuda is
 reached at run time through cudaGetDriverEntryPointByVersion.
 """
 from __future__ import annotations
