@@ -13,7 +13,8 @@ HERE = os.path.dirname(os.path.abspath(__file__))
 HQ, HKV, D, P = 8, 2, 64, 16
 
 
-def test_oracle_router_matches_hand_trace():
+def run_hand_trace(orc):
+    """Replay the hand-derived trace on `orc.Alg2Router` (asserts on a mismatch)."""
     g = json.load(open(os.path.join(HERE, "golden", "alg2_routing.json")))
     r = orc.Alg2Router()
     for ev in g["events"]:
@@ -25,6 +26,12 @@ def test_oracle_router_matches_hand_trace():
             got = r.inference(ev["j_t"], ev["k_t"], ev["j_eps_t"])
             assert list(got) == ev["expect"], ev
             assert (r.k, r.k_ready) == (ev["k"], ev["k_ready"]), ev
+            assert (r.j, r.j_eps) == (ev["j"], ev["j_eps"]), ev
+            assert [list(x) for x in r.buffer] == ev["buffer"], ev
+
+
+def test_oracle_router_matches_hand_trace():
+    run_hand_trace(orc)
 
 
 def _plan(libcsr, n_catchup):
