@@ -416,62 +416,102 @@ class OracleCSR:
 # Algorithm 2: asynchronous state reconciliation with concurrent request routing
 # --------------------------------------------------------------------------
 class Alg2Router:
-    """The routing procedure of Algorithm 2, step by step in the paper's order
-    and notation, over sequence metadata only (the states are represented by
-    their static lengths j, and the caches by the resource names R1, R2).
+    """Which resource serves a query, and with which context, while a
+    reconciliation runs (Algorithm 2, procedures Inference and Reconcile).
 
-    ``inference(j_t, k_t, j_eps_t)`` classifies one query and returns
-    (case, resource): "continue" (case 1, k_t = k), "bridge" (case 2,
-    k_t > k_ready), "swap" (case 2, k_t = k_ready), "straggler_primary"
-    (case 3 while reconciling) or "straggler_secondary" (case 3 otherwise).
-    ``reconcile_start`` / ``reconcile_done`` are the first and last steps of
-    procedure Reconcile (lock R2 from stragglers, empty the buffer; authorise
-    the swap with k_ready <- k_target)."""
+    The states are text.  A query carries its static state ``x_static`` (the
+    prefix and chunks, j_t = len(x_static) characters), its dynamic suffix
+    ``x_dyn`` (suffix and task), the sequence version k_t it was built on, and,
+    for a state of the sequence produced by an eviction, ``j_eps_t``: how many
+    characters of x_static are old chunks kept from before the eviction (the
+    chunks past it arrived afterwards).
+
+    Router state, in the algorithm's names: j and k (static length and version
+    of the active sequence), k_ready (highest version whose cache the
+    secondary resource holds in full), j_eps (cursor into the rebuilt
+    sequence: its chunks past j_eps have not been bridged yet; unset until the
+    first query of that sequence), x_recon (the active sequence's static state
+    extended with every chunk bridged since the eviction), buffer (Delta X_eps:
+    the bridged chunks the secondary has still to catch up on), the two
+    resource names, is_reconciling, and x_eps (the state whose cache the
+    secondary is computing).
+
+    ``inference`` returns (case, resource, context): the case ("continue",
+    "bridge", "swap", "straggler_primary", "straggler_secondary"), the
+    resource that runs the model, and the text it runs on.
+
+    Reading of the cursor: j_eps_t is a property of states of the rebuilt
+    sequence, so only a query of version k + 1 sets j_eps (a query of the
+    active version that happens to arrive first leaves it unset), and every
+    bridged range starts at or before its end."""
 
     def __init__(self):
-        self.j = 0                 # current active sequence static length
-        self.k = 0                 # current active sequence version
-        self.k_ready = 0           # highest version fully precomputed on the secondary
-        self.j_eps = None          # evicted sequence static length (the eviction cursor)
-        self.x_recon = None        # reconciliation state: (start, end) of the bridged chunks
-        self.buffer = []           # Delta X_eps: (start, end) ranges of bridged chunks
+        self.j = 0
+        self.k = 0
+        self.k_ready = 0
+        self.j_eps = None
+        self.x_recon = ""
+        self.buffer: List[str] = []
         self.primary, self.secondary = "R1", "R2"
         self.is_reconciling = False
+        self.x_eps = None
 
-    def reconcile_start(self, k_target: int) -> None:
+    # ---- procedure Reconcile ---------------------------------------------------
+    def reconcile_start(self, x_eps: str, k_target: int) -> None:
+        """First steps: close the secondary to stragglers, empty the catch-up
+        buffer, and start computing the evicted state X_eps there."""
         self.is_reconciling = True
         self.buffer = []
+        self.x_eps = x_eps
+
+    def catch_up(self) -> str:
+        """One pass of the catch-up loop: take the buffered chunks (the buffer
+        is emptied for the queries that keep arriving) and extend the state
+        the secondary computes.  Returns the text handed to the secondary."""
+        taken = "".join(self.buffer)
+        self.buffer = []
+        self.x_eps = self.x_eps + taken
+        return taken
 
     def reconcile_done(self, k_target: int) -> None:
+        """Last steps: drop what is left in the buffer (the swap query
+        computes it) and authorise the swap."""
         self.buffer = []
         self.k_ready = k_target
 
-    def inference(self, j_t: int, k_t: int, j_eps_t: int):
-        if self.j_eps is None:
-            self.j_eps = j_eps_t
-        # case 1: sequence continuation
+    # ---- procedure Inference ---------------------------------------------------
+    def inference(self, x_static: str, x_dyn: str, k_t: int, j_eps_t=None):
+        j_t = len(x_static)
         if k_t == self.k:
+            # case 1: the active sequence continues
             if j_t > self.j:
-                self.x_recon = (0, j_t)
+                self.x_recon = x_static
                 self.j = j_t
-            return "continue", self.primary
-        # case 2: reconciliation
-        if k_t > self.k:
+            return "continue", self.primary, x_static + x_dyn
+        if k_t == self.k + 1:
+            # case 2: a state of the sequence the secondary is rebuilding
+            if self.j_eps is None:
+                self.j_eps = j_eps_t
             if k_t > self.k_ready:
-                # the secondary has not finished: bridge the new chunks on the primary
-                delta = (self.j_eps, j_t)
+                # not rebuilt yet: serve it on the primary, on the active
+                # sequence extended with the chunks that are new since the cursor
+                if self.j_eps is None or not 0 <= self.j_eps <= j_t:
+                    raise ValueError("bridged range must run forward from the eviction cursor")
+                delta = x_static[self.j_eps:j_t]
+                self.x_recon = self.x_recon + delta
                 self.buffer.append(delta)
                 self.j_eps = j_t
-                return "bridge", self.primary
-            if k_t == self.k_ready:
-                # the secondary has finished: resource swap
-                self.primary, self.secondary = self.secondary, self.primary
-                self.is_reconciling = False
-                self.x_recon = (0, j_t)
-                self.j, self.k, self.j_eps = j_t, k_t, None
-                return "swap", self.primary
-        # case 3: straggler queries
-        if self.is_reconciling:
-            return "straggler_primary", self.primary
-        return "straggler_secondary", self.secondary
-
+                return "bridge", self.primary, self.x_recon + x_dyn
+            # k_t == k_ready: the secondary holds the rebuilt cache -> swap
+            self.primary, self.secondary = self.secondary, self.primary
+            self.is_reconciling = False
+            self.x_recon = x_static
+            self.j, self.k, self.j_eps = j_t, k_t, None
+            return "swap", self.primary, x_static + x_dyn
+        if k_t < self.k:
+            # case 3: a straggler built on an older version
+            if self.is_reconciling:
+                # the secondary is being rebuilt: stitch the query onto x_recon
+                return "straggler_primary", self.primary, self.x_recon + x_dyn
+            return "straggler_secondary", self.secondary, x_static + x_dyn
+        raise ValueError("query version is ahead of the sequence being rebuilt")

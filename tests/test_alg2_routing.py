@@ -19,15 +19,27 @@ def run_hand_trace(orc):
     r = orc.Alg2Router()
     for ev in g["events"]:
         if ev["op"] == "reconcile_start":
-            r.reconcile_start(ev["k_target"])
+            r.reconcile_start(ev["x_eps"], ev["k_target"])
+        elif ev["op"] == "catch_up":
+            assert r.catch_up() == ev["expect_taken"], ev
+            assert r.x_eps == ev["x_eps"], ev
         elif ev["op"] == "reconcile_done":
             r.reconcile_done(ev["k_target"])
+        elif ev.get("expect_error"):
+            try:
+                r.inference(ev["x_static"], ev["x_dyn"], ev["k_t"], ev["j_eps_t"])
+            except ValueError:
+                pass
+            else:
+                raise AssertionError(f"query not rejected: {ev}")
         else:
-            got = r.inference(ev["j_t"], ev["k_t"], ev["j_eps_t"])
+            got = r.inference(ev["x_static"], ev["x_dyn"], ev["k_t"], ev["j_eps_t"])
             assert list(got) == ev["expect"], ev
             assert (r.k, r.k_ready) == (ev["k"], ev["k_ready"]), ev
             assert (r.j, r.j_eps) == (ev["j"], ev["j_eps"]), ev
-            assert [list(x) for x in r.buffer] == ev["buffer"], ev
+            assert r.x_recon == ev["x_recon"], ev
+            assert list(r.buffer) == ev["buffer"], ev
+            assert r.is_reconciling == ev["is_reconciling"], ev
 
 
 def test_oracle_router_matches_hand_trace():
@@ -84,11 +96,11 @@ def test_library_routes_match_oracle_router(libcsr, after_swap, state, dk):
     if after_swap:                                   # bring both to version 1
         ctx.evict_and_reconcile(16)
         assert ctx.wait_reconcile(5.0) == libcsr.RECON_SWAPPED
-        r.reconcile_start(1), r.reconcile_done(1), r.inference(50, 1, 50)
+        r.reconcile_start("ab", 1), r.reconcile_done(1), r.inference("abc", "?", 1, 2)
         k = 1
     if state != "idle":
         ctx.evict_and_reconcile(16)
-        r.reconcile_start(k + 1)
+        r.reconcile_start("ab", k + 1)
         if state == "rebuilding":
             for _ in range(2):
                 ctx.append_chunk(None, None, None, n=16)
@@ -103,5 +115,60 @@ def test_library_routes_match_oracle_router(libcsr, after_swap, state, dk):
         with pytest.raises(libcsr.CsrError):
             ctx.route(k_t)
         return
-    case, _ = r.inference(100, k_t, 100)
+    case, _, _ = r.inference("abcd", "?", k_t, 2 if k_t > k else None)
     assert ctx.route(k_t) == getattr(libcsr, _CASE[case])
+
+
+def test_router_invariants_on_random_sessions():
+    """Properties that hold for any interleaving the clients can produce
+    (Algorithm 2): the bridged context is always the active sequence's static
+    state followed by every chunk bridged since the eviction, in order; the
+    secondary's state plus the buffered chunks is the rebuilt sequence up to
+    the cursor; and the swap query's static state starts with what the
+    secondary computed (only the remainder is computed at the swap)."""
+    import random
+    rng = random.Random(7)
+    import itertools
+    letters = (chr(0x4E00 + i) for i in itertools.count())   # a distinct character per chunk
+    for trial in range(200):
+        r = orc.Alg2Router()
+        active = "ab" + "".join(next(letters) for _ in range(4))   # the active static state
+        r.inference(active, "?", 0)
+        k = 0
+        rebuilt = None            # the static state of version k + 1, once evicted
+        old = None                # old chunks kept by the eviction
+        bridged = ""
+        done = False              # Reconcile has authorised the swap
+        for step in range(30):
+            a = rng.random()
+            if rebuilt is None and a < 0.2:
+                keep = rng.randrange(2, len(active))
+                old = active[:2] + active[keep:]
+                rebuilt, bridged, done = old, "", False
+                r.reconcile_start(old, k + 1)
+            elif rebuilt is not None and a < 0.5:
+                rebuilt += "".join(next(letters) for _ in range(rng.randrange(0, 3)))
+                case, res, ctx = r.inference(rebuilt, "?", k + 1, len(old))
+                if case == "bridge":
+                    bridged = rebuilt[len(old):]
+                    assert ctx == active + bridged + "?"
+                    assert r.x_recon == active + bridged
+                    assert not done and r.x_eps + "".join(r.buffer) == rebuilt[:r.j_eps]
+                else:
+                    assert done and case == "swap" and rebuilt.startswith(r.x_eps)
+                    active, rebuilt, k = rebuilt, None, k + 1
+            elif rebuilt is not None and not done and a < 0.6:
+                r.catch_up()
+                assert r.x_eps + "".join(r.buffer) == (rebuilt[:r.j_eps] if r.j_eps else old)
+            elif rebuilt is not None and not done and a < 0.7:
+                r.reconcile_done(k + 1)
+                done = True
+            elif rebuilt is None and a < 0.8:
+                active += next(letters)
+                assert r.inference(active, "?", k)[0] == "continue"
+            elif k > 0:
+                case, res, ctx = r.inference("stale", "?", k - 1)
+                if r.is_reconciling:
+                    assert (case, res, ctx) == ("straggler_primary", r.primary, r.x_recon + "?")
+                else:
+                    assert (case, res, ctx) == ("straggler_secondary", r.secondary, "stale?")

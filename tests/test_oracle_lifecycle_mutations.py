@@ -87,22 +87,41 @@ OracleCSR.sources_pos0 = _sources_pos0
 ROUTER_MUTATIONS = {
     # the swap does not exchange the primary and secondary resources
     "router_no_resource_exchange": (
-        "                self.primary, self.secondary = self.secondary, self.primary\n", ""),
+        "            self.primary, self.secondary = self.secondary, self.primary\n", ""),
     # the bridge condition is off by one version (queries of the rebuilt
-    # version that must be bridged fall through to the straggler case)
+    # version that must be bridged are swapped in too early)
     "router_bridge_condition_shifted": ("            if k_t > self.k_ready:",
-                                        "            if k_t > self.k_ready + 1:"),
+                                        "            if k_t > self.k_ready - 1:"),
     # the eviction cursor is not advanced after a bridged query
     "router_cursor_not_advanced": ("                self.j_eps = j_t\n                return \"bridge\"",
                                    "                return \"bridge\""),
+    # the cursor is taken from whichever query comes first after the eviction
+    # (the active version's own length included)
+    "router_cursor_set_by_any_query": ("        j_t = len(x_static)\n",
+                                       "        j_t = len(x_static)\n"
+                                       "        if self.j_eps is None:\n            self.j_eps = j_eps_t\n"),
+    # a bridged query does not extend the reconciliation state
+    "router_bridge_drops_recon_extension": ("                self.x_recon = self.x_recon + delta\n", ""),
+    # a bridged chunk is not buffered for the catch-up
+    "router_bridge_not_buffered": ("                self.buffer.append(delta)\n", ""),
     # stragglers while reconciling go to the secondary (the cache being rebuilt)
-    "router_straggler_to_secondary": ('            return "straggler_primary", self.primary',
-                                      '            return "straggler_primary", self.secondary'),
+    "router_straggler_to_secondary": (
+        '                return "straggler_primary", self.primary, self.x_recon + x_dyn',
+        '                return "straggler_primary", self.secondary, self.x_recon + x_dyn'),
+    # stragglers while reconciling keep their own stale static state
+    "router_straggler_not_stitched": (
+        '                return "straggler_primary", self.primary, self.x_recon + x_dyn',
+        '                return "straggler_primary", self.primary, x_static + x_dyn'),
+    # case 3 reached by falling through instead of by k_t < k
+    "router_case3_unguarded": ("        if k_t < self.k:\n", "        if True:\n"),
     # Reconcile never authorises the swap
     "router_no_k_ready": ("        self.k_ready = k_target\n", "        pass\n"),
     # a continuation does not advance the active length
-    "router_continuation_keeps_j": ("                self.x_recon = (0, j_t)\n                self.j = j_t\n",
-                                    "                self.x_recon = (0, j_t)\n"),
+    "router_continuation_keeps_j": ("                self.x_recon = x_static\n                self.j = j_t\n",
+                                    "                self.x_recon = x_static\n"),
+    # the catch-up hands the buffer to the secondary but keeps it buffered
+    "router_catch_up_keeps_buffer": ("        taken = \"\".join(self.buffer)\n        self.buffer = []\n",
+                                     "        taken = \"\".join(self.buffer)\n"),
 }
 
 
