@@ -307,6 +307,50 @@ csr_status csr_route(csr_ctx *ctx, int64_t k_t, csr_stream_t fg_stream, int *rou
  */
 csr_status csr_cancel_reconcile(csr_ctx *ctx);
 
+/* Result of csr_check_viability (times in seconds, sizes in tokens). */
+typedef struct csr_viability {
+  double t_warm_s;        /* Delta t_warm: warm-up of the evicted state */
+  double delta_n_tokens;  /* Delta N = append rate * Delta t_warm */
+  double t_recon_s;       /* Delta t_recon: extension of the rebuilt state by Delta N */
+  double t_mem_s;         /* Delta t_mem = N_buffer / append rate */
+  double n_buffer_tokens; /* N_buffer: tokens that fit before the page pool runs out */
+  double rebuilt_tokens;  /* |T^E|: length of the evicted state (prefix + retained chunks) */
+  double pair_seconds;    /* time of one query-key pair of the rebuild that was used */
+  int32_t viable;         /* 1 when Delta t_warm + Delta t_recon <= Delta t_mem */
+  int32_t measured;       /* 1 when pair_seconds was observed on this context */
+} csr_viability;
+
+/*
+ * Viability of the asynchronous reconciliation (App. D, Eq. recon_time_inequlity
+ * Delta t_warm + Delta t_recon <= Delta t_mem, with Eqs. warm-up_time, recon_time
+ * and oom_time): would an eviction of evict_tokens started now (the same
+ * chunks csr_evict_and_reconcile would drop) finish its rebuild and catch-up
+ * before the page pool is exhausted, at append_tokens_per_s new tokens per
+ * second?  With c the time of one query-key pair of the rebuild and
+ * |T^E| = prefix + retained chunk tokens:
+ *   Delta t_warm  = c * sum_{i = |X_pre|+1}^{|T^E|} i   (Eq. TTFT_derivation_2: the
+ *                   retained chunks are prefilled over the prefix and themselves;
+ *                   the prefix is not recomputed)
+ *   Delta N       = append_tokens_per_s * Delta t_warm
+ *   Delta t_recon = c * Delta N (2 |T^E| + Delta N + 1) / 2        (Eq. recon_time)
+ *   Delta t_mem   = N_buffer / append_tokens_per_s                 (Eq. oom_time)
+ * N_buffer is the largest number of tokens x such that the pages both
+ * versions need for x more tokens fit in the pool's free pages once the
+ * rebuilt version is reserved (while a reconciliation runs an appended chunk
+ * takes pages in both), capped by max_seq_tokens.  The paper's two resources
+ * give N_max - |T_t|; here one pool holds both versions.
+ * c = pair_seconds when > 0; otherwise the value observed on this context's
+ * last completed reconciliation (device time from the eviction to the end of
+ * its last catch-up on the low-priority stream, the foreground running
+ * alongside, divided by the query-key pairs it computed).  Host-only; nothing
+ * changes.  CSR_EINVAL for evict_tokens < 1, append_tokens_per_s <= 0 or a
+ * NULL out; CSR_ESTATE with a live suffix, while a reconciliation runs, with
+ * no chunk to evict, or with pair_seconds <= 0 before any reconciliation has
+ * completed.
+ */
+csr_status csr_check_viability(csr_ctx *ctx, int32_t evict_tokens, double append_tokens_per_s,
+                               double pair_seconds, csr_viability *out);
+
 /* Which version an inspection call reads. */
 #define CSR_VERSION_ACTIVE 0
 #define CSR_VERSION_PENDING 1

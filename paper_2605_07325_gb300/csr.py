@@ -64,6 +64,14 @@ class Timing(ctypes.Structure):
     _fields_ = [("ms", ctypes.c_double * 4), ("launches", ctypes.c_int64 * 4)]
 
 
+class Viability(ctypes.Structure):
+    _fields_ = [("t_warm_s", ctypes.c_double), ("delta_n_tokens", ctypes.c_double),
+                ("t_recon_s", ctypes.c_double), ("t_mem_s", ctypes.c_double),
+                ("n_buffer_tokens", ctypes.c_double), ("rebuilt_tokens", ctypes.c_double),
+                ("pair_seconds", ctypes.c_double), ("viable", ctypes.c_int32),
+                ("measured", ctypes.c_int32)]
+
+
 PROVIDER = ctypes.CFUNCTYPE(ctypes.c_int, ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32,
                             ctypes.POINTER(ctypes.c_void_p), ctypes.POINTER(ctypes.c_void_p),
                             ctypes.POINTER(ctypes.c_void_p), ctypes.POINTER(ctypes.c_void_p))
@@ -82,6 +90,8 @@ _SIGS = {
                                        ctypes.c_int),
     "csr_get_versions": ([_vp, _P64, _P64], ctypes.c_int),
     "csr_cancel_reconcile": ([_vp], ctypes.c_int),
+    "csr_check_viability": ([_vp, _i32, ctypes.c_double, ctypes.c_double, ctypes.POINTER(Viability)],
+                            ctypes.c_int),
     "csr_route": ([_vp, ctypes.c_int64, _vp, ctypes.POINTER(ctypes.c_int)], ctypes.c_int),
     "csr_attend_suffix": ([_vp, _vp, _vp, _vp, _i32, _vp, _vp, _vp], ctypes.c_int),
     "csr_truncate_suffix": ([_vp], ctypes.c_int),
@@ -285,6 +295,15 @@ class Context:
         """Abandon the running reconciliation; the active version stays."""
         self._check(_lib.csr_cancel_reconcile(self._h))
         self._keep.clear()
+
+    def check_viability(self, evict_tokens: int, append_tokens_per_s: float,
+                        pair_seconds: float = 0.0) -> Dict[str, float]:
+        """App. D viability of an eviction of evict_tokens started now
+        (csr_check_viability); pair_seconds <= 0 uses the observed rebuild pace."""
+        v = Viability()
+        self._check(_lib.csr_check_viability(self._h, int(evict_tokens), float(append_tokens_per_s),
+                                             float(pair_seconds), ctypes.byref(v)))
+        return {name: getattr(v, name) for name, _ in Viability._fields_}
 
     def versions(self) -> Tuple[int, int]:
         """(k, k_ready) of Algorithm 2."""

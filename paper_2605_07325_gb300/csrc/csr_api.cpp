@@ -257,6 +257,14 @@ struct csr_ctx {
   void *user = nullptr;
   cudaStream_t lo = nullptr;
   cudaEvent_t ev_fg = nullptr, ev_rb = nullptr;
+  // Observed pace of the rebuild (App. D viability check): timing events at
+  // the start of a reconciliation and after each of its tasks on the
+  // low-priority stream, the query-key pairs enqueued there, and the result of
+  // the last completed reconciliation.
+  cudaEvent_t ev_rb_t0 = nullptr, ev_rb_t1 = nullptr;
+  std::atomic<int64_t> rb_pairs{0};
+  bool rb_timed = false;           // rb_pair_seconds holds an observation
+  double rb_pair_seconds = 0.0;
   std::atomic<int64_t> launches{0};
   std::string err = "no error";
   Reconciler rw;
@@ -599,7 +607,8 @@ void worker_main(csr_ctx *c) {
         st = rebuild_chunk(c, t.ch, t.pos, t.ids, t.first_lp, 1, c->lo);
       }
       if (st == CSR_OK) {
-        const cudaError_t e = cudaEventRecord(c->ev_rb, c->lo);
+        cudaError_t e = cudaEventRecord(c->ev_rb, c->lo);
+        if (e == cudaSuccess) e = cudaEventRecord(c->ev_rb_t1, c->lo);
         if (e != cudaSuccess) st = cuda_fail(c, e, "recording the rebuild event");
       }
     }
@@ -646,6 +655,8 @@ void push_task(csr_ctx *c, ReconTask t) {
 // write_ids: K1 writes the chunk's page ids (pages reserved after the
 // compaction ran) into the device table.
 void push_chunk_task(csr_ctx *c, ChunkRec ch, int64_t pos, bool write_ids) {
+  // query-key pairs of the causal prefill of ch.len tokens at positions pos..
+  c->rb_pairs += static_cast<int64_t>(ch.len) * pos + static_cast<int64_t>(ch.len) * (ch.len + 1) / 2;
   ReconTask t;
   t.ch = ch;
   t.pos = pos;
@@ -759,9 +770,13 @@ csr_status csr_create(const csr_config *cfg, void *k_pool, void *v_pool, void *w
     if (e == cudaSuccess) e = cudaMemsetAsync(workspace, 0, c->lay.total, s);
     if (e == cudaSuccess) e = cudaEventCreateWithFlags(&c->ev_fg, cudaEventDisableTiming);
     if (e == cudaSuccess) e = cudaEventCreateWithFlags(&c->ev_rb, cudaEventDisableTiming);
+    if (e == cudaSuccess) e = cudaEventCreate(&c->ev_rb_t0);
+    if (e == cudaSuccess) e = cudaEventCreate(&c->ev_rb_t1);
     if (e != cudaSuccess) {
       if (c->ev_fg) cudaEventDestroy(c->ev_fg);
       if (c->ev_rb) cudaEventDestroy(c->ev_rb);
+      if (c->ev_rb_t0) cudaEventDestroy(c->ev_rb_t0);
+      if (c->ev_rb_t1) cudaEventDestroy(c->ev_rb_t1);
       delete c;
       return CSR_ECUDA;
     }
@@ -778,6 +793,8 @@ void csr_destroy(csr_ctx *c) {
     cudaDeviceSynchronize();
     if (c->ev_fg) cudaEventDestroy(c->ev_fg);
     if (c->ev_rb) cudaEventDestroy(c->ev_rb);
+    if (c->ev_rb_t0) cudaEventDestroy(c->ev_rb_t0);
+    if (c->ev_rb_t1) cudaEventDestroy(c->ev_rb_t1);
     for (auto &t : c->timed) {
       cudaEventDestroy(t.a);
       cudaEventDestroy(t.b);
@@ -943,10 +960,12 @@ csr_status csr_evict_and_reconcile(csr_ctx *c, int32_t evict_tokens, csr_stream_
   c->reconciling = true;
   c->buffer.clear();
   c->ids_checked = c->plan_only;
+  c->rb_pairs = 0;
   if (c->plan_only) return CSR_OK;
   const cudaStream_t fg = reinterpret_cast<cudaStream_t>(fg_stream);
   cudaError_t e = cudaEventRecord(c->ev_fg, fg);
   if (e == cudaSuccess) e = cudaStreamWaitEvent(c->lo, c->ev_fg, 0);
+  if (e == cudaSuccess) e = cudaEventRecord(c->ev_rb_t0, c->lo);
   if (e != cudaSuccess) {
     delete ep;
     abort_reconcile(c);
@@ -1037,6 +1056,14 @@ csr_status reconcile_progress(csr_ctx *c, csr_stream_t fg_stream, bool *ready) {
     }
     return CSR_OK;
   }
+  if (!c->plan_only && c->rb_pairs > 0) {
+    // Everything handed to R_2 so far has finished: its observed time per pair.
+    float ms = 0.f;
+    if (cudaEventElapsedTime(&ms, c->ev_rb_t0, c->ev_rb_t1) == cudaSuccess && ms > 0.f) {
+      c->rb_pair_seconds = 1e-3 * ms / static_cast<double>(c->rb_pairs.load());
+      c->rb_timed = true;
+    }
+  }
   *ready = true;
   return CSR_OK;
 }
@@ -1092,6 +1119,66 @@ csr_status csr_poll_swap(csr_ctx *c, csr_stream_t fg_stream, int *state) {
   st = reconcile_swap(c, fg_stream);
   if (st == CSR_OK) *state = CSR_RECON_SWAPPED;
   return st;
+}
+
+csr_status csr_check_viability(csr_ctx *c, int32_t evict_tokens, double append_tokens_per_s,
+                               double pair_seconds, csr_viability *out) {
+  if (!c || !out) return CSR_EINVAL;
+  if (evict_tokens < 1 || !(append_tokens_per_s > 0.0))
+    return fail(c, CSR_EINVAL, "evict_tokens must be >= 1 and the append rate > 0");
+  if (c->reconciling) return fail(c, CSR_ESTATE, "a reconciliation is running");
+  const Version &A = c->act();
+  if (A.suffix_len > 0) return fail(c, CSR_ESTATE, "a suffix is live");
+  if (A.chunks.empty()) return fail(c, CSR_ESTATE, "no chunk to evict");
+  double cp = pair_seconds;
+  int32_t measured = 0;
+  if (!(cp > 0.0)) {
+    if (!c->rb_timed) return fail(c, CSR_ESTATE, "no reconciliation has been observed yet");
+    cp = c->rb_pair_seconds;
+    measured = 1;
+  }
+  // The chunks csr_evict_and_reconcile would drop (Eq. eviction_operation).
+  size_t k = 0;
+  int64_t dropped = 0;
+  while (k < A.chunks.size() && dropped < evict_tokens) dropped += A.chunks[k++].len;
+  int64_t rebuilt = A.prefix_len;
+  for (size_t i = k; i < A.chunks.size(); ++i) rebuilt += A.chunks[i].len;
+  const int64_t active = A.length();
+  const int P = c->cfg.page_size;
+  const int64_t full = A.prefix_len / P;
+  const int64_t fresh = pages_for(c, rebuilt) - full;
+  const int64_t spare = static_cast<int64_t>(c->pool.n_free) - fresh;
+  // N_buffer: the most tokens x for which both versions' new pages fit (Eq. oom_time).
+  auto need = [&](int64_t x) {
+    return (pages_for(c, active + x) - pages_for(c, active)) + (pages_for(c, rebuilt + x) - pages_for(c, rebuilt));
+  };
+  int64_t n_buffer = 0;
+  if (spare > 0) {
+    int64_t lo = 0, hi = std::max<int64_t>(0, static_cast<int64_t>(c->cfg.max_seq_tokens) - active);
+    while (lo < hi) {
+      const int64_t mid = lo + (hi - lo + 1) / 2;
+      if (need(mid) <= spare) lo = mid;
+      else hi = mid - 1;
+    }
+    n_buffer = lo;
+  }
+  const double E = static_cast<double>(rebuilt);
+  const double pre = static_cast<double>(A.prefix_len);
+  // Eq. warm-up_time through Eq. TTFT_derivation_2 with i* = |X_pre| + 1.
+  const double t_warm = cp * (E - pre) * (E + pre + 1.0) / 2.0;
+  const double dN = append_tokens_per_s * t_warm;
+  const double t_recon = cp * dN * (2.0 * E + dN + 1.0) / 2.0;   // Eq. recon_time
+  const double t_mem = static_cast<double>(n_buffer) / append_tokens_per_s;  // Eq. oom_time
+  out->t_warm_s = t_warm;
+  out->delta_n_tokens = dN;
+  out->t_recon_s = t_recon;
+  out->t_mem_s = t_mem;
+  out->n_buffer_tokens = static_cast<double>(n_buffer);
+  out->rebuilt_tokens = E;
+  out->pair_seconds = cp;
+  out->viable = (t_warm + t_recon <= t_mem) ? 1 : 0;   // Eq. recon_time_inequlity
+  out->measured = measured;
+  return CSR_OK;
 }
 
 csr_status csr_get_versions(csr_ctx *c, int64_t *k, int64_t *k_ready) {
