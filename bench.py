@@ -254,8 +254,6 @@ def run_ours(args):
     pool_pages = math.ceil(max_tokens / P) + 16
     cfg = csr.make_config(HQ, HKV, D, P, BASE, max_new_tokens=PREFIX, pool_pages=pool_pages,
                           max_seq_tokens=max_tokens + P,
-                          flags={"pair": 0, "pipe": csr.FLAG_PIPE_64,
-                                 "single": csr.FLAG_SINGLE_TILE}[args.kernel],
                           fg_chunk_tiles=args.fg_chunk_tiles)
     stream = torch.cuda.Stream(device=dev, priority=-1)
     gen = torch.Generator(device=dev).manual_seed(1234 + rank)
@@ -424,16 +422,16 @@ def run_ours(args):
                    "replicas": world, "replica_us_per_step": us_step,
                    "foreground_ctas": ctx.cfg.num_ctas or props.multi_processor_count,
                    "kernel_events": "the timed region records a CUDA event pair around every kernel "
-                                    "launch (roofline.achieved); the events sit between launches the "
-                                    "library otherwise chains with programmatic dependent launch, so "
-                                    "value includes their cost and the e2e region, run without them, "
-                                    "can read lower"},
+                                    "launch (roofline.achieved); a call is one launch, so the events "
+                                    "sit between consecutive calls, which the library otherwise "
+                                    "chains with programmatic dependent launch; value includes their "
+                                    "cost and the e2e region, run without them, can read lower"},
         "roofline": {"bound": "tensor", "achieved": achieved, "peak": peak_burst, "unit": "TFLOP/s",
                      "frac": (achieved / peak_burst) if achieved else None,
                      "traffic": traffic,
-                     "kernel": {"pipe": "attn_pipe_kernel<128>", "pair": "attn_pair_kernel<128>",
-                                "single": "attn_kernel<128>"}[args.kernel] +
-                               " (tcgen05 QK^T and PV, TMA paged K/V)",
+                     "kernel": "attn_pair_kernel<128, true>: the whole call in one cooperative "
+                               "launch (RoPE + paged append, tcgen05 QK^T and PV over TMA-staged "
+                               "paged K/V, merge of split pieces after a grid barrier)",
                      "launches": att_n, "avg_launch_us": att_ms / max(1, att_n) * 1e3,
                      "peak_source": f"bf16_tflops ({peak_kind}, burst)",
                      "frac_of_sustained": (achieved / peak_sust) if achieved else None},
@@ -804,10 +802,6 @@ def main(argv=None):
                          "csr_attend_suffix) or fused (csr_append_chunk_attend_suffix, one pass)")
     ap.add_argument("--fg-chunk-tiles", type=int, default=0,
                     help="key tiles per attention work item (0: the library's cost model)")
-    ap.add_argument("--kernel", choices=["pair", "pipe", "single"], default="pair",
-                    help="attention kernel: pair (default: two query tiles per CTA, 128-key "
-                         "tiles), pipe (two query tiles, 64-key tiles, two score buffers each), "
-                         "single (one query tile per CTA)")
     ap.add_argument("--fill-chunk", type=int, default=CHUNK, choices=[256, 512, 1024, 2048, 4096],
                     help="chunk size used to fill the cache before timing (fewer launches "
                          "for profiler captures); the timed steps are unchanged")

@@ -72,11 +72,6 @@ typedef enum csr_status {
 #define CSR_FLAG_PLAN_ONLY 0x1   /* layout planning only: no device memory is touched
                                     and no kernel runs; compute calls update the page
                                     tables and lengths but produce no outputs */
-#define CSR_FLAG_SINGLE_TILE 0x2 /* attention CTAs own one 128-row query tile, 128-key tiles
-                                    (the first kernel design, kept for comparison) */
-#define CSR_FLAG_PIPE_64 0x4     /* two query tiles per CTA with 64-key tiles and two score
-                                    buffers each (an experimental third design); the default
-                                    uses 128-key tiles and one score buffer per query tile */
 
 typedef struct csr_config {
   int32_t num_q_heads;    /* H_q */
@@ -91,11 +86,14 @@ typedef struct csr_config {
   int32_t cap_tokens;     /* tau_mem of Algorithm 1; 0 disables automatic eviction */
   int32_t evict_tokens;   /* tokens of the oldest chunks dropped by an automatic eviction */
   int32_t n_catchup;      /* N_catchup of Algorithm 1 */
-  int32_t num_ctas;       /* CTAs of a foreground attention launch; 0 = one per SM */
+  int32_t num_ctas;       /* CTAs of a foreground attention launch (at most one per SM);
+                             0 = one per SM */
   int32_t rebuild_tiles_per_cta; /* key tiles (128 keys) per CTA in rebuild launches; 0 = 16 */
   int32_t flags;          /* CSR_FLAG_* */
-  int32_t fg_chunk_tiles; /* key tiles per split-KV item of a foreground launch; 0 = chosen
-                             per launch from its shape */
+  int32_t fg_chunk_tiles; /* > 0: a foreground launch splits every unit's key range into
+                             chunks of this many 128-key tiles (more if the split partials
+                             would not fit), dealt round-robin to its CTAs; 0 = whole units
+                             in rounds and only the leftover units split (the default) */
 } csr_config;
 
 /*
@@ -396,6 +394,28 @@ csr_status csr_device_status(csr_ctx *ctx, uint32_t *flags);
 
 /* Number of kernels the context has launched since creation. */
 int64_t csr_kernel_launches(const csr_ctx *ctx);
+
+/* One piece of a foreground launch's schedule (csr_foreground_schedule). */
+typedef struct csr_piece {
+  int32_t cta;    /* CTA that runs it */
+  int32_t order;  /* its position in that CTA's sequence */
+  int32_t unit;   /* pair * num_kv_heads + kv head; a pair is query tiles 2p, 2p+1 of
+                     128 packed rows (tokens x group heads) */
+  int32_t j0, j1; /* key tiles [j0, j1) of 128 keys */
+  int32_t slot;   /* partial-output slot, or -1 when the piece is the whole unit */
+} csr_piece;
+
+/*
+ * Inspection: the pieces a foreground call of n new tokens over L cached
+ * tokens runs, for a configuration and a CTA count (0 = one per SM of the
+ * current device; a plan-only configuration needs grid > 0).  Host-only.
+ * pieces may be NULL to count; *n_slots receives the partial slots merged
+ * after the grid barrier (0: the launch merges nothing).  CSR_EINVAL for a bad
+ * configuration or sizes, CSR_ENOMEM if capacity is too small.
+ */
+csr_status csr_foreground_schedule(const csr_config *cfg, int64_t L, int32_t n, int32_t grid,
+                                   csr_piece *pieces, int32_t capacity, int32_t *count,
+                                   int32_t *n_slots);
 
 /* Kernel kinds of csr_timing. */
 #define CSR_KERNEL_ROPE_APPEND 0

@@ -29,8 +29,6 @@ STATUS_NAMES = {0: "CSR_OK", 1: "CSR_EINVAL", 2: "CSR_ENOMEM", 3: "CSR_ESTATE", 
                 5: "CSR_ECUDA", 6: "CSR_ETIMEOUT", 7: "CSR_EDEVICE"}
 DEVERR_WAIT_TIMEOUT, DEVERR_BAD_PAGE, DEVERR_ALLOC = 0x1, 0x2, 0x4
 FLAG_PLAN_ONLY = 0x1
-FLAG_SINGLE_TILE = 0x2
-FLAG_PIPE_64 = 0x4
 RECON_IDLE, RECON_RUNNING, RECON_SWAPPED = 0, 1, 2
 ROUTE_CONTINUE, ROUTE_BRIDGE, ROUTE_SWAPPED, ROUTE_STRAGGLER = 0, 1, 2, 3
 VERSION_ACTIVE, VERSION_PENDING = 0, 1
@@ -64,6 +62,11 @@ class Timing(ctypes.Structure):
     _fields_ = [("ms", ctypes.c_double * 4), ("launches", ctypes.c_int64 * 4)]
 
 
+class Piece(ctypes.Structure):
+    _fields_ = [("cta", ctypes.c_int32), ("order", ctypes.c_int32), ("unit", ctypes.c_int32),
+                ("j0", ctypes.c_int32), ("j1", ctypes.c_int32), ("slot", ctypes.c_int32)]
+
+
 class Viability(ctypes.Structure):
     _fields_ = [("t_warm_s", ctypes.c_double), ("delta_n_tokens", ctypes.c_double),
                 ("t_recon_s", ctypes.c_double), ("t_mem_s", ctypes.c_double),
@@ -90,6 +93,8 @@ _SIGS = {
                                        ctypes.c_int),
     "csr_get_versions": ([_vp, _P64, _P64], ctypes.c_int),
     "csr_cancel_reconcile": ([_vp], ctypes.c_int),
+    "csr_foreground_schedule": ([ctypes.POINTER(Config), _i64, _i32, _i32, ctypes.POINTER(Piece), _i32,
+                                 _P32, _P32], ctypes.c_int),
     "csr_check_viability": ([_vp, _i32, ctypes.c_double, ctypes.c_double, ctypes.POINTER(Viability)],
                             ctypes.c_int),
     "csr_route": ([_vp, ctypes.c_int64, _vp, ctypes.POINTER(ctypes.c_int)], ctypes.c_int),
@@ -130,6 +135,22 @@ def make_config(num_q_heads, num_kv_heads, head_dim, page_size, rope_base, max_n
     return Config(num_q_heads, num_kv_heads, head_dim, page_size, float(rope_base),
                   float(softmax_scale), max_new_tokens, pool_pages, max_seq_tokens, cap_tokens,
                   evict_tokens, n_catchup, num_ctas, rebuild_tiles_per_cta, flags, fg_chunk_tiles)
+
+
+def foreground_schedule(cfg: Config, L: int, n: int, grid: int = 0):
+    """Pieces (cta, order, unit, j0, j1, slot) of a foreground call of n tokens
+    over L cached, and the number of partial slots it merges."""
+    cnt, slots = ctypes.c_int32(0), ctypes.c_int32(0)
+    st = _lib.csr_foreground_schedule(ctypes.byref(cfg), int(L), int(n), int(grid), None, 0,
+                                      ctypes.byref(cnt), ctypes.byref(slots))
+    if st != 0:
+        raise CsrError(st, "csr_foreground_schedule failed")
+    arr = (Piece * max(1, cnt.value))()
+    st = _lib.csr_foreground_schedule(ctypes.byref(cfg), int(L), int(n), int(grid), arr, cnt.value,
+                                      ctypes.byref(cnt), ctypes.byref(slots))
+    if st != 0:
+        raise CsrError(st, "csr_foreground_schedule failed")
+    return [tuple(getattr(arr[i], f) for f, _ in Piece._fields_) for i in range(cnt.value)], slots.value
 
 
 def pool_bytes(cfg: Config) -> int:

@@ -4,8 +4,10 @@
 // the transient X_dyn suffix), the physical page pool (smallest free id
 // first), two cache versions (the active one and the one a reconciliation
 // rebuilds, Algorithm 1 / App. D), and the launch of the kernels:
-//   K1 rope_append  -> K2 attention (split over key chunks) -> K3 merge   per block
-//   K4 evict_compact                                                       per eviction
+//   foreground block:  one cooperative launch of the fused attention kernel
+//                      (RoPE + paged append, attention, merge of split pieces)
+//   rebuild block:     K1 rope_append -> K2 attention (short items) -> K3 merge
+//   eviction:          K4 evict_compact
 // The foreground runs on the caller's stream; the rebuild and its catch-up
 // run on the low-priority stream registered with csr_set_reconciler, fed by
 // the context's reconciliation thread (the host side of R_2).
@@ -42,7 +44,6 @@ struct Range {
   Range &operator=(const Range &) = delete;
 };
 
-constexpr int kFgGridDefaultCap = 304;   // 2 x 152 SMs
 constexpr int kPartialItems = 4096;      // split partials a launch may write (per staging)
 constexpr int kDefaultRebuildTiles = 16;
 constexpr size_t kAlign = 256;
@@ -138,8 +139,8 @@ bool encode_rows(CUtensorMap *m, void *base, uint64_t rows, uint64_t d, uint32_t
 }
 
 struct Layout {  // workspace carve-out (byte offsets)
-  size_t qpack[2], rb_out, part_o[2], part_lse[2], pt[2], ids_out, err, total;
-  int32_t rows_cap, fg_cap, max_pages;
+  size_t qpack[2], rb_out, part_o[2], part_lse[2], pt[2], ids_out, err, sync, total;
+  int32_t rows_cap, max_pages;
 };
 
 bool valid_config(const csr_config *c, std::string *why) {
@@ -162,7 +163,8 @@ bool valid_config(const csr_config *c, std::string *why) {
     return bad("max_new_tokens / page_size too large for one launch");
   if (c->pool_pages < 1 || c->pool_pages > 32 * kMaxPoolWords)
     return bad("pool_pages must be in [1, 65536]");
-  if (c->max_seq_tokens < 1) return bad("max_seq_tokens must be >= 1");
+  if (c->max_seq_tokens < 1 || c->max_seq_tokens > (1 << 24))
+    return bad("max_seq_tokens must be in [1, 2^24] (positions are exact fp32 integers in RoPE)");
   if (static_cast<int64_t>(c->pool_pages) * c->num_kv_heads * c->page_size >= (1ll << 31))
     return bad("pool rows exceed the 32-bit TMA coordinate range");
   if (c->cap_tokens < 0 || c->evict_tokens < 0 || c->n_catchup < 0 || c->num_ctas < 0 ||
@@ -177,7 +179,6 @@ Layout make_layout(const csr_config *c) {
   const int g = c->num_q_heads / c->num_kv_heads;
   // whole pairs of 128-row tiles, so the two-tile kernel never reads past a head's rows
   L.rows_cap = static_cast<int32_t>(align_up(static_cast<size_t>(c->max_new_tokens) * g, 2 * kBM));
-  L.fg_cap = c->num_ctas > 0 ? c->num_ctas : kFgGridDefaultCap;
   L.max_pages = static_cast<int32_t>(ceil_div(c->max_seq_tokens, c->page_size) + 1);
   const size_t d = static_cast<size_t>(c->head_dim);
   size_t off = 0;
@@ -195,6 +196,7 @@ Layout make_layout(const csr_config *c) {
   for (int i = 0; i < 2; ++i) L.pt[i] = take(static_cast<size_t>(L.max_pages) * 4);
   L.ids_out = take(static_cast<size_t>(L.max_pages) * 4);
   L.err = take(256);
+  L.sync = take(256);
   L.total = off;
   return L;
 }
@@ -234,7 +236,13 @@ struct csr_ctx {
   uint8_t *ws = nullptr;
   CUtensorMap tm_q[2]{}, tm_k{}, tm_v{};
   double inv_turns[kMaxHalfDim]{};
+  TurnSplit turns[kMaxHalfDim]{};     // inv_turns as fp32 hi + lo (rope.cuh)
   float scale_log2 = 0.f;
+  // Arrivals the fused foreground launches have made on the workspace's two
+  // device counters (every CTA adds one per launch; the merge barrier only in
+  // launches that merge), so the next launch knows its targets.
+  uint32_t step_append = 0, step_barrier = 0;
+  StepParams step{};                  // parameter block of the last fused launch
   PagePool pool;
   Version ver[2];
   std::atomic<int> active{0};
@@ -303,39 +311,128 @@ csr_status cuda_fail(csr_ctx *c, cudaError_t e, const char *where) {
 
 int64_t pages_for(const csr_ctx *c, int64_t len) { return ceil_div(len, c->cfg.page_size); }
 
-// Key chunks per unit for a launch of `units` query tiles whose longest key
-// range is kv_max tiles.  Foreground: minimise a time estimate over the
-// persistent grid: waves x (tiles per item x t_tile + per-item cost) plus the
-// split partials' write + merge read.  Rebuild (max_tiles > 0): the fewest
-// chunks of at most max_tiles tiles, so each CTA is short and a foreground
-// launch waits at most one item for an SM.  Never more than kPartialItems
-// items when split.
-int32_t choose_chunk_tiles(int64_t units, int64_t kv_max, int64_t grid, int max_tiles,
-                           int head_dim, int unit_tiles, int kv_tile) {
-  // us per key tile per CTA, per item, per split partial (rough GB300 figures)
-  const double t_tile = 0.75 * unit_tiles * kv_tile / kBN, t_item = 2.0;
-  const double t_part = (head_dim == 128 ? 0.02 : 0.01) * unit_tiles;
-  const int64_t cap_items = kPartialItems / unit_tiles;
+// Key chunks per pair for a rebuild launch of `units` pairs whose longest key
+// range is kv_max tiles: the fewest chunks of at most max_tiles tiles, so each
+// CTA is short and a foreground launch waits at most one item for an SM;
+// never more items than the partial buffer holds.
+int32_t choose_chunk_tiles(int64_t units, int64_t kv_max, int max_tiles) {
+  const int64_t cap_items = kPartialItems / 2;   // pair slots
   int64_t best_c = kv_max;
-  double best_t = 1e300;
   for (int64_t S = 1; S <= std::min<int64_t>(kv_max, 256); ++S) {
     const int64_t C = ceil_div(kv_max, S);
     const int64_t Se = ceil_div(kv_max, C);
-    const int64_t items = units * Se;
-    if (Se > 1 && items > cap_items) break;
-    if (max_tiles > 0) {
-      if (C <= max_tiles) return static_cast<int32_t>(C);
-      best_c = C;  // the smallest chunk that still fits the partial buffer
-      continue;
-    }
-    const int64_t waves = ceil_div(items, grid);
-    const double t = waves * (C * t_tile + t_item) + (Se > 1 ? items * t_part : 0.0);
-    if (t < best_t - 1e-9) {
-      best_t = t;
-      best_c = C;
-    }
+    if (Se > 1 && units * Se > cap_items) break;
+    if (C <= max_tiles) return static_cast<int32_t>(C);
+    best_c = C;  // the smallest chunk that still fits the partial buffer
   }
   return static_cast<int32_t>(best_c);
+}
+
+// Schedule of a fused foreground launch (StepSchedule) for a block of n tokens
+// at L: units u = pair * hkv + head, unit u reading key tiles [0, K(u)).
+// With forced_chunk > 0: round-robin chunks of that many tiles (more if the
+// partial buffer requires).  Otherwise whole units in rounds of `grid`, and
+// the units left over after the last full round cut into pieces level by
+// level: each level cuts its pieces into S parts (S chosen from an estimate
+// of the level's time -- part length plus a per-piece cost -- and of the time
+// the leftover would take spread over the grid), the first `grid` parts (in
+// part-major order, so concurrent parts cover the same key section of
+// different units) run at this level and the rest go to the next; the last
+// level runs whole what is left.  Pieces of a split unit get consecutive
+// partial slots.
+constexpr double kPieceCostTiles = 2.0;   // fixed cost of a piece, in key-tile times
+constexpr double kSlotCostTiles = 0.02;   // partial write + merge read per piece
+constexpr int64_t kMinPieceTiles = 2;
+
+void build_step_schedule(int64_t L, int32_t n, int T, int hkv, int32_t n_tiles, int grid_cap,
+                         int forced_chunk, StepSchedule &S) {
+  S = StepSchedule{};
+  for (int l = 0; l < kMaxTailLevels; ++l)
+    for (int c = 0; c < kMaxStepGrid; ++c) {
+      S.piece[l][c] = kNoPiece;
+      S.slot[l][c] = kSlotWhole;
+    }
+  const int32_t pairs = static_cast<int32_t>(ceil_div(n_tiles, 2));
+  const int32_t U = pairs * hkv;
+  auto K = [&](int32_t u) { return unit_iters(L, n, T, 2 * (u / hkv) + 1); };
+  S.n_units = U;
+  const int64_t kv_max = K(U - 1);
+  if (forced_chunk > 0 || U > 0xffff) {
+    S.chunked = 1;
+    const int64_t cap_chunks = std::max<int64_t>(1, (kPartialItems / 2) / U);
+    const int64_t chunk = std::max<int64_t>(std::max(forced_chunk, 1), ceil_div(kv_max, cap_chunks));
+    const int64_t n_chunks = ceil_div(kv_max, chunk);
+    S.chunk_tiles = static_cast<int32_t>(chunk);
+    S.n_items = static_cast<int32_t>(n_chunks * U);
+    S.grid = static_cast<int32_t>(std::min<int64_t>(grid_cap, S.n_items));
+    S.n_slots = n_chunks > 1 ? S.n_items : 0;
+    return;
+  }
+  int64_t total = 0;
+  for (int32_t u = 0; u < U; ++u) total += K(u);
+  const int32_t grid = static_cast<int32_t>(std::max<int64_t>(1, std::min<int64_t>(grid_cap, total)));
+  S.grid = grid;
+  S.full_rounds = U / grid;
+  S.n_tail = U - S.full_rounds * grid;
+  struct Pc {
+    int32_t u;
+    int64_t a, b;
+  };
+  std::vector<Pc> pieces;
+  const int32_t first_tail = U - S.n_tail;
+  for (int32_t t = 0; t < S.n_tail; ++t) pieces.push_back({first_tail + t, 0, K(first_tail + t)});
+  std::vector<std::vector<std::pair<int, int>>> unit_pieces(S.n_tail);
+  int level = 0;
+  while (!pieces.empty()) {
+    const int64_t P = static_cast<int64_t>(pieces.size());
+    int64_t len_min = pieces[0].b - pieces[0].a;
+    double len_sum = 0;
+    for (const Pc &pc : pieces) {
+      len_min = std::min<int64_t>(len_min, pc.b - pc.a);
+      len_sum += static_cast<double>(pc.b - pc.a);
+    }
+    const double len = len_sum / static_cast<double>(P);
+    const bool last = level == kMaxTailLevels - 1;
+    const int64_t s_hi = last ? std::max<int64_t>(1, grid / P) : ceil_div(grid, P);
+    int64_t best_s = 1;
+    double best = 1e300;
+    for (int64_t sx = 1; sx <= s_hi; ++sx) {
+      if (sx > 1 && len_min / sx < kMinPieceTiles) break;
+      const int64_t tot = P * sx;
+      const double d = len / static_cast<double>(sx);
+      double cost = d + kPieceCostTiles + kSlotCostTiles * static_cast<double>(tot);
+      if (tot > grid) cost += static_cast<double>(tot - grid) * d / grid + kPieceCostTiles;
+      if (cost < best - 1e-9) {
+        best = cost;
+        best_s = sx;
+      }
+    }
+    std::vector<Pc> subs;
+    for (int64_t q = 0; q < best_s; ++q)
+      for (const Pc &pc : pieces) {
+        const int64_t len_p = pc.b - pc.a;
+        const int64_t a = pc.a + len_p * q / best_s, b = pc.a + len_p * (q + 1) / best_s;
+        if (b > a) subs.push_back({pc.u, a, b});
+      }
+    const int64_t take = std::min<int64_t>(static_cast<int64_t>(subs.size()), grid);
+    for (int64_t c = 0; c < take; ++c) {
+      const Pc &pc = subs[c];
+      S.piece[level][c] = static_cast<uint64_t>(pc.u) | (static_cast<uint64_t>(pc.a) << 16) |
+                          (static_cast<uint64_t>(pc.b) << 40);
+      unit_pieces[pc.u - first_tail].push_back({level, static_cast<int>(c)});
+    }
+    pieces.assign(subs.begin() + take, subs.end());
+    ++level;
+  }
+  S.levels = level;
+  int32_t next = 0;
+  for (int32_t t = 0; t < S.n_tail; ++t) {
+    S.tail_slot0[t] = static_cast<uint16_t>(next);
+    if (unit_pieces[t].size() > 1)
+      for (const auto &lc : unit_pieces[t]) S.slot[lc.first][lc.second] = static_cast<uint16_t>(next++);
+  }
+  S.tail_slot0[S.n_tail] = static_cast<uint16_t>(next);
+  S.n_slots = next;
 }
 
 cudaEvent_t take_event(csr_ctx *c) {
@@ -364,14 +461,67 @@ cudaError_t timed_launch(csr_ctx *c, int kind, bool foreground, cudaStream_t s, 
   return cudaSuccess;
 }
 
-// K1 -> K2 -> K3 for n tokens at positions L.. of version `slot`.
-// ws: 0 = foreground staging, 1 = rebuild staging.  ids/n_ids name the physical
-// pages of logical pages first_lp.. (written into the device table by K1);
+// Attend n new tokens at positions L.. of version `slot` (and append their
+// keys/values).  ws 0 (foreground, the caller's stream): one cooperative
+// launch of the fused kernel.  ws 1 (rebuild, the low-priority stream):
+// K1 -> K2 (short items) -> K3.  ids/n_ids name the physical pages of
+// logical pages first_lp.. (written into the device table by the launch);
 // n_ids == 0 reads the device table instead.
 csr_status run_block(csr_ctx *c, int slot, int ws, const void *q, const void *k, const void *v,
                      int32_t n, int64_t L, const int32_t *ids, int32_t n_ids, int32_t first_lp,
                      void *out, float *lse, cudaStream_t s) {
   const csr_config &cf = c->cfg;
+  const bool fg = ws == 0;
+  AttnParams ap{};
+  ap.tm_q = c->tm_q[ws];
+  ap.tm_k = c->tm_k;
+  ap.tm_v = c->tm_v;
+  ap.page_table = c->d_pt(slot);
+  ap.out = static_cast<uint16_t *>(out);
+  ap.lse = lse;
+  ap.part_o = c->wsp<float>(c->lay.part_o[ws]);
+  ap.part_lse = c->wsp<float>(c->lay.part_lse[ws]);
+  ap.err = c->wsp<uint32_t>(c->lay.err);
+  ap.L = L;
+  ap.n = n;
+  ap.hq = cf.num_q_heads;
+  ap.hkv = cf.num_kv_heads;
+  ap.group = c->group;
+  ap.page_size = cf.page_size;
+  ap.rows_cap = c->lay.rows_cap;
+  ap.n_tiles = static_cast<int32_t>(ceil_div(static_cast<int64_t>(n) * c->group, kBM));
+  ap.n_pages_valid = static_cast<int32_t>(pages_for(c, L + n));
+  ap.pool_pages = cf.pool_pages;
+  ap.scale_log2 = c->scale_log2;
+  const int T = kBM / c->group;
+
+  if (fg) {
+    StepParams &sp = c->step;
+    build_step_schedule(L, n, T, cf.num_kv_heads, ap.n_tiles, c->fg_grid, cf.fg_chunk_tiles, sp.s);
+    ap.grid = sp.s.grid;
+    sp.a = ap;
+    sp.q = static_cast<const uint16_t *>(q);
+    sp.k = static_cast<const uint16_t *>(k);
+    sp.v = static_cast<const uint16_t *>(v);
+    sp.k_pool = c->k_pool;
+    sp.v_pool = c->v_pool;
+    sp.sync = c->wsp<uint32_t>(c->lay.sync);
+    sp.append_target = c->step_append + static_cast<uint32_t>(sp.s.grid);
+    sp.barrier_target = c->step_barrier + static_cast<uint32_t>(sp.s.grid);
+    sp.first_lp = first_lp;
+    sp.n_ids = n_ids;
+    sp.new_lp = static_cast<int32_t>(L / cf.page_size);
+    std::memcpy(sp.inv_turns, c->turns, sizeof(sp.inv_turns));
+    for (int i = 0; i < n_ids; ++i) sp.ids[i] = ids[i];
+    const cudaError_t e =
+        timed_launch(c, CSR_KERNEL_ATTENTION, true, s, [&] { return launch_step(sp, cf.head_dim, s); });
+    if (e != cudaSuccess) return cuda_fail(c, e, "attention launch");
+    c->step_append += static_cast<uint32_t>(sp.s.grid);
+    if (sp.s.n_slots > 0) c->step_barrier += static_cast<uint32_t>(sp.s.grid);
+    ++c->launches;
+    return CSR_OK;
+  }
+
   RopeAppendParams rp{};
   rp.q = static_cast<const uint16_t *>(q);
   rp.k = static_cast<const uint16_t *>(k);
@@ -380,7 +530,7 @@ csr_status run_block(csr_ctx *c, int slot, int ws, const void *q, const void *k,
   rp.v_pool = c->v_pool;
   rp.q_pack = c->wsp<uint16_t>(c->lay.qpack[ws]);
   rp.page_table = c->d_pt(slot);
-  rp.err = c->wsp<uint32_t>(c->lay.err);
+  rp.err = ap.err;
   rp.pos0 = L;
   rp.n = n;
   rp.hq = cf.num_q_heads;
@@ -392,56 +542,21 @@ csr_status run_block(csr_ctx *c, int slot, int ws, const void *q, const void *k,
   rp.pool_pages = cf.pool_pages;
   rp.first_lp = first_lp;
   rp.n_ids = n_ids;
-  std::memcpy(rp.inv_turns, c->inv_turns, sizeof(rp.inv_turns));
+  std::memcpy(rp.inv_turns, c->turns, sizeof(rp.inv_turns));
   for (int i = 0; i < n_ids; ++i) rp.ids[i] = ids[i];
-  const bool fg = ws == 0;
 
-  AttnParams ap{};
-  ap.tm_q = c->tm_q[ws];
-  ap.tm_k = c->tm_k;
-  ap.tm_v = c->tm_v;
-  ap.page_table = c->d_pt(slot);
-  ap.out = static_cast<uint16_t *>(out);
-  ap.lse = lse;
-  ap.part_o = c->wsp<float>(c->lay.part_o[ws]);
-  ap.part_lse = c->wsp<float>(c->lay.part_lse[ws]);
-  ap.err = rp.err;
-  ap.L = L;
-  ap.n = n;
-  ap.hq = cf.num_q_heads;
-  ap.hkv = cf.num_kv_heads;
-  ap.group = c->group;
-  ap.page_size = cf.page_size;
-  ap.rows_cap = c->lay.rows_cap;
-  ap.n_tiles = static_cast<int32_t>(ceil_div(static_cast<int64_t>(n) * c->group, kBM));
-  ap.n_pages_valid = static_cast<int32_t>(pages_for(c, L + n));
-  ap.pool_pages = cf.pool_pages;
-  const int T = kBM / c->group;
-  ap.unit_tiles = (cf.flags & CSR_FLAG_SINGLE_TILE) ? 1 : 2;
-  ap.kv_tile = (!(cf.flags & CSR_FLAG_SINGLE_TILE) && (cf.flags & CSR_FLAG_PIPE_64)) ? kBN64 : kBN;
-  const int64_t uph = ceil_div(ap.n_tiles, ap.unit_tiles);
+  const int64_t uph = ceil_div(ap.n_tiles, 2);
   const int64_t units = uph * cf.num_kv_heads;
-  const int64_t kv_max =
-      unit_iters(L, n, T, static_cast<int32_t>(uph * ap.unit_tiles - 1), ap.kv_tile);
+  const int64_t kv_max = unit_iters(L, n, T, static_cast<int32_t>(uph * 2 - 1));
   const int tpc = cf.rebuild_tiles_per_cta > 0 ? cf.rebuild_tiles_per_cta : kDefaultRebuildTiles;
-  if (ws == 0 && cf.fg_chunk_tiles > 0) {
-    // fixed chunk length, but never more split items than the partial buffer holds
-    const int64_t cap_units = std::max<int64_t>(1, kPartialItems / ap.unit_tiles / units);
-    const int64_t min_c = ceil_div(kv_max, cap_units);
-    ap.chunk_tiles = static_cast<int32_t>(std::max<int64_t>(cf.fg_chunk_tiles, min_c));
-  } else {
-    ap.chunk_tiles = choose_chunk_tiles(units, kv_max, c->fg_grid, ws == 0 ? 0 : tpc, cf.head_dim,
-                                        ap.unit_tiles, ap.kv_tile);
-  }
+  ap.chunk_tiles = choose_chunk_tiles(units, kv_max, tpc);
   const int64_t n_chunks = ceil_div(kv_max, ap.chunk_tiles);
   ap.n_items = static_cast<int32_t>(n_chunks * units);
-  // foreground: persistent CTAs over the items; rebuild: one item per CTA
-  ap.grid = ws == 0 ? static_cast<int32_t>(std::min<int64_t>(c->fg_grid, ap.n_items)) : ap.n_items;
-  ap.scale_log2 = c->scale_log2;
-  cudaError_t e = timed_launch(c, CSR_KERNEL_ROPE_APPEND, fg, s, [&] { return launch_rope_append(rp, s); });
+  ap.grid = ap.n_items;   // one item per CTA
+  cudaError_t e = launch_rope_append(rp, s);
   if (e != cudaSuccess) return cuda_fail(c, e, "rope_append launch");
   ++c->launches;
-  e = timed_launch(c, CSR_KERNEL_ATTENTION, fg, s, [&] { return launch_attention(ap, cf.head_dim, s); });
+  e = launch_attention(ap, cf.head_dim, s);
   if (e != cudaSuccess) return cuda_fail(c, e, "attention launch");
   ++c->launches;
   if (n_chunks > 1) {
@@ -457,11 +572,9 @@ csr_status run_block(csr_ctx *c, int slot, int ws, const void *q, const void *k,
     mp.group = ap.group;
     mp.n_tiles = ap.n_tiles;
     mp.chunk_tiles = ap.chunk_tiles;
-    mp.unit_tiles = ap.unit_tiles;
-    mp.kv_tile = ap.kv_tile;
     mp.d = cf.head_dim;
     mp.slots_per_row = merge_slots_per_row(n_chunks, mp.d);
-    e = timed_launch(c, CSR_KERNEL_MERGE, fg, s, [&] { return launch_merge(mp, s); });
+    e = launch_merge(mp, s);
     if (e != cudaSuccess) return cuda_fail(c, e, "merge launch");
     ++c->launches;
   }
@@ -730,8 +843,11 @@ csr_status csr_create(const csr_config *cfg, void *k_pool, void *v_pool, void *w
                                                 : 1.0 / std::sqrt(static_cast<double>(cfg->head_dim));
   c->scale_log2 = static_cast<float>(scale * 1.4426950408889634);  // log2(e)
   const double two_pi = 6.283185307179586476925286766559;
-  for (int i = 0; i < cfg->head_dim / 2; ++i)
+  for (int i = 0; i < cfg->head_dim / 2; ++i) {
     c->inv_turns[i] = std::pow(cfg->rope_base, -2.0 * i / cfg->head_dim) / two_pi;
+    c->turns[i].hi = static_cast<float>(c->inv_turns[i]);
+    c->turns[i].lo = static_cast<float>(c->inv_turns[i] - static_cast<double>(c->turns[i].hi));
+  }
   c->pool.init(cfg->pool_pages);
   if (!c->plan_only) {
     const uintptr_t a = reinterpret_cast<uintptr_t>(k_pool) | reinterpret_cast<uintptr_t>(v_pool) |
@@ -751,7 +867,9 @@ csr_status csr_create(const csr_config *cfg, void *k_pool, void *v_pool, void *w
       delete c;
       return CSR_ECUDA;
     }
-    c->fg_grid = cfg->num_ctas > 0 ? cfg->num_ctas : std::min(c->num_sms, c->lay.fg_cap);
+    // the fused foreground launch is cooperative: at most one CTA per SM
+    c->fg_grid = std::min(std::min(cfg->num_ctas > 0 ? cfg->num_ctas : c->num_sms, c->num_sms),
+                          kMaxStepGrid);
     const uint64_t pool_rows = static_cast<uint64_t>(cfg->pool_pages) * cfg->num_kv_heads * cfg->page_size;
     const uint32_t kv_box = static_cast<uint32_t>(std::min(cfg->page_size, 64));
     bool ok = encode_rows(&c->tm_k, k_pool, pool_rows, cfg->head_dim, kv_box) &&
@@ -1377,6 +1495,63 @@ csr_status csr_get_timing(csr_ctx *c, csr_timing *out) {
     c->spare_events.push_back(t.b);
   }
   c->timed.clear();
+  return CSR_OK;
+}
+
+csr_status csr_foreground_schedule(const csr_config *cfg, int64_t L, int32_t n, int32_t grid,
+                                   csr_piece *pieces, int32_t capacity, int32_t *count,
+                                   int32_t *n_slots) {
+  if (!count || !valid_config(cfg, nullptr) || L < 0 || n < 1 || n > cfg->max_new_tokens || grid < 0)
+    return CSR_EINVAL;
+  if (grid == 0) {
+    if (cfg->flags & CSR_FLAG_PLAN_ONLY) return CSR_EINVAL;
+    int dev = 0, sms = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+      return CSR_ECUDA;
+    grid = sms;
+  }
+  grid = std::min(grid, kMaxStepGrid);
+  const int group = cfg->num_q_heads / cfg->num_kv_heads;
+  const int T = kBM / group;
+  const int32_t n_tiles = static_cast<int32_t>(ceil_div(static_cast<int64_t>(n) * group, kBM));
+  StepSchedule S;
+  build_step_schedule(L, n, T, cfg->num_kv_heads, n_tiles, grid, cfg->fg_chunk_tiles, S);
+  // Enumerate what each CTA's walker yields, in order.
+  std::vector<csr_piece> out;
+  const int hkv = cfg->num_kv_heads;
+  auto K = [&](int32_t u) { return unit_iters(L, n, T, 2 * (u / hkv) + 1); };
+  for (int32_t c = 0; c < S.grid; ++c) {
+    int32_t order = 0;
+    if (S.chunked) {
+      for (int32_t it = c; it < S.n_items; it += S.grid) {
+        const int32_t k = it / S.n_units, u = it - k * S.n_units;
+        const int64_t kv = K(u), j0 = static_cast<int64_t>(k) * S.chunk_tiles;
+        if (j0 >= kv) continue;
+        const int64_t j1 = std::min<int64_t>(j0 + S.chunk_tiles, kv);
+        out.push_back({c, order++, u, static_cast<int32_t>(j0), static_cast<int32_t>(j1),
+                       kv <= S.chunk_tiles ? -1 : it});
+      }
+      continue;
+    }
+    for (int32_t r = 0; r < S.full_rounds; ++r) {
+      const int32_t u = r * S.grid + ((r & 1) ? S.grid - 1 - c : c);
+      out.push_back({c, order++, u, 0, static_cast<int32_t>(K(u)), -1});
+    }
+    for (int l = 0; l < S.levels; ++l) {
+      const uint64_t e = S.piece[l][c];
+      if (e == kNoPiece) continue;
+      out.push_back({c, order++, static_cast<int32_t>(e & 0xffffu), static_cast<int32_t>((e >> 16) & 0xffffffu),
+                     static_cast<int32_t>((e >> 40) & 0xffffffu),
+                     S.slot[l][c] == kSlotWhole ? -1 : static_cast<int32_t>(S.slot[l][c])});
+    }
+  }
+  *count = static_cast<int32_t>(out.size());
+  if (n_slots) *n_slots = S.n_slots;
+  if (pieces) {
+    if (capacity < *count) return CSR_ENOMEM;
+    std::copy(out.begin(), out.end(), pieces);
+  }
   return CSR_OK;
 }
 

@@ -105,9 +105,14 @@ extern "C" csr_status csr_attend_block_noalloc(const csr_block_args *a, csr_stre
     if (!p || !aligned16(p)) return CSR_EINVAL;
   if (!a->k_pool || !a->v_pool || !a->page_table || !aligned16(a->k_pool) || !aligned16(a->v_pool))
     return CSR_EINVAL;
-  // the packed queries of this call must fit the static scratch
+  // The packed queries of this call must fit the static scratch.  Bound each
+  // factor before multiplying: max_rows is at most 2^22 and n * g at most
+  // 2^38, so nothing below overflows 64 bits whatever the arguments.
+  const int64_t max_rows = static_cast<int64_t>(kQBytes) / (static_cast<int64_t>(hkv) * d * 2);
+  if (static_cast<int64_t>(a->n) * g > max_rows) return CSR_EINVAL;
   const int64_t rows_cap = cdiv(static_cast<int64_t>(a->n) * g, 2 * kBM) * 2 * kBM;
-  if (rows_cap * hkv * d * 2 > static_cast<int64_t>(kQBytes)) return CSR_EINVAL;
+  if (rows_cap > max_rows) return CSR_EINVAL;
+  if (a->L > (1ll << 24) - a->n) return CSR_EINVAL;   // RoPE positions stay exact fp32 integers
 
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return CSR_ECUDA;
@@ -145,7 +150,11 @@ extern "C" csr_status csr_attend_block_noalloc(const csr_block_args *a, csr_stre
   rp.first_lp = 0;
   rp.n_ids = 0;
   const double two_pi = 6.283185307179586476925286766559;
-  for (int i = 0; i < d / 2; ++i) rp.inv_turns[i] = std::pow(a->rope_base, -2.0 * i / d) / two_pi;
+  for (int i = 0; i < d / 2; ++i) {
+    const double w = std::pow(a->rope_base, -2.0 * i / d) / two_pi;
+    rp.inv_turns[i].hi = static_cast<float>(w);
+    rp.inv_turns[i].lo = static_cast<float>(w - static_cast<double>(rp.inv_turns[i].hi));
+  }
   if (launch_rope_append(rp, s) != cudaSuccess) return CSR_ECUDA;
 
   // K2: two-tile attention over keys [0, L + n)
@@ -171,12 +180,10 @@ extern "C" csr_status csr_attend_block_noalloc(const csr_block_args *a, csr_stre
   ap.n_tiles = static_cast<int32_t>(cdiv(static_cast<int64_t>(a->n) * g, kBM));
   ap.n_pages_valid = static_cast<int32_t>(cdiv(a->L + a->n, P));
   ap.pool_pages = a->pool_pages;
-  ap.unit_tiles = 2;
-  ap.kv_tile = kBN;
   const int T = kBM / g;
   const int64_t uph = cdiv(ap.n_tiles, 2);
   const int64_t units = uph * hkv;
-  const int64_t kv_max = unit_iters(a->L, a->n, T, static_cast<int32_t>(uph * 2 - 1), kBN);
+  const int64_t kv_max = unit_iters(a->L, a->n, T, static_cast<int32_t>(uph * 2 - 1));
   // Split the key range only as far as the static partial buffer allows:
   // one chunk per unit when there are enough units to fill the SMs, else
   // the most chunks (up to one wave) whose partials fit.
@@ -213,8 +220,6 @@ extern "C" csr_status csr_attend_block_noalloc(const csr_block_args *a, csr_stre
     mp.group = g;
     mp.n_tiles = ap.n_tiles;
     mp.chunk_tiles = ap.chunk_tiles;
-    mp.unit_tiles = 2;
-    mp.kv_tile = kBN;
     mp.d = d;
     mp.slots_per_row = merge_slots_per_row(n_chunks, mp.d);
     if (launch_merge(mp, s) != cudaSuccess) return CSR_ECUDA;

@@ -9,13 +9,21 @@
 namespace csr {
 
 // Attention tile shape: 128 packed query rows (tokens x group heads) against
-// 128 keys per step.  TMEM: two score buffers of 128 columns and one output
-// accumulator of head_dim columns.
+// 128 keys per step.  A unit is two consecutive query tiles of one KV head (a
+// pair); TMEM holds one score buffer of 128 columns and one output
+// accumulator of head_dim columns per query tile.
 constexpr int kBM = 128;
 constexpr int kBN = 128;
-constexpr int kMaxIdsPerCall = 1024;   // new pages named by one rope/append launch
+constexpr int kPairRows = 2 * kBM;
+constexpr int kMaxIdsPerCall = 1024;   // new pages named by one launch
 constexpr int kMaxPoolWords = 2048;    // free-bitmap words a compaction launch carries
 constexpr int kMaxHalfDim = 64;        // head_dim / 2 upper bound
+
+// RoPE frequency w_i = base^(-2i/d) / (2 pi) as two fp32 words (hi + lo), so
+// that the turn count of a position is formed to about 2^-25 (rope.cuh).
+struct TurnSplit {
+  float hi, lo;
+};
 
 // K1: RoPE + paged append (+ GQA packing of the rotated queries).
 struct RopeAppendParams {
@@ -31,11 +39,11 @@ struct RopeAppendParams {
   int32_t n, hq, hkv, d, page_size, group, rows_cap, pool_pages;
   int32_t first_lp;        // logical page of pos0
   int32_t n_ids;           // > 0: ids[] give the physical pages first_lp..; 0: read page_table
-  double inv_turns[kMaxHalfDim];  // base^(-2i/d) / (2 pi), i < d/2
+  TurnSplit inv_turns[kMaxHalfDim];
   int32_t ids[kMaxIdsPerCall];
 };
 
-// K2: split-KV attention of the packed query tiles over the paged cache.
+// K2: split-KV attention of pairs of packed query tiles over the paged cache.
 struct AttnParams {
   CUtensorMap tm_q;        // q_pack as [hkv * rows_cap][d], box 64 x 128
   CUtensorMap tm_k;        // k pool as [pool_pages*hkv*P][d], box 64 x P
@@ -49,21 +57,62 @@ struct AttnParams {
   int64_t L;               // cached tokens before this call
   int32_t n, hq, hkv, group, page_size, rows_cap, n_tiles, n_pages_valid, pool_pages;
   int32_t chunk_tiles;     // key tiles per item
-  int32_t unit_tiles;      // query tiles per item: 1 (attn_kernel) or 2 (pair / pipe kernels)
-  int32_t kv_tile;         // keys per key tile: 128, or 64 for attn_pipe_kernel
-  int32_t n_items;         // n_chunks * hkv * units per head, numbered (chunk, head, unit)
+  int32_t n_items;         // n_chunks * hkv * pairs per head, numbered (chunk, head, pair)
   int32_t grid;            // CTAs; CTA c runs items c, c + grid, ...
   float scale_log2;        // softmax_scale * log2(e)
 };
 
-// K3: merge of split partials.
+// Schedule of a fused foreground launch (attn_pair_kernel<HD, true>): which
+// pieces (unit, key tiles [j0, j1)) each CTA runs, and where split pieces
+// leave their partial outputs.  Units are numbered u = pair * hkv + head.
+constexpr int kMaxStepGrid = 160;
+constexpr int kMaxTailLevels = 6;
+constexpr uint64_t kNoPiece = ~0ull;
+constexpr uint16_t kSlotWhole = 0xffff;  // the piece is a whole unit: written directly
+struct StepSchedule {
+  int32_t grid;          // CTAs (<= kMaxStepGrid)
+  int32_t n_units;
+  int32_t chunked;       // 1: round-robin chunks (forced chunk length); 0: rounds + tail levels
+  // chunked form: items (chunk k, unit u) = k * n_units + u, CTA c runs c, c + grid, ...;
+  // every unit with more than one chunk is merged (slot = item)
+  int32_t chunk_tiles, n_items;
+  // rounds + tail form: CTA c runs units r * grid + (r odd ? grid - 1 - c : c)
+  // whole for r < full_rounds; units n_units - n_tail .. n_units - 1 are cut
+  // into the pieces of the tail levels, piece[l][c] being CTA c's at level l
+  int32_t full_rounds, n_tail, levels;
+  int32_t n_slots;       // partial slots written (0: the launch merges nothing)
+  uint64_t piece[kMaxTailLevels][kMaxStepGrid];  // unit | j0 << 16 | j1 << 40, or kNoPiece
+  uint16_t slot[kMaxTailLevels][kMaxStepGrid];   // partial slot, or kSlotWhole
+  uint16_t tail_slot0[kMaxStepGrid + 1];         // tail unit t's slots [tail_slot0[t], tail_slot0[t+1])
+};
+
+// Fused foreground block (one cooperative launch): RoPE + paged append of the
+// new keys/values, RoPE of the queries straight into shared memory, attention,
+// and the merge of split pieces after a grid barrier.
+struct StepParams {
+  AttnParams a;            // tm_q, part_* of the chunked form, n_items, chunk_tiles unused
+  const uint16_t *q;       // [n][hq][d] bf16, before RoPE
+  const uint16_t *k;       // [n][hkv][d]
+  const uint16_t *v;
+  uint16_t *k_pool, *v_pool;
+  uint32_t *sync;          // [0]: append arrivals, [1]: merge-barrier arrivals (both monotonic)
+  uint32_t append_target;  // sync[0] once every CTA of this launch has appended its share
+  uint32_t barrier_target; // sync[1] once every CTA of this launch has written its partials
+  int32_t first_lp, n_ids; // logical pages first_lp.. get ids[] (written to the table by CTA 0)
+  int32_t new_lp;          // logical page holding position L: key tiles reaching it wait for the append
+  TurnSplit inv_turns[kMaxHalfDim];
+  int32_t ids[kMaxIdsPerCall];
+  StepSchedule s;
+};
+
+// K3: merge of split partials (rebuild launches and the no-allocation block path).
 struct MergeParams {
   const float *part_o;
   const float *part_lse;
   uint16_t *out;
   float *lse;
   int64_t L;
-  int32_t n, hq, hkv, group, n_tiles, chunk_tiles, unit_tiles, kv_tile, d;
+  int32_t n, hq, hkv, group, n_tiles, chunk_tiles, d;
   int32_t slots_per_row;   // lane groups sharing one row's chunks (a power of two)
 };
 
@@ -107,25 +156,18 @@ struct GatherParams {
   int32_t n, hkv, d, page_size, pool_pages;
 };
 
-// Shared-memory bytes of the attention kernels for a head dim.
-size_t attn_smem_bytes(int head_dim);
-size_t attn_pair_smem_bytes(int head_dim);
-size_t attn_pipe_smem_bytes(int head_dim);
-
-// Key tiles (of `bn` keys) of query tile `tile`: its keys are [0, L + last token].
+// Key tiles (of kBN keys) of query tile `tile`: its keys are [0, L + last token].
 __host__ __device__ inline int64_t unit_iters(int64_t L, int32_t n, int32_t tokens_per_tile,
-                                              int32_t tile, int32_t bn = kBN) {
+                                              int32_t tile) {
   int64_t hi = static_cast<int64_t>(tile + 1) * tokens_per_tile;
   if (hi > n) hi = n;
-  return (L + hi + bn - 1) / bn;
+  return (L + hi + kBN - 1) / kBN;
 }
-
-// Key tile of the pipelined kernel (attn_pipe_kernel): 64 keys, so two score
-// buffers per query tile fit TMEM next to the two output accumulators.
-constexpr int kBN64 = 64;
 
 cudaError_t launch_rope_append(const RopeAppendParams &p, cudaStream_t s);
 cudaError_t launch_attention(const AttnParams &p, int head_dim, cudaStream_t s);
+// Cooperative launch of the fused foreground kernel (grid = p.s.grid CTAs).
+cudaError_t launch_step(const StepParams &p, int head_dim, cudaStream_t s);
 cudaError_t launch_merge(const MergeParams &p, cudaStream_t s);
 cudaError_t launch_evict(const EvictParams &p, cudaStream_t s);
 cudaError_t launch_gather(const GatherParams &p, cudaStream_t s);

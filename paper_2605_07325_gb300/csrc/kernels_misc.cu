@@ -11,41 +11,15 @@
 #include "../../include/csr.h"
 #include "internal.h"
 #include "ptx.cuh"
+#include "rope.cuh"
 
 namespace csr {
 
-__device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
-__device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xffff0000u); }
-__device__ __forceinline__ uint32_t pack2(float lo, float hi) {
-  __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
-  return *reinterpret_cast<uint32_t *>(&v);
-}
-
-// Rotate 8 pairs (x[i0..i0+7], x[i0+h..i0+h+7]) held as two 16-byte vectors.
-__device__ __forceinline__ void rotate8(const uint4 &a, const uint4 &b, const float *cs,
-                                        const float *sn, uint4 &ya, uint4 &yb) {
-  const uint32_t aw[4] = {a.x, a.y, a.z, a.w};
-  const uint32_t bw[4] = {b.x, b.y, b.z, b.w};
-  uint32_t ra[4], rb[4];
-#pragma unroll
-  for (int e = 0; e < 4; ++e) {
-    const float x0 = bf16_lo(aw[e]), x1 = bf16_hi(aw[e]);
-    const float z0 = bf16_lo(bw[e]), z1 = bf16_hi(bw[e]);
-    const float c0 = cs[2 * e], c1 = cs[2 * e + 1];
-    const float s0 = sn[2 * e], s1 = sn[2 * e + 1];
-    ra[e] = pack2(x0 * c0 - z0 * s0, x1 * c1 - z1 * s1);
-    rb[e] = pack2(z0 * c0 + x0 * s0, z1 * c1 + x1 * s1);
-  }
-  ya = make_uint4(ra[0], ra[1], ra[2], ra[3]);
-  yb = make_uint4(rb[0], rb[1], rb[2], rb[3]);
-}
-
 // Block (token t, part y): the token's 16-byte work items (rotated query
 // pairs, rotated key pairs, value vectors) y, y + gridDim.y, ... in units of
-// 256.  Angles: theta_i =
-// pos * base^(-2i/d); the turn count pos * base^(-2i/d) / (2 pi) is formed in
-// fp64 and reduced to [-1/2, 1/2] before the fp32 sincospi, so positions past
-// 10^5 keep full fp32 angle accuracy.
+// 256.  Angles theta_i = pos * base^(-2i/d) from rope_cos_sin (rope.cuh: the
+// turn count in two fp32 words, reduced to [-1/2, 1/2] before the fp32
+// sincospi, so positions past 10^5 keep full fp32 angle accuracy).
 __global__ void __launch_bounds__(256) rope_append_kernel(const __grid_constant__ RopeAppendParams p) {
   __shared__ float cs[kMaxHalfDim], sn[kMaxHalfDim];
   // The attention kernel may launch now: its setup (barriers, TMEM, tensor
@@ -55,14 +29,7 @@ __global__ void __launch_bounds__(256) rope_append_kernel(const __grid_constant_
   const int t = blockIdx.x;
   const int64_t pos = p.pos0 + t;
   const int half = p.d / 2;
-  for (int i = threadIdx.x; i < half; i += blockDim.x) {
-    const double turns = static_cast<double>(pos) * p.inv_turns[i];
-    const double fr = turns - rint(turns);
-    float s, c;
-    sincospif(static_cast<float>(2.0 * fr), &s, &c);
-    cs[i] = c;
-    sn[i] = s;
-  }
+  for (int i = threadIdx.x; i < half; i += blockDim.x) rope_cos_sin(pos, p.inv_turns[i], cs[i], sn[i]);
   // The previous kernel of the stream may still read the packed queries and
   // cache pages this block overwrites.
   pdl_wait();
@@ -91,7 +58,7 @@ __global__ void __launch_bounds__(256) rope_append_kernel(const __grid_constant_
       const uint4 a = *reinterpret_cast<const uint4 *>(src + i0);
       const uint4 b = *reinterpret_cast<const uint4 *>(src + i0 + half);
       uint4 ya, yb;
-      rotate8(a, b, cs + i0, sn + i0, ya, yb);
+      rope_rotate8(a, b, cs + i0, sn + i0, ya, yb);
       uint16_t *dst;
       if (is_q) {
         const int kvh = h / p.group, g = h % p.group;
