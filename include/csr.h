@@ -72,6 +72,12 @@ typedef enum csr_status {
 #define CSR_FLAG_PLAN_ONLY 0x1   /* layout planning only: no device memory is touched
                                     and no kernel runs; compute calls update the page
                                     tables and lengths but produce no outputs */
+#define CSR_FLAG_FUSED_ALWAYS 0x2 /* every foreground call is one cooperative launch of the
+                                     fused kernel (RoPE + append, attention, merge) */
+#define CSR_FLAG_FUSED_NEVER 0x4  /* every foreground call is three chained launches (RoPE +
+                                     append, attention items, merge of split items); by
+                                     default a call takes the fused launch when its attention
+                                     work is at least 600 key tiles per CTA */
 
 typedef struct csr_config {
   int32_t num_q_heads;    /* H_q */
@@ -92,8 +98,10 @@ typedef struct csr_config {
   int32_t flags;          /* CSR_FLAG_* */
   int32_t fg_chunk_tiles; /* > 0: a foreground launch splits every unit's key range into
                              chunks of this many 128-key tiles (more if the split partials
-                             would not fit), dealt round-robin to its CTAs; 0 = whole units
-                             in rounds and only the leftover units split (the default) */
+                             would not fit), dealt round-robin to its CTAs; 0 = the fused
+                             launch runs whole units in rounds and splits only the leftover
+                             units, the three-launch path picks the chunk length from a
+                             cost estimate (the default) */
 } csr_config;
 
 /*

@@ -29,6 +29,8 @@ STATUS_NAMES = {0: "CSR_OK", 1: "CSR_EINVAL", 2: "CSR_ENOMEM", 3: "CSR_ESTATE", 
                 5: "CSR_ECUDA", 6: "CSR_ETIMEOUT", 7: "CSR_EDEVICE"}
 DEVERR_WAIT_TIMEOUT, DEVERR_BAD_PAGE, DEVERR_ALLOC = 0x1, 0x2, 0x4
 FLAG_PLAN_ONLY = 0x1
+FLAG_FUSED_ALWAYS = 0x2
+FLAG_FUSED_NEVER = 0x4
 RECON_IDLE, RECON_RUNNING, RECON_SWAPPED = 0, 1, 2
 ROUTE_CONTINUE, ROUTE_BRIDGE, ROUTE_SWAPPED, ROUTE_STRAGGLER = 0, 1, 2, 3
 VERSION_ACTIVE, VERSION_PENDING = 0, 1

@@ -46,6 +46,8 @@ struct Range {
 
 constexpr int kPartialItems = 4096;      // split partials a launch may write (per staging)
 constexpr int kDefaultRebuildTiles = 16;
+// Key tiles per CTA from which a foreground block takes the fused launch.
+constexpr int kFusedMinTilesPerCta = 600;
 constexpr size_t kAlign = 256;
 
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
@@ -136,6 +138,22 @@ bool encode_rows(CUtensorMap *m, void *base, uint64_t rows, uint64_t d, uint32_t
   return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, base, dims, strides, box, estr,
             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// 3-D bf16 tensor map over the block's queries q[n][hq][d]: box {64 columns,
+// group heads, 128/group tokens} -- one 128-row packed query tile (rows t*G + g)
+// per 64-column half, 128-byte-swizzled like the MMA operand; tokens past n
+// read as zero.
+bool encode_queries(CUtensorMap *m, const void *q, uint64_t n, uint64_t hq, uint64_t d, uint32_t group) {
+  auto fn = tensor_map_encoder();
+  if (!fn) return false;
+  cuuint64_t dims[3] = {d, hq, n};
+  cuuint64_t strides[2] = {d * 2, hq * d * 2};
+  cuuint32_t box[3] = {64, group, static_cast<cuuint32_t>(kBM / group)};
+  cuuint32_t estr[3] = {1, 1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(q), dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
 struct Layout {  // workspace carve-out (byte offsets)
@@ -311,6 +329,32 @@ csr_status cuda_fail(csr_ctx *c, cudaError_t e, const char *where) {
 
 int64_t pages_for(const csr_ctx *c, int64_t len) { return ceil_div(len, c->cfg.page_size); }
 
+// Key chunks per pair for a foreground three-launch block of `units` pairs
+// whose longest key range is kv_max tiles: minimise a time estimate over the
+// persistent grid -- waves x (tiles per item x t_tile + per-item cost) plus
+// the split partials' write + merge read -- never more items than the
+// partial buffer holds.
+int32_t choose_fg_chunk_tiles(int64_t units, int64_t kv_max, int64_t grid, int head_dim) {
+  // us per key tile per CTA, per item, per split partial (rough GB300 figures)
+  const double t_tile = 1.5, t_item = 2.0, t_part = head_dim == 128 ? 0.04 : 0.02;
+  const int64_t cap_items = kPartialItems / 2;
+  int64_t best_c = kv_max;
+  double best_t = 1e300;
+  for (int64_t S = 1; S <= std::min<int64_t>(kv_max, 256); ++S) {
+    const int64_t C = ceil_div(kv_max, S);
+    const int64_t Se = ceil_div(kv_max, C);
+    const int64_t items = units * Se;
+    if (Se > 1 && items > cap_items) break;
+    const int64_t waves = ceil_div(items, grid);
+    const double t = waves * (C * t_tile + t_item) + (Se > 1 ? items * t_part : 0.0);
+    if (t < best_t - 1e-9) {
+      best_t = t;
+      best_c = C;
+    }
+  }
+  return static_cast<int32_t>(best_c);
+}
+
 // Key chunks per pair for a rebuild launch of `units` pairs whose longest key
 // range is kv_max tiles: the fewest chunks of at most max_tiles tiles, so each
 // CTA is short and a foreground launch waits at most one item for an SM;
@@ -463,8 +507,9 @@ cudaError_t timed_launch(csr_ctx *c, int kind, bool foreground, cudaStream_t s, 
 
 // Attend n new tokens at positions L.. of version `slot` (and append their
 // keys/values).  ws 0 (foreground, the caller's stream): one cooperative
-// launch of the fused kernel.  ws 1 (rebuild, the low-priority stream):
-// K1 -> K2 (short items) -> K3.  ids/n_ids name the physical pages of
+// launch of the fused kernel for long calls, else K1 -> K2 (persistent items)
+// -> K3.  ws 1 (rebuild, the low-priority stream): K1 -> K2 (short items) ->
+// K3.  ids/n_ids name the physical pages of
 // logical pages first_lp.. (written into the device table by the launch);
 // n_ids == 0 reads the device table instead.
 csr_status run_block(csr_ctx *c, int slot, int ws, const void *q, const void *k, const void *v,
@@ -495,12 +540,30 @@ csr_status run_block(csr_ctx *c, int slot, int ws, const void *q, const void *k,
   ap.scale_log2 = c->scale_log2;
   const int T = kBM / c->group;
 
+  // Foreground: one cooperative launch of the fused kernel when the call is
+  // long enough for its fixed costs (query preparation, grid barrier, merge:
+  // about 25 us) to vanish, else three chained launches (the rebuild's path
+  // with a persistent grid).  Flags force either.
+  bool fused = false;
   if (fg) {
+    if (cf.flags & CSR_FLAG_FUSED_ALWAYS) {
+      fused = true;
+    } else if (!(cf.flags & CSR_FLAG_FUSED_NEVER)) {
+      int64_t tiles = 0;
+      const int64_t pairs = ceil_div(ap.n_tiles, 2);
+      for (int64_t pr = 0; pr < pairs; ++pr) tiles += unit_iters(L, n, T, static_cast<int32_t>(2 * pr + 1));
+      tiles *= cf.num_kv_heads;
+      fused = tiles >= static_cast<int64_t>(kFusedMinTilesPerCta) * c->fg_grid;
+    }
+  }
+  if (fused) {
     StepParams &sp = c->step;
     build_step_schedule(L, n, T, cf.num_kv_heads, ap.n_tiles, c->fg_grid, cf.fg_chunk_tiles, sp.s);
     ap.grid = sp.s.grid;
     sp.a = ap;
     sp.q = static_cast<const uint16_t *>(q);
+    if (!encode_queries(&sp.tm_qraw, q, static_cast<uint64_t>(n), cf.num_q_heads, cf.head_dim, c->group))
+      return fail(c, CSR_ECUDA, "encoding the queries' tensor map");
     sp.k = static_cast<const uint16_t *>(k);
     sp.v = static_cast<const uint16_t *>(v);
     sp.k_pool = c->k_pool;
@@ -511,6 +574,12 @@ csr_status run_block(csr_ctx *c, int slot, int ws, const void *q, const void *k,
     sp.first_lp = first_lp;
     sp.n_ids = n_ids;
     sp.new_lp = static_cast<int32_t>(L / cf.page_size);
+    // The append's 16-byte work items: up to two per lane of one warp per CTA
+    // go to the MMA warp (idle until the first queries and keys are in
+    // place); more go to the eight softmax warps, after their first queries
+    // (one warp alone takes tens of microseconds over a few hundred tokens).
+    const int64_t append_items = static_cast<int64_t>(n) * cf.num_kv_heads * (cf.head_dim / 16 + cf.head_dim / 8);
+    sp.append_by_mma = append_items <= 2ll * 32 * sp.s.grid ? 1 : 0;
     std::memcpy(sp.inv_turns, c->turns, sizeof(sp.inv_turns));
     for (int i = 0; i < n_ids; ++i) sp.ids[i] = ids[i];
     const cudaError_t e =
@@ -548,15 +617,27 @@ csr_status run_block(csr_ctx *c, int slot, int ws, const void *q, const void *k,
   const int64_t uph = ceil_div(ap.n_tiles, 2);
   const int64_t units = uph * cf.num_kv_heads;
   const int64_t kv_max = unit_iters(L, n, T, static_cast<int32_t>(uph * 2 - 1));
-  const int tpc = cf.rebuild_tiles_per_cta > 0 ? cf.rebuild_tiles_per_cta : kDefaultRebuildTiles;
-  ap.chunk_tiles = choose_chunk_tiles(units, kv_max, tpc);
+  if (fg) {
+    // persistent CTAs over the items: a forced chunk length (never more items
+    // than the partial buffer holds) or the cost model's
+    if (cf.fg_chunk_tiles > 0) {
+      const int64_t cap_units = std::max<int64_t>(1, kPartialItems / 2 / units);
+      ap.chunk_tiles = static_cast<int32_t>(std::max<int64_t>(cf.fg_chunk_tiles, ceil_div(kv_max, cap_units)));
+    } else {
+      ap.chunk_tiles = choose_fg_chunk_tiles(units, kv_max, c->fg_grid, cf.head_dim);
+    }
+  } else {
+    const int tpc = cf.rebuild_tiles_per_cta > 0 ? cf.rebuild_tiles_per_cta : kDefaultRebuildTiles;
+    ap.chunk_tiles = choose_chunk_tiles(units, kv_max, tpc);
+  }
   const int64_t n_chunks = ceil_div(kv_max, ap.chunk_tiles);
   ap.n_items = static_cast<int32_t>(n_chunks * units);
-  ap.grid = ap.n_items;   // one item per CTA
-  cudaError_t e = launch_rope_append(rp, s);
+  // foreground: persistent CTAs over the items; rebuild: one item per CTA
+  ap.grid = fg ? static_cast<int32_t>(std::min<int64_t>(c->fg_grid, ap.n_items)) : ap.n_items;
+  cudaError_t e = timed_launch(c, CSR_KERNEL_ROPE_APPEND, fg, s, [&] { return launch_rope_append(rp, s); });
   if (e != cudaSuccess) return cuda_fail(c, e, "rope_append launch");
   ++c->launches;
-  e = launch_attention(ap, cf.head_dim, s);
+  e = timed_launch(c, CSR_KERNEL_ATTENTION, fg, s, [&] { return launch_attention(ap, cf.head_dim, s); });
   if (e != cudaSuccess) return cuda_fail(c, e, "attention launch");
   ++c->launches;
   if (n_chunks > 1) {
@@ -574,7 +655,7 @@ csr_status run_block(csr_ctx *c, int slot, int ws, const void *q, const void *k,
     mp.chunk_tiles = ap.chunk_tiles;
     mp.d = cf.head_dim;
     mp.slots_per_row = merge_slots_per_row(n_chunks, mp.d);
-    e = launch_merge(mp, s);
+    e = timed_launch(c, CSR_KERNEL_MERGE, fg, s, [&] { return launch_merge(mp, s); });
     if (e != cudaSuccess) return cuda_fail(c, e, "merge launch");
     ++c->launches;
   }

@@ -90,7 +90,8 @@ struct StepSchedule {
 // new keys/values, RoPE of the queries straight into shared memory, attention,
 // and the merge of split pieces after a grid barrier.
 struct StepParams {
-  AttnParams a;            // tm_q, part_* of the chunked form, n_items, chunk_tiles unused
+  AttnParams a;            // tm_q, n_items, chunk_tiles unused
+  CUtensorMap tm_qraw;     // q as [n][hq][d] (3-D), box {64, G, 128/G}: one query tile per column half
   const uint16_t *q;       // [n][hq][d] bf16, before RoPE
   const uint16_t *k;       // [n][hkv][d]
   const uint16_t *v;
@@ -100,6 +101,7 @@ struct StepParams {
   uint32_t barrier_target; // sync[1] once every CTA of this launch has written its partials
   int32_t first_lp, n_ids; // logical pages first_lp.. get ids[] (written to the table by CTA 0)
   int32_t new_lp;          // logical page holding position L: key tiles reaching it wait for the append
+  int32_t append_by_mma;   // 1: the MMA warp appends (few tokens); 0: the softmax warps
   TurnSplit inv_turns[kMaxHalfDim];
   int32_t ids[kMaxIdsPerCall];
   StepSchedule s;

@@ -60,11 +60,17 @@
 
 namespace csr {
 
-// One piece of work: key tiles [j0, j1) of a unit (head, pair).  slot: the
-// partial-output slot of a split piece.
+// One piece of work: key tiles [j0, j1) of a unit (head, pair).  A split
+// piece writes row r (0..255) of its partial output at row pbase + r * pstride
+// of the partial buffer: slot-major (pbase = slot * 256, pstride = 1) for
+// item launches and the chunked form, row-major over the unit's slots
+// (pbase = first slot * 256 + slot index, pstride = the unit's slot count) for
+// the rounds + tail form, so that a merge batch of rows is one contiguous copy.
 struct Seg {
   int32_t head, pair, slot;
   int64_t j0, j1;
+  int64_t pbase;
+  int32_t pstride;
   bool complete;
 };
 
@@ -121,6 +127,16 @@ __device__ __forceinline__ void tma_load_2d_if(uint32_t pred, void *dst, const C
       "@p cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
       " [%0], [%1, {%2, %3}], [%4];\n\t}" ::"r"(smem_u32(dst)),
       "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_u32(bar)), "r"(pred)
+      : "memory");
+}
+
+__device__ __forceinline__ void tma_load_3d_if(uint32_t pred, void *dst, const CUtensorMap *map,
+                                               uint64_t *bar, int32_t x, int32_t y, int32_t z) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %6, 0;\n\t"
+      "@p cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3, %4}], [%5];\n\t}" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(smem_u32(bar)), "r"(pred)
       : "memory");
 }
 
@@ -214,8 +230,16 @@ struct PairCfg {
   static constexpr int kPtStage = 512;
   static constexpr int kAngOff = kPtOff + kPtStage * 4;
   static constexpr int kAngEntries = 256;                      // (cos, sin) pairs per softmax warp
+  static constexpr int kTurnOff = kAngOff + 8 * kAngEntries * 8;   // RoPE frequencies (TurnSplit[d/2])
+  static constexpr int kIdsOff = kTurnOff + kMaxHalfDim * 8;       // the launch's first new page ids
+  static constexpr int kSmemIds = 256;
   static constexpr int kSmem = kAngOff + 1024;                 // + alignment slack
-  static constexpr int kSmemStep = kAngOff + 8 * kAngEntries * 8 + 1024;
+  static constexpr int kSmemStep = kIdsOff + kSmemIds * 4 + 1024;
+  // fused form, after the attention loops: the merge stages partial rows in
+  // the Q and K/V region and keeps row LSEs and weights in the angle tables
+  static constexpr int kMergeBuf = kBarOff;
+  static constexpr int kMergeRows = 40;                        // rows per merge batch
+  static constexpr int kMergeWts = (8 * kAngEntries * 8) / 4 - kMergeRows;  // weight floats
   static constexpr uint32_t kTmemCols = 512;
   static constexpr uint32_t kOCol = 2 * kBN;                   // O_A; O_B at kOCol + HD
 };
@@ -225,7 +249,7 @@ struct PairBars {
   uint64_t q_full, q_empty;
   uint64_t k_full[4], k_empty[4], v_full[4], v_empty[4];
   uint64_t s_full[2], p_full[2], o_final[2], o_free[2];
-  uint64_t drain;
+  uint64_t drain, merge_full, qraw_full;
   uint32_t tmem_base;
   int abort;
 };
@@ -253,6 +277,8 @@ struct PairWalker {
       s.head = head;
       s.pair = pair;
       s.slot = it;
+      s.pbase = static_cast<int64_t>(it) * kPairRows;
+      s.pstride = 1;
       s.j0 = j0;
       s.j1 = min(j0 + p.chunk_tiles, kv);
       s.complete = kv <= p.chunk_tiles;
@@ -281,6 +307,8 @@ struct StepWalker {
         s.head = u - pair * A.hkv;
         s.pair = pair;
         s.slot = it;
+        s.pbase = static_cast<int64_t>(it) * kPairRows;
+        s.pstride = 1;
         s.j0 = j0;
         s.j1 = min(j0 + S.chunk_tiles, kv);
         s.complete = kv <= S.chunk_tiles;
@@ -295,6 +323,8 @@ struct StepWalker {
       s.head = u - pair * A.hkv;
       s.pair = pair;
       s.slot = kSlotWhole;
+      s.pbase = 0;
+      s.pstride = 1;
       s.j0 = 0;
       s.j1 = unit_iters(A.L, A.n, T, 2 * pair + 1);
       s.complete = true;
@@ -312,6 +342,14 @@ struct StepWalker {
       s.j0 = static_cast<int64_t>((e >> 16) & 0xffffffu);
       s.j1 = static_cast<int64_t>((e >> 40) & 0xffffffu);
       s.complete = s.slot == kSlotWhole;
+      s.pbase = 0;
+      s.pstride = 1;
+      if (!s.complete) {
+        const int32_t t = u - (S.n_units - S.n_tail);
+        const int32_t s0 = S.tail_slot0[t];
+        s.pbase = static_cast<int64_t>(s0) * kPairRows + (s.slot - s0);
+        s.pstride = S.tail_slot0[t + 1] - s0;
+      }
       return true;
     }
     return false;
@@ -338,239 +376,384 @@ __device__ __forceinline__ StepWalker make_walker(const StepParams &) {
 
 // ============================================================ fused-form steps
 // Physical page of logical page lp of the block's version: the launch's new
-// pages come from ids[], the older ones from the table.  -1 when out of range.
-__device__ __forceinline__ int32_t step_page(const StepParams &p, int64_t lp) {
+// pages come from its id list (the first kSmemIds copied to shared memory at
+// entry, `ids_s`), the older ones from the table.  -1 when out of range.
+__device__ __forceinline__ int32_t step_page(const StepParams &p, const int32_t *ids_s, int64_t lp) {
   const AttnParams &A = p.a;
-  int32_t phys = (lp >= p.first_lp && lp < p.first_lp + p.n_ids) ? p.ids[lp - p.first_lp]
-                                                                   : A.page_table[lp];
+  int32_t phys;
+  if (lp >= p.first_lp && lp < p.first_lp + p.n_ids) {
+    const int64_t i = lp - p.first_lp;
+    phys = i < 256 ? ids_s[i] : p.ids[i];
+  } else {
+    phys = A.page_table[lp];
+  }
   return (phys < 0 || phys >= A.pool_pages) ? -1 : phys;
 }
 
-// This CTA's share of the append (256 softmax threads, tid 0..255): rotated
-// keys and values of the new tokens into their cache slots, and (CTA 0) the
-// new pages' ids into the device table.  Work items of 16 bytes out: 8 key
-// pairs (two stores) or 8 values.
+// This CTA's share of the append (nthreads threads, tid 0..nthreads-1):
+// rotated keys and values of the new tokens into their cache slots, and
+// (CTA 0) the new pages' ids into the device table.  Work items of 16 bytes
+// out: 8 key pairs (two stores) or 8 values.
 template <int HD>
-__device__ void step_append(const StepParams &p, int tid) {
+__device__ __noinline__ void step_append(const StepParams &p, const TurnSplit *turns, const int32_t *ids_s, int tid,
+                                         int nthreads) {
   const AttnParams &A = p.a;
   constexpr int half = HD / 2, c16 = HD / 16, c8 = HD / 8;
+  constexpr int kBatch = 4;   // items whose input loads are in flight together
   if (blockIdx.x == 0) {
     int32_t *table = const_cast<int32_t *>(A.page_table);
-    for (int i = tid; i < p.n_ids; i += 256) table[p.first_lp + i] = p.ids[i];
+    for (int i = tid; i < p.n_ids; i += nthreads) table[p.first_lp + i] = p.ids[i];
   }
   const int64_t nk = static_cast<int64_t>(A.n) * A.hkv * c16;
   const int64_t nv = static_cast<int64_t>(A.n) * A.hkv * c8;
-  for (int64_t w = static_cast<int64_t>(blockIdx.x) * 256 + tid; w < nk + nv;
-       w += static_cast<int64_t>(gridDim.x) * 256) {
-    const bool is_k = w < nk;
-    const int64_t ww = is_k ? w : w - nk;
-    const int per_tok = A.hkv * (is_k ? c16 : c8);
-    const int64_t t = ww / per_tok;
-    const int rem = static_cast<int>(ww - t * per_tok);
-    const int h = rem / (is_k ? c16 : c8);
-    const int i0 = (rem % (is_k ? c16 : c8)) * 8;
-    const int64_t pos = A.L + t;
-    const int64_t lp = pos / A.page_size;
-    const int32_t phys = step_page(p, lp);
-    if (phys < 0) {
-      atomicOr(A.err, CSR_DEVERR_BAD_PAGE);
-      continue;
-    }
-    const int64_t slot_row = (static_cast<int64_t>(phys) * A.hkv + h) * A.page_size + (pos - lp * A.page_size);
-    if (is_k) {
-      const uint16_t *src = p.k + (t * A.hkv + h) * HD;
-      const uint4 a = *reinterpret_cast<const uint4 *>(src + i0);
-      const uint4 b = *reinterpret_cast<const uint4 *>(src + i0 + half);
-      float cs[8], sn[8];
+  // items interleaved over the CTAs (item g = tid * grid + CTA), so a small
+  // block spreads over every CTA instead of filling the first ones
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * nthreads;
+  for (int64_t w0 = static_cast<int64_t>(tid) * gridDim.x + blockIdx.x; w0 < nk + nv; w0 += kBatch * stride) {
+    uint4 a[kBatch], b[kBatch];
 #pragma unroll
-      for (int e = 0; e < 8; ++e) rope_cos_sin(pos, p.inv_turns[i0 + e], cs[e], sn[e]);
-      uint4 ya, yb;
-      rope_rotate8(a, b, cs, sn, ya, yb);
-      uint16_t *dst = p.k_pool + slot_row * HD;
-      *reinterpret_cast<uint4 *>(dst + i0) = ya;
-      *reinterpret_cast<uint4 *>(dst + i0 + half) = yb;
-    } else {
-      const uint16_t *src = p.v + (t * A.hkv + h) * HD + i0;
-      *reinterpret_cast<uint4 *>(p.v_pool + slot_row * HD + i0) = *reinterpret_cast<const uint4 *>(src);
+    for (int u = 0; u < kBatch; ++u) {   // the inputs of up to four items
+      const int64_t w = w0 + u * stride;
+      if (w >= nk + nv) break;
+      const bool is_k = w < nk;
+      const int64_t ww = is_k ? w : w - nk;
+      const int per_tok = A.hkv * (is_k ? c16 : c8);
+      const int64_t t = ww / per_tok;
+      const int rem = static_cast<int>(ww - t * per_tok);
+      const int h = rem / (is_k ? c16 : c8);
+      const int i0 = (rem % (is_k ? c16 : c8)) * 8;
+      if (is_k) {
+        const uint16_t *src = p.k + (t * A.hkv + h) * HD;
+        a[u] = *reinterpret_cast<const uint4 *>(src + i0);
+        b[u] = *reinterpret_cast<const uint4 *>(src + i0 + half);
+      } else {
+        a[u] = *reinterpret_cast<const uint4 *>(p.v + (t * A.hkv + h) * HD + i0);
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < kBatch; ++u) {
+      const int64_t w = w0 + u * stride;
+      if (w >= nk + nv) break;
+      const bool is_k = w < nk;
+      const int64_t ww = is_k ? w : w - nk;
+      const int per_tok = A.hkv * (is_k ? c16 : c8);
+      const int64_t t = ww / per_tok;
+      const int rem = static_cast<int>(ww - t * per_tok);
+      const int h = rem / (is_k ? c16 : c8);
+      const int i0 = (rem % (is_k ? c16 : c8)) * 8;
+      const int64_t pos = A.L + t;
+      const int64_t lp = pos / A.page_size;
+      const int32_t phys = step_page(p, ids_s, lp);
+      if (phys < 0) {
+        atomicOr(A.err, CSR_DEVERR_BAD_PAGE);
+        continue;
+      }
+      const int64_t slot_row = (static_cast<int64_t>(phys) * A.hkv + h) * A.page_size + (pos - lp * A.page_size);
+      if (is_k) {
+        float cs[8], sn[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) rope_cos_sin(pos, turns[i0 + e], cs[e], sn[e]);
+        uint4 ya, yb;
+        rope_rotate8(a[u], b[u], cs, sn, ya, yb);
+        uint16_t *dst = p.k_pool + slot_row * HD;
+        *reinterpret_cast<uint4 *>(dst + i0) = ya;
+        *reinterpret_cast<uint4 *>(dst + i0 + half) = yb;
+      } else {
+        *reinterpret_cast<uint4 *>(p.v_pool + slot_row * HD + i0) = a[u];
+      }
     }
   }
   fence_proxy_async_global();   // the other CTAs read these slots by TMA
 }
 
-// Rotate the queries of query tile `wg` of unit (head, pair) into that tile's
-// shared-memory operand.  Called by each softmax warp for its 32 rows (thread
-// `row` = TMEM lane = tile row): row r holds token r / G, query head
-// head * G + r % G, in the 128-byte-swizzled K-major layout the MMA
-// descriptors describe (16-byte chunk c of row r at chunk position c ^ (r % 8)
-// of its 128-byte line; box b of 64 columns at b * 128 rows * 128 bytes).  The
-// (cos, sin) of the warp's tokens are computed once per token and pair index
-// into the warp's own table `ang` (batches of kAngEntries), shared by the G
-// heads of a token; only __syncwarp orders it, so a warp never waits for
-// another.  Rows past the block are zero.  Ends with the proxy fence that
-// lets the tensor core read the tile.
+// The raw queries of a unit's two query tiles, brought by the producer: one
+// 3-D TMA box {64 columns, G heads, 128/G tokens} per tile and column half,
+// landing in the 128-byte-swizzled K-major layout the MMA descriptors describe
+// (tile row r = token r / G, head head * G + r % G; tokens past the block read
+// as zero).
 template <int HD>
-__device__ void step_prep_q(const StepParams &p, uint8_t *qtile, float2 *ang, int head, int pair,
-                            int wg, int row, int lane, int T) {
-  const AttnParams &A = p.a;
-  constexpr int half = HD / 2, c8 = HD / 8, c16 = HD / 16;
-  constexpr int per_batch = PairCfg<HD>::kAngEntries / half;   // tokens per table batch
-  const int G = A.group;
-  const int tile = pair * 2 + wg;
-  const int64_t tok0 = static_cast<int64_t>(tile) * T;
-  const int tr = row / G;
-  const int g = row - tr * G;
-  const bool valid = tile < A.n_tiles && tok0 + tr < A.n;
-  const int w0 = (row - lane) / G, w1 = (row - lane + 31) / G + 1;   // the warp's tokens
-  uint8_t *line = qtile + row * 128;
-  const uint32_t sw = static_cast<uint32_t>(row & 7);
-  for (int b0 = w0; b0 < w1; b0 += per_batch) {
-    const int bt = min(per_batch, w1 - b0);
-    __syncwarp();   // the previous batch's table is no longer read
-    for (int e = lane; e < bt * half; e += 32) {
-      const int tt = e / half;
-      const int i = e - tt * half;
-      float c, s;
-      rope_cos_sin(A.L + tok0 + b0 + tt, p.inv_turns[i], c, s);
-      ang[e] = make_float2(c, s);
-    }
-    __syncwarp();
-    if (tr < b0 || tr >= b0 + bt) continue;
-    uint4 x[c8];
-    if (valid) {
-      const uint16_t *src = p.q + ((tok0 + tr) * A.hq + head * G + g) * HD;
+__device__ __forceinline__ void step_qraw_issue(uint32_t pred, const StepParams &p, uint8_t *smem,
+                                                uint64_t *bar, int head, int pair, int T) {
+  using C = PairCfg<HD>;
+  const int G = p.a.group;
+  mbar_arrive_expect_tx_if(pred, bar, 2 * C::kQBytes);
 #pragma unroll
-      for (int c = 0; c < c8; ++c) x[c] = reinterpret_cast<const uint4 *>(src)[c];
-      const float2 *a = ang + (tr - b0) * half;
+  for (int x = 0; x < 2; ++x)
 #pragma unroll
-      for (int c = 0; c < c16; ++c) {
-        float cs[8], sn[8];
-#pragma unroll
-        for (int e = 0; e < 8; ++e) {
-          const float2 v = a[c * 8 + e];
-          cs[e] = v.x;
-          sn[e] = v.y;
-        }
-        uint4 ya, yb;
-        rope_rotate8(x[c], x[c + c16], cs, sn, ya, yb);
-        x[c] = ya;
-        x[c + c16] = yb;
-      }
-    } else {
-#pragma unroll
-      for (int c = 0; c < c8; ++c) x[c] = make_uint4(0u, 0u, 0u, 0u);
-    }
-#pragma unroll
-    for (int c = 0; c < c8; ++c) {
-      const int box = c >> 3;
-      const uint32_t pos = static_cast<uint32_t>(c & 7) ^ sw;
-      *reinterpret_cast<uint4 *>(line + box * (kBM * 128) + pos * 16) = x[c];
-    }
-  }
-  fence_proxy_async_smem();
+    for (int b = 0; b < C::kBoxes; ++b)
+      tma_load_3d_if(pred, smem + C::kQOff + x * C::kQBytes + b * (kBM * 128), &p.tm_qraw, bar, b * 64,
+                     head * G, (pair * 2 + x) * T);
 }
 
-// After the grid barrier: merge a share of the split rows (all 320 threads).
-// A row is read by a group of HD / 8 lanes (eight floats each); its slots'
-// LSEs give lse = log2 sum_k 2^lse_k and out = sum_k 2^(lse_k - lse) O_k.
+// The (cos, sin) of the tokens of this softmax warp's 32 rows (token r / G of
+// tile `wg` of the pair) into the warp's table `ang`: entry (token - w0) *
+// d/2 + i, tokens w0 .. w1 - 1.  Shared by the G heads of a token; only
+// __syncwarp orders it.  Returns the number of tokens held (at most
+// kAngEntries / (d/2)); rows of later tokens are rotated in a second batch.
 template <int HD>
-__device__ void step_merge(const StepParams &p, int T) {
+__device__ __forceinline__ int step_angles(const StepParams &p, float2 *ang, const TurnSplit *turns,
+                                           int pair, int wg, int row, int lane, int T, int b0, int w1) {
+  constexpr int half = HD / 2;
+  constexpr int per_batch = PairCfg<HD>::kAngEntries / half;
+  const int64_t tok0 = static_cast<int64_t>(pair * 2 + wg) * T;
+  const int bt = min(per_batch, w1 - b0);
+  __syncwarp();   // the previous batch's table is no longer read
+  for (int e = lane; e < bt * half; e += 32) {
+    const int tt = e / half;
+    const int i = e - tt * half;
+    float c, s;
+    rope_cos_sin(p.a.L + tok0 + b0 + tt, turns[i], c, s);
+    ang[e] = make_float2(c, s);
+  }
+  __syncwarp();
+  return bt;
+}
+
+// Rotate this thread's query row in place (its own 128-byte lines of the two
+// column boxes: 16-byte chunk c at position c ^ (r % 8)), with the angles of
+// its token (row `ang_row` of the table); ends with the proxy fence that lets
+// the tensor core read the rotated tile.
+template <int HD>
+__device__ __forceinline__ void step_rotate_row(uint8_t *qtile, const float2 *a, int row) {
+  constexpr int c16 = HD / 16;
+  uint8_t *line = qtile + row * 128;
+  const uint32_t sw = static_cast<uint32_t>(row & 7);
+  auto at = [&](int c) {
+    return reinterpret_cast<uint4 *>(line + (c >> 3) * (kBM * 128) + ((static_cast<uint32_t>(c & 7) ^ sw) * 16));
+  };
+  // a rolled loop: this runs once per piece, and a short body is fetched once
+#pragma unroll 1
+  for (int c = 0; c < c16; ++c) {
+    const uint4 xa = *at(c), xb = *at(c + c16);
+    float cs[8], sn[8];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+      const float2 v = a[c * 8 + e];
+      cs[e] = v.x;
+      sn[e] = v.y;
+    }
+    uint4 ya, yb;
+    rope_rotate8(xa, xb, cs, sn, ya, yb);
+    *at(c) = ya;
+    *at(c + c16) = yb;
+  }
+}
+
+// A softmax warp's share of a piece's query preparation: the angle tables of
+// its tokens, then (once the raw queries are in, `qraw_parity` of the
+// producer's barrier) the in-place rotation of its 32 rows, the proxy fence
+// and one arrival on q_full.  Returns false if the wait gave up.
+template <int HD>
+__device__ __noinline__ bool step_q_prep(const StepParams &p, uint8_t *qtile, float2 *ang, const TurnSplit *turns,
+                                         uint64_t *qraw_full, uint32_t qraw_parity, uint64_t *q_full,
+                                         volatile int *abort, int pair, int wg, int row, int lane, int T) {
+  constexpr int half = HD / 2;
+  const int G = p.a.group;
+  const int tr = row / G;
+  const int w0 = (row - lane) / G, w1 = (row - lane + 31) / G + 1;   // the warp's tokens
+  int b0 = w0;
+  int bt = step_angles<HD>(p, ang, turns, pair, wg, row, lane, T, b0, w1);
+  const bool got = mbar_wait(qraw_full, qraw_parity, abort, p.a.err, CSR_DEVERR_WAIT_TIMEOUT);
+  if (!__all_sync(0xffffffffu, got)) return false;
+  while (true) {
+    if (tr >= b0 && tr < b0 + bt) step_rotate_row<HD>(qtile, ang + (tr - b0) * half, row);
+    b0 += bt;
+    if (b0 >= w1) break;
+    bt = step_angles<HD>(p, ang, turns, pair, wg, row, lane, T, b0, w1);
+  }
+  fence_proxy_async_smem();
+  __syncwarp();
+  if (lane == 0) mbar_arrive(q_full);
+  return true;
+}
+
+// The merge of a fused launch, in batches of at most kMergeRows rows of one
+// unit.  Rows are numbered unit by unit over the split units (every unit of
+// the chunked form with more than one chunk, the split tail units otherwise);
+// each CTA takes a contiguous range [m0, m1) of them.
+// Partial row of slot k (0..cnt-1) and batch row r is base + k * kstride +
+// r * rstride; rows_major: the rows of the batch are contiguous over all its
+// slots (one bulk copy), else each slot's rows are (one copy per slot).
+struct MergeBatch {
+  int32_t unit, ra, R, cnt;
+  int64_t base, kstride, rstride;
+  bool rows_major;
+};
+
+__device__ __forceinline__ void merge_range(const StepSchedule &S, int64_t &m0, int64_t &m1) {
+  const int64_t n_mu = S.chunked ? S.n_units : S.n_tail;
+  const int64_t rows = n_mu * kPairRows;
+  const int64_t per = (rows + gridDim.x - 1) / gridDim.x;
+  m0 = static_cast<int64_t>(blockIdx.x) * per;
+  m1 = min(rows, m0 + per);
+}
+
+// The batch starting at merge row m (rows up to m1): cnt == 0 for a unit that
+// the attention loop wrote whole.
+template <int HD>
+__device__ __forceinline__ MergeBatch merge_batch(const StepParams &p, int T, int64_t m, int64_t m1) {
+  using C = PairCfg<HD>;
   const AttnParams &A = p.a;
   const StepSchedule &S = p.s;
-  constexpr int kLanes = HD / 8;
-  constexpr int kGroups = kPairThreads / kLanes;
-  const int grp = threadIdx.x / kLanes;
-  const int sl = threadIdx.x - grp * kLanes;
-  const int64_t n_merge_units = S.chunked ? S.n_units : S.n_tail;
-  const int64_t rows = n_merge_units * kPairRows;
-  const int64_t per = (rows + gridDim.x - 1) / gridDim.x;
-  const int64_t r0 = static_cast<int64_t>(blockIdx.x) * per;
-  const int64_t r1 = min(rows, r0 + per);
-  for (int64_t base = r0; base < r1; base += kGroups) {   // the same trip count on every lane
-    const int64_t m = base + grp;
-    int32_t unit = 0, r = 0, cnt = 0, s0 = 0, stride = 1;
-    if (m < r1) {
-      const int32_t mu = static_cast<int32_t>(m / kPairRows);
-      r = static_cast<int32_t>(m - static_cast<int64_t>(mu) * kPairRows);
-      if (S.chunked) {
-        unit = mu;
-        const int64_t kv = unit_iters(A.L, A.n, T, 2 * (unit / A.hkv) + 1);
-        const int32_t nk = static_cast<int32_t>((kv + S.chunk_tiles - 1) / S.chunk_tiles);
-        cnt = nk > 1 ? nk : 0;
-        s0 = unit;
-        stride = S.n_units;
+  const int32_t mu = static_cast<int32_t>(m / kPairRows);
+  MergeBatch b;
+  b.ra = static_cast<int32_t>(m - static_cast<int64_t>(mu) * kPairRows);
+  int64_t rmax = kPairRows - b.ra;
+  if (S.chunked) {
+    b.unit = mu;
+    const int64_t kv = unit_iters(A.L, A.n, T, 2 * (mu / A.hkv) + 1);
+    const int32_t nk = static_cast<int32_t>((kv + S.chunk_tiles - 1) / S.chunk_tiles);
+    b.cnt = nk > 1 ? nk : 0;
+    b.base = static_cast<int64_t>(mu) * kPairRows + b.ra;
+    b.kstride = static_cast<int64_t>(S.n_units) * kPairRows;
+    b.rstride = 1;
+    b.rows_major = false;
+  } else {
+    b.unit = S.n_units - S.n_tail + mu;
+    const int32_t s0 = S.tail_slot0[mu];
+    b.cnt = S.tail_slot0[mu + 1] - s0;
+    b.base = static_cast<int64_t>(s0) * kPairRows + static_cast<int64_t>(b.ra) * b.cnt;
+    b.kstride = 1;
+    b.rstride = b.cnt;
+    b.rows_major = true;
+    // one copy of whole rows: as many rows as the staging buffer holds
+    if (b.cnt > 0) rmax = min(rmax, static_cast<int64_t>(max(1, C::kMergeBuf / (b.cnt * HD * 4))));
+  }
+  b.R = static_cast<int32_t>(min(min(m1 - m, rmax), static_cast<int64_t>(C::kMergeRows)));
+  return b;
+}
+
+// After the grid barrier: merge this CTA's batches (all 320 threads).  Per
+// batch and slot batch: warp 9 issues one bulk copy per slot of the slot's
+// partial rows (consecutive in memory) into shared memory, all in flight at
+// once, while warps 0-8 find the row LSEs (lse = log2 sum_k 2^lse_k, one pass
+// over each row's slot LSEs kept in registers) and the weights 2^(lse_k -
+// lse); then every thread accumulates its (row, 4 columns) outputs from
+// shared memory and writes bf16 out and the natural-log lse.
+template <int HD>
+__device__ __noinline__ void step_merge(const StepParams &p, int T, uint8_t *smem, uint64_t *bar, MergeBatch first,
+                                        int64_t m, int64_t m1) {
+  using C = PairCfg<HD>;
+  const AttnParams &A = p.a;
+  constexpr int kRowBytes = HD * 4;
+  constexpr int kCols = HD / 4;                                   // 4-float columns per row
+  constexpr int kOwn = (C::kMergeRows * kCols + kPairThreads - 1) / kPairThreads;
+  float *buf = reinterpret_cast<float *>(smem);                   // [slot][row][HD]
+  float *row_lse = reinterpret_cast<float *>(smem + C::kAngOff);  // [kMergeRows]
+  float *wts = row_lse + C::kMergeRows;                           // [slot][row]
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  volatile int no_abort = 0;
+  uint32_t phase = 0;
+  bool use_first = true;
+  while (m < m1) {
+    const MergeBatch b = use_first ? first : merge_batch<HD>(p, T, m, m1);
+    use_first = false;
+    m += b.R;
+    if (b.cnt == 0) continue;   // the unit was written whole by the attention loop
+    const int32_t R = b.R, cnt = b.cnt;
+    auto prow = [&](int32_t k, int32_t r) { return b.base + k * b.kstride + r * b.rstride; };
+    // slots per copy round: all of them when whole rows are copied
+    const int32_t kb_max = b.rows_major ? cnt : max(1, min(C::kMergeBuf / (R * kRowBytes), C::kMergeWts / R));
+    float4 acc[kOwn];
+#pragma unroll
+    for (int j = 0; j < kOwn; ++j) acc[j] = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int32_t k0 = 0; k0 < cnt; k0 += kb_max) {
+      const int32_t kb = min(kb_max, cnt - k0);
+      if (tid == 9 * 32) {
+        fence_proxy_async_global();   // partials another SM wrote, now read by the async proxy
+        mbar_arrive_expect_tx(bar, static_cast<uint32_t>(kb * R * kRowBytes));
+        if (b.rows_major) {
+          // the batch's rows over all slots: one copy, buffer [row][slot][HD]
+          bulk_load_1d(buf, A.part_o + prow(0, 0) * HD, static_cast<uint32_t>(R * cnt * kRowBytes), bar);
+        } else {
+          for (int32_t k = 0; k < kb; ++k)   // buffer [slot][row][HD]
+            bulk_load_1d(buf + static_cast<int64_t>(k) * R * HD, A.part_o + prow(k0 + k, 0) * HD,
+                         static_cast<uint32_t>(R * kRowBytes), bar);
+        }
+      }
+      if (k0 == 0) {
+        // row LSEs and the first slot batch's weights, one row per warp of 0-8
+        if (warp < 9) {
+          for (int r = warp; r < R; r += 9) {
+            float v[4];
+            float mx = -CUDART_INF_F;
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+              const int k = lane + 32 * j;
+              v[j] = k < cnt ? ld_cg_f(A.part_lse + prow(k, r)) : -CUDART_INF_F;
+              mx = fmaxf(mx, v[j]);
+            }
+            for (int k = 128 + lane; k < cnt; k += 32) mx = fmaxf(mx, ld_cg_f(A.part_lse + prow(k, r)));
+#pragma unroll
+            for (int off = 16; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
+            const float m_use = mx == -CUDART_INF_F ? 0.f : mx;
+            float sum = 0.f;
+#pragma unroll
+            for (int j = 0; j < 4; ++j) sum += ex2_approx(v[j] - m_use);
+            for (int k = 128 + lane; k < cnt; k += 32) sum += ex2_approx(ld_cg_f(A.part_lse + prow(k, r)) - m_use);
+#pragma unroll
+            for (int off = 16; off > 0; off >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, off);
+            const float lr = sum > 0.f ? m_use + log2f(sum) : -CUDART_INF_F;
+            if (lane == 0) row_lse[r] = lr;
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+              const int k = lane + 32 * j;
+              if (k < kb) wts[k * R + r] = lr == -CUDART_INF_F ? 0.f : ex2_approx(v[j] - lr);
+            }
+            for (int k = 128 + lane; k < kb; k += 32)
+              wts[k * R + r] = lr == -CUDART_INF_F ? 0.f : ex2_approx(ld_cg_f(A.part_lse + prow(k, r)) - lr);
+          }
+        }
       } else {
-        unit = S.n_units - S.n_tail + mu;
-        s0 = S.tail_slot0[mu];
-        cnt = S.tail_slot0[mu + 1] - s0;
-      }
-    }
-    const int32_t pair = unit / A.hkv;
-    const int32_t head = unit - pair * A.hkv;
-    const int32_t tile = pair * 2 + r / kBM;
-    const int32_t rr = r % kBM;
-    const int64_t t = static_cast<int64_t>(tile) * T + rr / A.group;
-    const bool valid = cnt > 0 && tile < A.n_tiles && t < A.n;
-    auto prow = [&](int i) { return static_cast<int64_t>(s0 + i * stride) * kPairRows + r; };
-    float mx = -CUDART_INF_F;
-    if (valid)
-      for (int i = sl; i < cnt; i += kLanes) mx = fmaxf(mx, ld_cg_f(A.part_lse + prow(i)));
-#pragma unroll
-    for (int off = kLanes / 2; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off, kLanes));
-    const float m_use = mx == -CUDART_INF_F ? 0.f : mx;
-    float sum = 0.f;
-    if (valid)
-      for (int i = sl; i < cnt; i += kLanes) sum += ex2_approx(ld_cg_f(A.part_lse + prow(i)) - m_use);
-#pragma unroll
-    for (int off = kLanes / 2; off > 0; off >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, off, kLanes);
-    if (!valid) continue;
-    const float lse2 = sum > 0.f ? m_use + log2f(sum) : -CUDART_INF_F;
-    float acc[8];
-#pragma unroll
-    for (int e = 0; e < 8; ++e) acc[e] = 0.f;
-    if (sum > 0.f) {
-      int i = 0;
-      for (; i + 4 <= cnt; i += 4) {   // four partial rows in flight
-        float4 v[4][2];
-        float w[4];
-#pragma unroll
-        for (int u = 0; u < 4; ++u) {
-          const float *src = A.part_o + prow(i + u) * HD + sl * 8;
-          v[u][0] = ld_cg_f4(src);
-          v[u][1] = ld_cg_f4(src + 4);
-          w[u] = ld_cg_f(A.part_lse + prow(i + u));
-        }
-#pragma unroll
-        for (int u = 0; u < 4; ++u) {
-          const float wt = ex2_approx(w[u] - lse2);
-          acc[0] = fmaf(wt, v[u][0].x, acc[0]);
-          acc[1] = fmaf(wt, v[u][0].y, acc[1]);
-          acc[2] = fmaf(wt, v[u][0].z, acc[2]);
-          acc[3] = fmaf(wt, v[u][0].w, acc[3]);
-          acc[4] = fmaf(wt, v[u][1].x, acc[4]);
-          acc[5] = fmaf(wt, v[u][1].y, acc[5]);
-          acc[6] = fmaf(wt, v[u][1].z, acc[6]);
-          acc[7] = fmaf(wt, v[u][1].w, acc[7]);
+        for (int i = tid; i < kb * R; i += kPairThreads) {
+          const int k = i / R, r = i - k * R;
+          const float lr = row_lse[r];
+          wts[i] = lr == -CUDART_INF_F ? 0.f : ex2_approx(ld_cg_f(A.part_lse + prow(k0 + k, r)) - lr);
         }
       }
-      for (; i < cnt; ++i) {
-        const float *src = A.part_o + prow(i) * HD + sl * 8;
-        const float4 a = ld_cg_f4(src), b = ld_cg_f4(src + 4);
-        const float wt = ex2_approx(ld_cg_f(A.part_lse + prow(i)) - lse2);
-        acc[0] = fmaf(wt, a.x, acc[0]);
-        acc[1] = fmaf(wt, a.y, acc[1]);
-        acc[2] = fmaf(wt, a.z, acc[2]);
-        acc[3] = fmaf(wt, a.w, acc[3]);
-        acc[4] = fmaf(wt, b.x, acc[4]);
-        acc[5] = fmaf(wt, b.y, acc[5]);
-        acc[6] = fmaf(wt, b.z, acc[6]);
-        acc[7] = fmaf(wt, b.w, acc[7]);
+      __syncthreads();
+      // wait for the copies even after an abort elsewhere (none may still be
+      // writing this CTA's shared memory when it exits); bounded all the same
+      mbar_wait(bar, phase & 1, &no_abort, A.err, CSR_DEVERR_WAIT_TIMEOUT);
+      ++phase;
+#pragma unroll
+      for (int j = 0; j < kOwn; ++j) {
+        const int idx = tid + j * kPairThreads;
+        if (idx < R * kCols) {
+          const int r = idx / kCols, c = idx - r * kCols;
+          for (int k = 0; k < kb; ++k) {
+            const float w = wts[k * R + r];
+            const int64_t bi = b.rows_major ? static_cast<int64_t>(r) * kb + k : static_cast<int64_t>(k) * R + r;
+            const float4 v = reinterpret_cast<const float4 *>(buf + bi * HD)[c];
+            acc[j].x = fmaf(w, v.x, acc[j].x);
+            acc[j].y = fmaf(w, v.y, acc[j].y);
+            acc[j].z = fmaf(w, v.z, acc[j].z);
+            acc[j].w = fmaf(w, v.w, acc[j].w);
+          }
+        }
+      }
+      __syncthreads();   // the buffer and weights are rewritten by the next slot batch
+    }
+    const int32_t pair = b.unit / A.hkv;
+    const int32_t head = b.unit - pair * A.hkv;
+#pragma unroll
+    for (int j = 0; j < kOwn; ++j) {
+      const int idx = tid + j * kPairThreads;
+      if (idx < R * kCols) {
+        const int r = idx / kCols, c = idx - r * kCols;
+        const int rr = (b.ra + r) % kBM;
+        const int tile = pair * 2 + (b.ra + r) / kBM;
+        const int64_t t = static_cast<int64_t>(tile) * T + rr / A.group;
+        if (tile < A.n_tiles && t < A.n) {
+          const int hq_idx = head * A.group + rr % A.group;
+          uint16_t *dst = A.out + (t * A.hq + hq_idx) * HD + c * 4;
+          *reinterpret_cast<uint2 *>(dst) = make_uint2(pack_bf16x2(acc[j].x, acc[j].y),
+                                                       pack_bf16x2(acc[j].z, acc[j].w));
+          if (c == 0 && A.lse) A.lse[static_cast<int64_t>(hq_idx) * A.n + t] = row_lse[r] * 0.69314718055994531f;
+        }
       }
     }
-    const int hq_idx = head * A.group + rr % A.group;
-    uint16_t *dst = A.out + (t * A.hq + hq_idx) * HD + sl * 8;
-    *reinterpret_cast<uint4 *>(dst) = make_uint4(pack_bf16x2(acc[0], acc[1]), pack_bf16x2(acc[2], acc[3]),
-                                                 pack_bf16x2(acc[4], acc[5]), pack_bf16x2(acc[6], acc[7]));
-    if (sl == 0 && A.lse) A.lse[static_cast<int64_t>(hq_idx) * A.n + t] = lse2 * 0.69314718055994531f;
+    __syncthreads();   // row_lse is rewritten by the next batch
   }
 }
 
@@ -605,11 +788,14 @@ __global__ void __launch_bounds__(kPairThreads, 1)
       mbar_init(&bars->o_free[w], 4);
     }
     mbar_init(&bars->drain, 1);
+    mbar_init(&bars->merge_full, 1);
+    mbar_init(&bars->qraw_full, 1);
     bars->abort = 0;
     fence_barrier_init();
   }
   if (warp == 8 && lane == 0) {
     if constexpr (!kStep) tma_prefetch_desc(&A.tm_q);
+    if constexpr (kStep) tma_prefetch_desc(&p.tm_qraw);
     tma_prefetch_desc(&A.tm_k);
     tma_prefetch_desc(&A.tm_v);
   }
@@ -617,10 +803,22 @@ __global__ void __launch_bounds__(kPairThreads, 1)
     tmem_alloc(&bars->tmem_base, C::kTmemCols);
     tmem_relinquish();
   }
+  TurnSplit *turns = reinterpret_cast<TurnSplit *>(smem + C::kTurnOff);
+  int32_t *ids_s = reinterpret_cast<int32_t *>(smem + C::kIdsOff);
+  if constexpr (kStep) {
+    // RoPE frequencies and the new page ids into shared memory (lanes read
+    // them at different indices; parameter reads would serialise)
+    if (threadIdx.x < HD / 2) turns[threadIdx.x] = p.inv_turns[threadIdx.x];
+    for (int i = threadIdx.x; i < min(p.n_ids, C::kSmemIds); i += kPairThreads) ids_s[i] = p.ids[i];
+  }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
-  pdl_wait();   // queries, keys and the page table come from (or are still read by) the previous kernel
+  // The cache, the page table and the partial buffers may still be read or
+  // written by the previous kernel: every role waits for it before its first
+  // access to them.  The fused form's softmax warps first rotate their first
+  // queries (inputs of this call, not written by the previous kernel).
+  if constexpr (!kStep) pdl_wait();
   const uint32_t tmem = bars->tmem_base;
   volatile int *abort = &bars->abort;
   auto walk = make_walker(p);
@@ -637,8 +835,28 @@ __global__ void __launch_bounds__(kPairThreads, 1)
     uint32_t q_round = 0, k_it = 0, v_it = 0;
     bool ok = true;
     bool appended = false;   // fused form: the launch's new keys are in the cache
-    while (ok && walk.next(p, T, seg)) {
-      if constexpr (!kStep) {
+    bool pending = false;
+    if constexpr (kStep) {
+      // the first piece's raw queries before waiting for the previous kernel
+      // (they are inputs of this call); then every cache access waits
+      pending = walk.next(p, T, seg);
+      if (pending) {
+        step_qraw_issue<HD>(leader, p, smem, &bars->qraw_full, seg.head, seg.pair, T);
+        q_round = 1;
+      }
+      pdl_wait();
+    }
+    while (ok && (pending || walk.next(p, T, seg))) {
+      if constexpr (kStep) {
+        if (!pending) {
+          ok = __all_sync(0xffffffffu, mbar_wait(&bars->q_empty, (q_round - 1) & 1, abort, A.err,
+                                                 CSR_DEVERR_WAIT_TIMEOUT));
+          if (!ok) break;
+          step_qraw_issue<HD>(leader, p, smem, &bars->qraw_full, seg.head, seg.pair, T);
+          ++q_round;
+        }
+        pending = false;
+      } else {
         if (q_round > 0)
           ok = __all_sync(0xffffffffu, mbar_wait(&bars->q_empty, (q_round - 1) & 1, abort, A.err,
                                                  CSR_DEVERR_WAIT_TIMEOUT));
@@ -656,20 +874,17 @@ __global__ void __launch_bounds__(kPairThreads, 1)
       for (int64_t jb = seg.j0; ok && jb < seg.j1; jb += tiles_per_block) {
         const int64_t je = min(jb + tiles_per_block, seg.j1);
         const int npages = static_cast<int>(je - jb) * ppt;
-        if constexpr (kStep) {
-          // key tiles at or past the page holding position L hold the new keys
-          if (!appended && je * ppt > p.new_lp) {
-            if (lane == 0) ok = wait_counter(p.sync, p.append_target, A.err, abort);
-            ok = __shfl_sync(0xffffffffu, ok, 0);
-            if (!ok) break;
-            fence_proxy_async_global();
-            appended = true;
-          }
-        }
         __syncwarp();
         for (int i = lane; i < npages; i += 32) {
           const int64_t lp = jb * ppt + i;
-          int32_t phys = (lp < A.n_pages_valid) ? A.page_table[lp] : A.page_table[0];
+          int32_t phys;
+          if constexpr (kStep) {
+            // the launch's new pages come from its id list: staging never
+            // waits for the append, only the TMA of the new keys does
+            phys = (lp < A.n_pages_valid) ? step_page(p, ids_s, lp) : A.page_table[0];
+          } else {
+            phys = (lp < A.n_pages_valid) ? A.page_table[lp] : A.page_table[0];
+          }
           if (phys < 0 || phys >= A.pool_pages) {
             atomicOr(A.err, CSR_DEVERR_BAD_PAGE);
             phys = 0;
@@ -678,6 +893,16 @@ __global__ void __launch_bounds__(kPairThreads, 1)
         }
         __syncwarp();
         for (int64_t j = jb; j < je; ++j) {
+          if constexpr (kStep) {
+            // key tiles at or past the page holding position L hold the new keys
+            if (!appended && (j + 1) * ppt > p.new_lp) {
+              if (lane == 0) ok = wait_counter(p.sync, p.append_target, A.err, abort);
+              ok = __shfl_sync(0xffffffffu, ok, 0);
+              if (!ok) break;
+              fence_proxy_async_global();
+              appended = true;
+            }
+          }
           const int32_t *phys = stage + static_cast<int>(j - jb) * ppt;
           const int ks = k_it % C::kStages;
           ok = __all_sync(0xffffffffu, mbar_wait(&bars->k_empty[ks], ((k_it / C::kStages) & 1) ^ 1,
@@ -699,7 +924,7 @@ __global__ void __launch_bounds__(kPairThreads, 1)
       }
     }
     if (!ok && lane == 0) {
-      if (!kStep && q_round > 0) drain_wait(&bars->q_full, (q_round - 1) & 1);
+      if (q_round > 0) drain_wait(kStep ? &bars->qraw_full : &bars->q_full, (q_round - 1) & 1);
       for (uint32_t i = (k_it > C::kStages ? k_it - C::kStages : 0); i < k_it; ++i)
         drain_wait(&bars->k_full[i % C::kStages], (i / C::kStages) & 1);
       for (uint32_t i = (v_it > C::kStages ? v_it - C::kStages : 0); i < v_it; ++i)
@@ -717,6 +942,19 @@ __global__ void __launch_bounds__(kPairThreads, 1)
     uint32_t q_round = 0, k_it = 0, v_it = 0, seg_n = 0;
     uint32_t pv_n[2] = {0, 0};
     bool ok = true;
+    if constexpr (kStep) {
+      pdl_wait();
+      if (p.append_by_mma) {
+        // few new tokens: this warp appends the CTA's share while the softmax
+        // warps rotate the first queries, then arrives once for the CTA
+        step_append<HD>(p, turns, ids_s, lane, 32);
+        __syncwarp();
+        if (lane == 0) {
+          __threadfence();
+          red_release_gpu_add(p.sync, 1u);
+        }
+      }
+    }
     auto wait = [&](uint64_t *bar, uint32_t parity) {
       if (ok)
         ok = __all_sync(0xffffffffu, mbar_wait(bar, parity, abort, A.err, CSR_DEVERR_WAIT_TIMEOUT));
@@ -805,32 +1043,39 @@ __global__ void __launch_bounds__(kPairThreads, 1)
     const uint32_t o_col = C::kOCol + wg * HD;
     uint32_t s_it = 0, seg_n = 0;
     bool ok = true;
+    bool pending = false;   // fused form: the first piece, taken before the loop
+    uint8_t *qtile = smem + C::kQOff + wg * C::kQBytes;
+    float2 *ang = reinterpret_cast<float2 *>(smem + C::kAngOff) + warp * C::kAngEntries;
     if constexpr (kStep) {
-      // this CTA's share of the new keys/values, then one arrival per CTA
-      step_append<HD>(p, threadIdx.x);
-      named_sync(3, 256);
-      if (threadIdx.x == 0) {
-        __threadfence();
-        red_release_gpu_add(p.sync, 1u);
+      // the first piece's queries before waiting for the previous kernel
+      pending = walk.next(p, T, seg);
+      if (pending && !step_q_prep<HD>(p, qtile, ang, turns, &bars->qraw_full, 0, &bars->q_full, abort,
+                                      seg.pair, wg, row, lane, T))
+        ok = false;
+      pdl_wait();
+      if (!p.append_by_mma) {
+        // this CTA's share of the new keys/values, then one arrival per CTA
+        // (every softmax thread gets here exactly once)
+        step_append<HD>(p, turns, ids_s, threadIdx.x, 256);
+        named_sync(3, 256);
+        if (threadIdx.x == 0) {
+          __threadfence();
+          red_release_gpu_add(p.sync, 1u);
+        }
       }
     }
-    while (ok && walk.next(p, T, seg)) {
+    while (ok && (pending || walk.next(p, T, seg))) {
+      pending = false;
       if constexpr (kStep) {
-        // the unit's queries, rotated into this warpgroup's Q tile once the
-        // previous piece's last score MMA has read the old ones
         if (seg_n > 0) {
-          const bool got = mbar_wait(&bars->q_empty, (seg_n - 1) & 1, abort, A.err,
-                                     CSR_DEVERR_WAIT_TIMEOUT);
-          if (!__all_sync(0xffffffffu, got)) {
+          // the unit's queries, rotated in place once the producer's raw copy
+          // (issued after the previous piece's last score MMA) is in
+          if (!step_q_prep<HD>(p, qtile, ang, turns, &bars->qraw_full, seg_n & 1, &bars->q_full, abort,
+                               seg.pair, wg, row, lane, T)) {
             ok = false;
             break;
           }
         }
-        step_prep_q<HD>(p, smem + C::kQOff + wg * C::kQBytes,
-                        reinterpret_cast<float2 *>(smem + C::kAngOff) + warp * C::kAngEntries,
-                        seg.head, seg.pair, wg, row, lane, T);
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&bars->q_full);
       }
       const int tile = seg.pair * 2 + wg;
       const int64_t t = static_cast<int64_t>(tile) * T + row / A.group;
@@ -940,7 +1185,7 @@ __global__ void __launch_bounds__(kPairThreads, 1)
           if (A.lse) A.lse[static_cast<int64_t>(hq_idx) * A.n + t] = lse2 * 0.69314718055994531f;
         }
       } else {
-        const int64_t base = static_cast<int64_t>(seg.slot) * kPairRows + wg * kBM + row;
+        const int64_t base = seg.pbase + static_cast<int64_t>(wg * kBM + row) * seg.pstride;
         // the partial buffer is 256-byte aligned and rows are HD floats: 32-byte stores
         float *dst = A.part_o + base * HD;
 #pragma unroll
@@ -969,15 +1214,23 @@ __global__ void __launch_bounds__(kPairThreads, 1)
   }
   if constexpr (kStep) {
     if (p.s.n_slots > 0) {
-      // grid barrier (every CTA is resident: cooperative launch), then the merge
+      // grid barrier (every CTA is resident: cooperative launch), then the
+      // merge; every thread works out its first batch (the schedule's
+      // parameters) while the barrier is pending
       if (threadIdx.x == 0) {
         __threadfence();
         red_release_gpu_add(p.sync + 1, 1u);
+      }
+      int64_t m0, m1;
+      merge_range(p.s, m0, m1);
+      MergeBatch first{};
+      if (m0 < m1) first = merge_batch<HD>(p, T, m0, m1);
+      if (threadIdx.x == 0) {
         wait_counter(p.sync + 1, p.barrier_target, A.err, nullptr);
         __threadfence();
       }
       __syncthreads();
-      step_merge<HD>(p, T);
+      step_merge<HD>(p, T, smem, &bars->merge_full, first, m0, m1);
     }
   }
 }

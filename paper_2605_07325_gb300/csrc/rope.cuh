@@ -26,8 +26,10 @@
 namespace csr {
 
 // Reduced turn count of position pos (< 2^24) for the split frequency w.
+// The position is converted from 32 bits: a 64-bit integer conversion costs
+// several times the rest of the angle on this GPU.
 __device__ __forceinline__ float rope_turns(int64_t pos, TurnSplit w) {
-  const float x = static_cast<float>(pos);          // exact below 2^24
+  const float x = __int2float_rn(static_cast<int32_t>(pos));   // exact below 2^24
   const float p = __fmul_rn(x, w.hi);
   const float e = __fmaf_rn(x, w.hi, -p);           // x * w.hi = p + e exactly
   const float frac = __fsub_rn(p, rintf(p));        // exact: p and its nearest integer

@@ -51,10 +51,17 @@ def test_single_token_prefix_returns_v(libcsr):
     p.device_clean()
 
 
+# Foreground paths: one cooperative launch of the fused kernel, or three
+# chained launches (the library picks by the call's work; the flags force).
+PATHS = {"fused": 0x2, "three": 0x4}
+
+
+@pytest.mark.parametrize("path", sorted(PATHS))
 @pytest.mark.parametrize("shape", [C1, C2], ids=["d64_p16_g4", "d128_p64_g16"])
 @pytest.mark.parametrize("chunk_tiles", [0, 2])
-def test_ragged_sizes(libcsr, shape, chunk_tiles):
-    p = Pair(shape, pool_pages=128, max_seq=4096, max_new=512, fg_chunk_tiles=chunk_tiles)
+def test_ragged_sizes(libcsr, shape, chunk_tiles, path):
+    p = Pair(shape, pool_pages=128, max_seq=4096, max_new=512, fg_chunk_tiles=chunk_tiles,
+             flags=PATHS[path])
     p.init_static(p.blk(10, 37))
     for i, n in enumerate([1, 129, 64, 300, 17]):
         p.append(p.blk(11 + i, n))
@@ -68,13 +75,16 @@ def test_ragged_sizes(libcsr, shape, chunk_tiles):
     p.device_clean()
 
 
+@pytest.mark.parametrize("path", sorted(PATHS))
 @pytest.mark.parametrize("num_ctas,chunk_tiles", [(1, 0), (3, 1), (7, 2), (19, 3), (64, 5),
-                                                   (152, 1), (0, 4)])
-def test_split_kv_partials_any_grid(libcsr, num_ctas, chunk_tiles):
+                                                   (152, 1), (0, 4), (0, 0), (5, 0)])
+def test_split_kv_partials_any_grid(libcsr, num_ctas, chunk_tiles, path):
     """Forced CTA counts and key-chunk lengths: every split into items (down to
-    one 128-key tile per item) must merge back to the oracle."""
+    one 128-key tile per item) must merge back to the oracle, on both paths
+    (chunk 0: the fused kernel's rounds + tail schedule, the three-launch
+    path's cost model)."""
     p = Pair(C2, pool_pages=256, max_seq=8192, max_new=1024, num_ctas=num_ctas,
-             fg_chunk_tiles=chunk_tiles)
+             fg_chunk_tiles=chunk_tiles, flags=PATHS[path])
     p.init_static(p.blk(30, 700))
     p.append(p.blk(31, 1000))
     p.append(p.blk(32, 33))
@@ -187,15 +197,21 @@ def test_8k_context_step(libcsr):
 
 
 def test_launch_count_reported(libcsr):
-    """A foreground call is one launch of the fused kernel (RoPE + append,
-    attention, merge), split or not."""
-    p = Pair(C1, pool_pages=64, max_seq=2048, max_new=256)
+    """A fused foreground call is one launch (RoPE + append, attention, merge),
+    split or not; the three-launch path runs RoPE/append and attention, plus
+    the merge when the keys were split."""
+    p = Pair(C1, pool_pages=64, max_seq=2048, max_new=256, flags=PATHS["fused"])
     before = p.ctx.kernel_launches()
     p.init_static(p.blk(70, 100))
     assert p.ctx.kernel_launches() - before == 1
     p.append(p.blk(71, 37))
     assert p.ctx.kernel_launches() - before == 2
     p.device_clean()
+    q = Pair(C1, pool_pages=64, max_seq=2048, max_new=256, flags=PATHS["three"])
+    before = q.ctx.kernel_launches()
+    q.init_static(q.blk(70, 100))
+    assert 2 <= q.ctx.kernel_launches() - before <= 3
+    q.device_clean()
 
 
 def test_rewind_then_append_matches_never_appended(libcsr):
@@ -219,13 +235,15 @@ def test_rewind_then_append_matches_never_appended(libcsr):
     a.device_clean()
 
 
+@pytest.mark.parametrize("path", sorted(PATHS))
 @pytest.mark.parametrize("shape", [C1, C2], ids=["d64_p16_g4", "d128_p64_g16"])
 @pytest.mark.parametrize("chunk_tiles", [0, 2])
-def test_fused_step_matches_oracle(libcsr, shape, chunk_tiles):
+def test_fused_step_matches_oracle(libcsr, shape, chunk_tiles, path):
     """csr_append_chunk_attend_suffix: the chunk's outputs equal those of
     append_chunk and the suffix's those of attend_suffix on the same cache;
     the layout after the truncation equals the two-call layout."""
-    p = Pair(shape, pool_pages=160, max_seq=4096, max_new=1024, fg_chunk_tiles=chunk_tiles)
+    p = Pair(shape, pool_pages=160, max_seq=4096, max_new=1024, fg_chunk_tiles=chunk_tiles,
+             flags=PATHS[path])
     p.init_static(p.blk(40, 77))
     for i, (nc, ns) in enumerate([(1, 1), (37, 100), (129, 300), (256, 512)]):
         p.fused(p.blk(41 + i, nc + ns), nc)
@@ -237,14 +255,16 @@ def test_fused_step_matches_oracle(libcsr, shape, chunk_tiles):
     p.device_clean()
 
 
+@pytest.mark.parametrize("path", sorted(PATHS))
 @pytest.mark.parametrize("shape", [C1, C2], ids=["d64_p16_g4", "d128_p64_g16"])
 @pytest.mark.parametrize("chunk_tiles", [1, 2, 3, 9])
-def test_merge_many_chunks_per_row(libcsr, shape, chunk_tiles):
+def test_merge_many_chunks_per_row(libcsr, shape, chunk_tiles, path):
     """Long context, short blocks, short key chunks: rows merged from up to 67
     partials (the merge spreads such rows over several lane groups, and above
     64 partials takes its general path)."""
     pages = 16384 // shape["P"] + 64
-    p = Pair(shape, pool_pages=pages, max_seq=16384, max_new=4096, fg_chunk_tiles=chunk_tiles)
+    p = Pair(shape, pool_pages=pages, max_seq=16384, max_new=4096, fg_chunk_tiles=chunk_tiles,
+             flags=PATHS[path])
     p.init_static(p.blk(70, 4000), compare=False)
     p.append(p.blk(71, 4000), compare=False)
     p.append(p.blk(72, 500))
