@@ -184,9 +184,53 @@ def _oracle_step_sample(k_cache, v_cache, n_chunk: int, n_suffix: int, seed: int
     return secs, sampled, full
 
 
+def _oracle_config_tiny() -> float:
+    """The tiny correctness case in full through the oracle (8 q / 2 kv heads,
+    d 64, page 16, base 1e4): a 256-token prefix, three 256-token chunks, a
+    32-token suffix, truncate, one more chunk, the suffix again; every output
+    computed.  Returns seconds."""
+    from oracle import oracle as orc
+    from paper_2605_07325_gb300 import synth
+    t0 = time.perf_counter()
+    o = orc.OracleCSR(8, 2, 64, 16, 1e4, pool_pages=256)
+    blk = lambda seed, n: synth.block(seed, n, 8, 2, 64).f64()
+    o.init_static(*blk(0, 256))
+    for i in range(3):
+        o.append_chunk(*blk(1 + i, 256))
+    o.attend_suffix(*blk(100, 32))
+    o.truncate_suffix()
+    o.append_chunk(*blk(4, 256))
+    o.attend_suffix(*blk(101, 32))
+    o.truncate_suffix()
+    return time.perf_counter() - t0
+
+
+def _oracle_config_8k() -> float:
+    """One step of the 8K-context case in full through the oracle (64 q / 4 kv
+    heads, d 128, page 64, base 1e6): over a 2,048-token prefix + 48 chunks
+    of 128 (cache bookkeeping only while filling), append a 128-token chunk,
+    attend a 64-token suffix, truncate.  Returns the step's seconds."""
+    from oracle import oracle as orc
+    from paper_2605_07325_gb300 import synth
+    o = orc.OracleCSR(HQ, HKV, D, P, BASE, pool_pages=(8192 + 256) // P + 8)
+    blk = lambda seed, n: synth.block(seed, n, HQ, HKV, D).f64()
+    o.attend = False
+    o.init_static(*blk(200, 2048))
+    for i in range(48):
+        o.append_chunk(*blk(201 + i, 128))
+    o.attend = True
+    chunk, suffix = blk(300, 128), blk(301, 64)
+    t0 = time.perf_counter()
+    o.append_chunk(*chunk)
+    o.attend_suffix(*suffix)
+    o.truncate_suffix()
+    return time.perf_counter() - t0
+
+
 def cpu_baseline(target_s: float = 15.0):
-    """The oracle as it stands, on this host's cores, on a bounded sample of
-    the step, scaled by query-key pairs to microseconds per layer-step."""
+    """The oracle as it stands, on this host's cores: the 120K step on a
+    bounded sample scaled by query-key pairs to microseconds per layer-step
+    (extrapolated), and the tiny and 8K cases in full."""
     from oracle import oracle as orc
     k, v = _oracle_cache()
     s1, p1, full = _oracle_step_sample(k, v, 1, 1, seed=11)       # calibration
@@ -196,14 +240,30 @@ def cpu_baseline(target_s: float = 15.0):
     n_s = min(SUFFIX, tokens - n_c)
     secs, pairs, full = _oracle_step_sample(k, v, n_c, n_s, seed=12)
     us = secs * full / pairs * 1e6
-    return {"value": us, "unit": UNIT, "cores": orc.default_threads(), "kind": "oracle",
+    cores = orc.default_threads()
+    tiny_s = _oracle_config_tiny()
+    step8k_s = _oracle_config_8k()
+    return {"value": us, "unit": UNIT, "cores": cores, "kind": "oracle",
+            "extrapolated": True, "sampled_fraction": pairs / full, "sample_seconds": secs,
             "sample": (f"fp64 C oracle: RoPE of the step's 768 new keys + attention of {n_c} chunk "
                        f"and {n_s} suffix query tokens (all 64 heads) over 122,880+ keys, "
-                       f"{secs:.1f} s, scaled by query-key pairs to the full step")}
+                       f"{secs:.1f} s, scaled by query-key pairs to the full step"),
+            "configs": [
+                {"config": "tiny correctness case: full session (prefix 256, 3 chunks of 256, "
+                           "suffix 32, truncate, chunk, suffix), 8 q / 2 kv heads, d 64",
+                 "seconds": tiny_s, "cores": cores, "extrapolated": False},
+                {"config": "8K-context step: append 128 + attend 64 + truncate over 8,192 cached, "
+                           "64 q / 4 kv heads, d 128", "us_per_step": step8k_s * 1e6,
+                 "cores": cores, "extrapolated": False},
+                {"config": WORKLOAD_NAME, "us_per_step": us, "cores": cores, "extrapolated": True,
+                 "sampled_fraction": pairs / full}]}
 
 
 def run_reference(args):
-    """--impl reference: the fp64 oracle timed alone on the host cores."""
+    """--impl reference: the fp64 oracle timed alone on the host cores.  Each
+    step runs a bounded sample of the 120K step; `value` scales it by
+    query-key pairs to the whole step (extrapolated: true), `ms_per_step` is
+    the time a step actually took."""
     from oracle import oracle as orc
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
@@ -213,21 +273,27 @@ def run_reference(args):
     budget = 150.0 / max(1, args.steps + args.warmup)              # seconds per step
     tokens = max(2, int(budget / (s1 / p1 * (L0 + 300))))
     n_c, n_s = tokens // 2, tokens - tokens // 2
-    vals = []
+    vals, spent, fracs = [], [], []
     for i in range(args.warmup + args.steps):
         secs, pairs, full = _oracle_step_sample(k, v, n_c, n_s, seed=100 + i)
         if i >= args.warmup:
             vals.append(secs * full / pairs * 1e6)
+            spent.append(secs)
+            fracs.append(pairs / full)
     value = statistics.mean(vals)
     cores = orc.default_threads()
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT,
             "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
-            "ms_per_step": value / 1e3, "higher_is_better": False, "scaling": "weak",
+            "ms_per_step": statistics.mean(spent) * 1e3, "higher_is_better": False, "scaling": "weak",
             "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "extrapolated": True, "sampled_fraction": statistics.mean(fracs),
             "config": {"workload": WORKLOAD_NAME},
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
-                             "sample": f"per step: {n_c} chunk + {n_s} suffix query tokens, "
-                                       "scaled by query-key pairs"},
+                             "extrapolated": True, "sampled_fraction": statistics.mean(fracs),
+                             "sample": f"per step: {n_c} chunk + {n_s} suffix query tokens "
+                                       f"({statistics.mean(spent):.2f} s actually spent per step, "
+                                       "ms_per_step), scaled by query-key pairs to the whole step "
+                                       "(value)"},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
     return 0
@@ -487,7 +553,8 @@ def run_asr(args):
     cfg = csr.make_config(HQ, HKV, D, P, BASE, max_new_tokens=PREFIX, pool_pages=pool_pages,
                           max_seq_tokens=n_max, cap_tokens=cap,
                           evict_tokens=evict, n_catchup=0,
-                          rebuild_tiles_per_cta=args.asr_rebuild_tiles)
+                          rebuild_tiles_per_cta=args.asr_rebuild_tiles,
+                          flags=csr.FLAG_UNPACED_REBUILD if args.asr_unpaced else 0)
     fg = torch.cuda.Stream(device=dev, priority=-1)     # high priority
     lo = torch.cuda.Stream(device=dev, priority=0)      # low priority (rebuild, R_2)
     gen = torch.Generator(device=dev).manual_seed(4321)
@@ -588,6 +655,8 @@ def run_asr(args):
         "step_calls": ("csr_append_chunk_attend_suffix + csr_truncate_suffix" if fused else
                        "csr_append_chunk + csr_attend_suffix + csr_truncate_suffix"),
         "cadence_hz": args.asr_cadence_hz, "rebuild_tiles_per_cta": args.asr_rebuild_tiles or 16,
+        "rebuild_pacing": "all tasks at once" if args.asr_unpaced else
+                          "one task in flight, started after the foreground work",
         "cycles": cycles, "steps": step,
         "steps_during_rebuild": len(dur),
         "fg_ms_host": {"p50_outside": pct(out, 50), "p99_outside": pct(out, 99),
@@ -611,6 +680,12 @@ def run_asr(args):
         line["viability"] = {"x_dot_tokens_per_s": x_dot, "dt_mem_s": dt_mem,
                              "dt_rebuild_max_s": max(rebuilds),
                              "holds": max(rebuilds) <= dt_mem and peak_len <= n_max}
+        # the library's own check (csr_check_viability) for an eviction started
+        # now, from the rebuild pace it observed on the last reconciliation
+        try:
+            line["viability_library"] = ctx.check_viability(evict, x_dot)
+        except csr.CsrError as e:
+            line["viability_library"] = {"error": str(e)}
     print(json.dumps(line), flush=True)
     ctx.close()
     return 0 if layout_ok and flags == 0 else 1
@@ -647,7 +722,7 @@ def run_unordered(args):
         left -= n
     times = []
     with torch.cuda.stream(stream):
-        for step in range(args.warmup + max(1, args.steps // 100)):
+        for step in range(args.warmup + max(5, args.steps // 100)):
             ctx = csr.Context(cfg, device=str(dev), stream=stream)
             stream.synchronize()
             e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -667,6 +742,8 @@ def run_unordered(args):
     line = {"workload": "unordered baseline: full causal prefill of 123,648 tokens per step, "
                         "64 q / 4 kv heads, d 128, page 64, bf16, 1 layer",
             "unordered_ms_per_layer": unordered_ms, "steps": len(times),
+            "unordered_ms_min": min(times), "unordered_ms_max": max(times),
+            "unordered_ms_stdev": statistics.stdev(times) if len(times) > 1 else 0.0,
             "tflops": flops / (unordered_ms * 1e-3) / 1e12,
             "note": "compare with the CSR step (value of the default bench line) measured "
                     "in the same process below"}
@@ -782,12 +859,58 @@ def run_sweep(args):
                       "roofline_frac": floor / us}
                 points.append(pt)
                 print(json.dumps(pt), flush=True)
+    status = ctx.device_status()
+    ctx.close()
+    oracle_points = _sweep_oracle(args, points) if args.sweep_oracle else []
     print(json.dumps({"sweep": "L x n, one attend call each", "peaks": {"bf16_tflops": peak, "hbm_gbs": hbm,
                       "source": kind}, "points": len(points),
                       "min_frac": min(p["roofline_frac"] for p in points),
-                      "device_error_flags": ctx.device_status()}), flush=True)
-    ctx.close()
+                      "oracle_points": len(oracle_points),
+                      "device_error_flags": status}), flush=True)
     return 0
+
+
+def _sweep_oracle(args, points):
+    """The oracle column of the sweep: the fp64 C oracle on the same call (RoPE
+    of the n new queries and keys, attention of all 64 heads over L + n keys)
+    in full, on the host cores, for n in {16, 256} at every L."""
+    import numpy as np
+    from oracle import oracle as orc
+    from paper_2605_07325_gb300 import synth
+    ls = sorted(args.sweep_l or SWEEP_L)
+    ns = [n for n in (16, 256) if n in (args.sweep_n or SWEEP_N)]
+    if not ns:
+        return []
+    rng = np.random.default_rng(5)
+    cap = max(ls) + max(ns)
+    bf = lambda shape: synth.bf16_to_f64(synth.bf16_bits(rng.standard_normal(shape, dtype=np.float32)))
+    k_all = np.empty((cap, HKV, D))
+    v_all = np.empty((cap, HKV, D))
+    for i in range(0, cap, 4096):                 # the cache: rotated keys, values (not timed)
+        m = min(4096, cap - i)
+        k_all[i:i + m] = orc.rope(bf((m, HKV, D)), np.arange(i, i + m), BASE)
+        v_all[i:i + m] = bf((m, HKV, D))
+    kpos = np.arange(cap)
+    gpu = {(p["L"], p["n"]): p["us_per_call"] for p in points}
+    out = []
+    for L in ls:
+        for n in ns:
+            q, kn, vn = bf((n, HQ, D)), bf((n, HKV, D)), bf((n, HKV, D))
+            pos = np.arange(L, L + n)
+            t0 = time.perf_counter()
+            q_rot = orc.rope(q, pos, BASE)
+            k_all[L:L + n] = orc.rope(kn, pos, BASE)
+            v_all[L:L + n] = vn
+            orc.attention(q_rot, pos, k_all[:L + n], v_all[:L + n], kpos[:L + n], 1.0 / math.sqrt(D))
+            secs = time.perf_counter() - t0
+            pt = {"L": L, "n": n, "oracle_us": secs * 1e6, "cores": orc.default_threads(),
+                  "extrapolated": False, "kind": "oracle (fp64 C, all 64 heads, in full)"}
+            if (L, n) in gpu:
+                pt["gpu_us"] = gpu[(L, n)]
+                pt["oracle_over_gpu"] = secs * 1e6 / gpu[(L, n)]
+            out.append(pt)
+            print(json.dumps(pt), flush=True)
+    return out
 
 
 def main(argv=None):
@@ -813,6 +936,9 @@ def main(argv=None):
     ap.add_argument("--asr-chunk", type=int, default=CHUNK, help="tokens per state chunk")
     ap.add_argument("--asr-rebuild-tiles", type=int, default=0,
                     help="key tiles per rebuild CTA (0: the library default, 16)")
+    ap.add_argument("--asr-unpaced", action="store_true",
+                    help="enqueue every rebuild task at once (default: one in flight, started "
+                         "after the foreground work)")
     ap.add_argument("--asr-cadence-hz", type=float, default=2.0,
                     help="foreground step rate; 0 runs steps back to back")
     ap.add_argument("--sweep", action="store_true",
@@ -821,6 +947,8 @@ def main(argv=None):
                     help="cached lengths of the sweep (default: 16K 32K 64K 96K 128K)")
     ap.add_argument("--sweep-n", type=int, nargs="*", default=None,
                     help="new-token counts of the sweep (default: 16 64 256 1024 4096)")
+    ap.add_argument("--sweep-oracle", action="store_true",
+                    help="with --sweep: also time the fp64 oracle in full on every L at n = 16 and 256")
     ap.add_argument("--unordered", action="store_true",
                     help="time the unordered baseline (full recompute per step) beside CSR")
     args = ap.parse_args(argv)

@@ -78,6 +78,13 @@ typedef enum csr_status {
                                      append, attention items, merge of split items); by
                                      default a call takes the fused launch when its attention
                                      work is at least 600 key tiles per CTA */
+#define CSR_FLAG_UNPACED_REBUILD 0x8 /* the reconciliation thread enqueues each rebuild task
+                                        as soon as it is due; by default it keeps one task
+                                        (one chunk's recomputation, or the compaction) in
+                                        flight on the low-priority stream and starts it only
+                                        once the foreground work enqueued before it has
+                                        finished, so that a foreground call finds at most
+                                        one short task's CTAs on the SMs */
 
 typedef struct csr_config {
   int32_t num_q_heads;    /* H_q */
@@ -96,11 +103,11 @@ typedef struct csr_config {
                              0 = one per SM */
   int32_t rebuild_tiles_per_cta; /* key tiles (128 keys) per CTA in rebuild launches; 0 = 16 */
   int32_t flags;          /* CSR_FLAG_* */
-  int32_t fg_chunk_tiles; /* > 0: a foreground launch splits every unit's key range into
-                             chunks of this many 128-key tiles (more if the split partials
-                             would not fit), dealt round-robin to its CTAs; 0 = the fused
-                             launch runs whole units in rounds and splits only the leftover
-                             units, the three-launch path picks the chunk length from a
+  int32_t fg_chunk_tiles; /* > 0: a foreground launch cuts every unit's key range into
+                             pieces of at most this many 128-key tiles (the three-launch
+                             path: chunks of exactly this many, more if the split partials
+                             would not fit); 0 = the fused launch cuts only as balance
+                             needs, the three-launch path picks the chunk length from a
                              cost estimate (the default) */
 } csr_config;
 
@@ -410,16 +417,21 @@ typedef struct csr_piece {
   int32_t unit;   /* pair * num_kv_heads + kv head; a pair is query tiles 2p, 2p+1 of
                      128 packed rows (tokens x group heads) */
   int32_t j0, j1; /* key tiles [j0, j1) of 128 keys */
-  int32_t slot;   /* partial-output slot, or -1 when the piece is the whole unit */
+  int32_t slot;   /* merges == 0: the partial slot the piece writes, or -1 when the piece
+                     is the whole unit (written directly); merges > 0: the first of the
+                     slots it merges */
+  int32_t merges; /* > 0: the piece is the last of a cut unit; it waits for the partials
+                     of slots slot .. slot + merges - 1, combines them with its own rows
+                     and writes the unit's output */
 } csr_piece;
 
 /*
- * Inspection: the pieces a foreground call of n new tokens over L cached
- * tokens runs, for a configuration and a CTA count (0 = one per SM of the
- * current device; a plan-only configuration needs grid > 0).  Host-only.
- * pieces may be NULL to count; *n_slots receives the partial slots merged
- * after the grid barrier (0: the launch merges nothing).  CSR_EINVAL for a bad
- * configuration or sizes, CSR_ENOMEM if capacity is too small.
+ * Inspection: the pieces a fused foreground call of n new tokens over L
+ * cached tokens runs, for a configuration and a CTA count (0 = one per SM of
+ * the current device; a plan-only configuration needs grid > 0).  Host-only.
+ * pieces may be NULL to count; *n_slots receives the partial slots written
+ * (0: no unit is cut).  CSR_EINVAL for a bad configuration or sizes, or a
+ * block one fused launch cannot run; CSR_ENOMEM if capacity is too small.
  */
 csr_status csr_foreground_schedule(const csr_config *cfg, int64_t L, int32_t n, int32_t grid,
                                    csr_piece *pieces, int32_t capacity, int32_t *count,
@@ -484,12 +496,16 @@ typedef struct csr_block_args {
  * (so n * num_q_heads * head_dim * 2 bytes, rounded up to whole pairs of
  * 128-row tiles, must not exceed 8 MiB: n <= 512 for 64 query heads of 128
  * dims; larger n returns CSR_EINVAL), 24.5 MiB of split-KV partials (the key
- * range is split only as far as they fit) and the device error word.  The
- * first call on a device resolves that array's address and sets the kernels'
- * shared-memory limit for the device (cudaGetSymbolAddress,
- * cudaFuncSetAttribute); make that first call before any stream capture.
- * Every call shares the array and it keeps the last call's contents; the
- * error word is cleared at the start of each call and not reported.  Calls
+ * range is split only as far as they fit) and the device error word.  Every
+ * call looks the array's address up (cudaGetSymbolAddress); the first call in
+ * a context of the device -- the runtime's primary context, and again after
+ * cudaDeviceReset has replaced it -- also sets the kernels' shared-memory
+ * limit (cudaFuncSetAttribute): make that call before any stream capture.
+ * Every call shares the array and it keeps the last call's contents.  The
+ * error word is cleared at the start of each call and not reported: a page
+ * id out of range in page_table (which the workspace entry points report
+ * through csr_device_status) goes unnoticed here, and the output rows that
+ * needed that page are unspecified; check the table before the call.  Calls
  * that overlap on the same GPU (issued on different streams and not ordered)
  * race on the array: order them.  Each GPU has its own copy of the array.
  * Asynchronous on `stream`.

@@ -26,7 +26,7 @@ NVCC = os.path.join(CUDA_HOME, "bin", "nvcc")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 SOURCES = ["csr_api.cpp", "kernels_attn.cu", "kernels_misc.cu", "csr_noalloc.cu"]
-HEADERS = ["internal.h", "ptx.cuh"]
+HEADERS = ["internal.h", "ptx.cuh", "rope.cuh"]
 
 
 def _stale(target, deps):

@@ -31,6 +31,7 @@ DEVERR_WAIT_TIMEOUT, DEVERR_BAD_PAGE, DEVERR_ALLOC = 0x1, 0x2, 0x4
 FLAG_PLAN_ONLY = 0x1
 FLAG_FUSED_ALWAYS = 0x2
 FLAG_FUSED_NEVER = 0x4
+FLAG_UNPACED_REBUILD = 0x8
 RECON_IDLE, RECON_RUNNING, RECON_SWAPPED = 0, 1, 2
 ROUTE_CONTINUE, ROUTE_BRIDGE, ROUTE_SWAPPED, ROUTE_STRAGGLER = 0, 1, 2, 3
 VERSION_ACTIVE, VERSION_PENDING = 0, 1
@@ -66,7 +67,8 @@ class Timing(ctypes.Structure):
 
 class Piece(ctypes.Structure):
     _fields_ = [("cta", ctypes.c_int32), ("order", ctypes.c_int32), ("unit", ctypes.c_int32),
-                ("j0", ctypes.c_int32), ("j1", ctypes.c_int32), ("slot", ctypes.c_int32)]
+                ("j0", ctypes.c_int32), ("j1", ctypes.c_int32), ("slot", ctypes.c_int32),
+                ("merges", ctypes.c_int32)]
 
 
 class Viability(ctypes.Structure):
@@ -140,8 +142,8 @@ def make_config(num_q_heads, num_kv_heads, head_dim, page_size, rope_base, max_n
 
 
 def foreground_schedule(cfg: Config, L: int, n: int, grid: int = 0):
-    """Pieces (cta, order, unit, j0, j1, slot) of a foreground call of n tokens
-    over L cached, and the number of partial slots it merges."""
+    """Pieces (cta, order, unit, j0, j1, slot, merges) of a fused foreground
+    call of n tokens over L cached, and the number of partial slots written."""
     cnt, slots = ctypes.c_int32(0), ctypes.c_int32(0)
     st = _lib.csr_foreground_schedule(ctypes.byref(cfg), int(L), int(n), int(grid), None, 0,
                                       ctypes.byref(cnt), ctypes.byref(slots))

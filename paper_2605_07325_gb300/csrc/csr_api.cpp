@@ -19,6 +19,7 @@
 #include <cstring>
 #include <deque>
 #include <mutex>
+#include <queue>
 #include <string>
 #include <thread>
 #include <vector>
@@ -157,7 +158,7 @@ bool encode_queries(CUtensorMap *m, const void *q, uint64_t n, uint64_t hq, uint
 }
 
 struct Layout {  // workspace carve-out (byte offsets)
-  size_t qpack[2], rb_out, part_o[2], part_lse[2], pt[2], ids_out, err, sync, total;
+  size_t qpack[2], rb_out, part_o[2], part_lse[2], pt[2], ids_out, err, sync, flags, total;
   int32_t rows_cap, max_pages;
 };
 
@@ -215,6 +216,7 @@ Layout make_layout(const csr_config *c) {
   L.ids_out = take(static_cast<size_t>(L.max_pages) * 4);
   L.err = take(256);
   L.sync = take(256);
+  L.flags = take(static_cast<size_t>(kPartialItems / 2) * 8 * 4);
   L.total = off;
   return L;
 }
@@ -256,10 +258,11 @@ struct csr_ctx {
   double inv_turns[kMaxHalfDim]{};
   TurnSplit turns[kMaxHalfDim]{};     // inv_turns as fp32 hi + lo (rope.cuh)
   float scale_log2 = 0.f;
-  // Arrivals the fused foreground launches have made on the workspace's two
-  // device counters (every CTA adds one per launch; the merge barrier only in
-  // launches that merge), so the next launch knows its targets.
-  uint32_t step_append = 0, step_barrier = 0;
+  // Arrivals the fused foreground launches have made on the workspace's
+  // append counter (every CTA adds one per launch), so the next launch knows
+  // its target; and the generation of the last fused launch (its partial
+  // slots' flags hold it once written).
+  uint32_t step_append = 0, step_gen = 0;
   StepParams step{};                  // parameter block of the last fused launch
   PagePool pool;
   Version ver[2];
@@ -283,6 +286,9 @@ struct csr_ctx {
   void *user = nullptr;
   cudaStream_t lo = nullptr;
   cudaEvent_t ev_fg = nullptr, ev_rb = nullptr;
+  // recorded after every foreground launch while a reconciler is set: the
+  // paced reconciliation thread starts a task only once it has completed
+  cudaEvent_t ev_fg_done = nullptr;
   // Observed pace of the rebuild (App. D viability check): timing events at
   // the start of a reconciliation and after each of its tasks on the
   // low-priority stream, the query-key pairs enqueued there, and the result of
@@ -374,109 +380,169 @@ int32_t choose_chunk_tiles(int64_t units, int64_t kv_max, int max_tiles) {
 
 // Schedule of a fused foreground launch (StepSchedule) for a block of n tokens
 // at L: units u = pair * hkv + head, unit u reading key tiles [0, K(u)).
-// With forced_chunk > 0: round-robin chunks of that many tiles (more if the
-// partial buffer requires).  Otherwise whole units in rounds of `grid`, and
-// the units left over after the last full round cut into pieces level by
-// level: each level cuts its pieces into S parts (S chosen from an estimate
-// of the level's time -- part length plus a per-piece cost -- and of the time
-// the leftover would take spread over the grid), the first `grid` parts (in
-// part-major order, so concurrent parts cover the same key section of
-// different units) run at this level and the rest go to the next; the last
-// level runs whole what is left.  Pieces of a split unit get consecutive
-// partial slots.
-constexpr double kPieceCostTiles = 2.0;   // fixed cost of a piece, in key-tile times
-constexpr double kSlotCostTiles = 0.02;   // partial write + merge read per piece
-constexpr int64_t kMinPieceTiles = 2;
-
-void build_step_schedule(int64_t L, int32_t n, int T, int hkv, int32_t n_tiles, int grid_cap,
-                         int forced_chunk, StepSchedule &S) {
+//
+// Balance: W = sum K(u) tiles on P CTAs takes T = ceil(W / P) tile-times.  A
+// unit longer than T (cap_tiles when forced smaller) is first cut into equal
+// key segments of at most that length; each segment s then runs for k_s
+// tile-times and idles for T - k_s.  With V > P segments, exactly V - P of
+// them idle at any time: the idle intervals are laid end to end on V - P + 1
+// tracks of length T (an interval that crosses a track's end continues at the
+// start of the next, so its segment idles at both ends and runs once in the
+// middle).  The active intervals then never number more than P at a time, and
+// dealing them to CTAs in order of start time (a CTA is free again when its
+// interval ends) keeps every CTA's load within T.
+//
+// Locality: every segment advances one tile per tile-time while it runs, so
+// at any time the keys in use lie within max(T - k_s) tiles of each other
+// and the CTAs of one head read each key tile through L2 at about the same
+// time: the cache is read about once.
+//
+// Merge: the pieces of a cut unit (one per active interval) other than the
+// one that ends last write partial slots (consecutive per unit); the last one
+// merges them.  A piece only ever waits for pieces that end earlier in the
+// schedule (or at the same time on a lower CTA), and every CTA runs its
+// pieces in schedule order, so the waits cannot form a cycle.
+// One attempt with segments of at most seg_cap tiles: 1 = scheduled, 0 = more
+// pieces or partial slots than one launch holds, -1 = not schedulable at all.
+static int try_step_schedule(const std::vector<int64_t> &K, int64_t P, int64_t seg_cap, StepSchedule &S) {
   S = StepSchedule{};
-  for (int l = 0; l < kMaxTailLevels; ++l)
-    for (int c = 0; c < kMaxStepGrid; ++c) {
-      S.piece[l][c] = kNoPiece;
-      S.slot[l][c] = kSlotWhole;
+  const int32_t U = static_cast<int32_t>(K.size());
+  int64_t W = 0;
+  for (int64_t k : K) W += k;
+  const int64_t T0 = ceil_div(W, P);
+  struct Seg {
+    int32_t u;
+    int64_t j0, j1;
+  };
+  std::vector<Seg> seg;
+  for (int32_t u = 0; u < U; ++u) {
+    const int64_t m = ceil_div(K[u], seg_cap);
+    for (int64_t s = 0; s < m; ++s) seg.push_back({u, s * K[u] / m, (s + 1) * K[u] / m});
+  }
+  const int64_t V = static_cast<int64_t>(seg.size());
+  struct Act {
+    int64_t a, b;   // schedule times [a, b)
+    int32_t v;
+  };
+  std::vector<Act> act;
+  if (V <= P) {
+    for (int32_t v = 0; v < V; ++v) act.push_back({0, seg[v].j1 - seg[v].j0, v});
+  } else {
+    // idle intervals laid end to end on tracks of length T0
+    int64_t pos = 0;
+    for (int32_t v = 0; v < V; ++v) {
+      const int64_t k = seg[v].j1 - seg[v].j0, d = T0 - k;
+      if (d == 0) {
+        act.push_back({0, T0, v});
+      } else if (pos + d <= T0) {
+        if (pos > 0) act.push_back({0, pos, v});
+        if (pos + d < T0) act.push_back({pos + d, T0, v});
+        pos = pos + d == T0 ? 0 : pos + d;
+      } else {
+        act.push_back({pos + d - T0, pos, v});   // idle [pos, T0) and [0, pos + d - T0)
+        pos = pos + d - T0;
+      }
     }
+  }
+  std::sort(act.begin(), act.end(), [](const Act &x, const Act &y) {
+    return x.a != y.a ? x.a < y.a : (x.b != y.b ? x.b < y.b : x.v < y.v);
+  });
+  // deal the intervals to CTAs in order of start time: the lowest free CTA
+  std::priority_queue<std::pair<int64_t, int32_t>, std::vector<std::pair<int64_t, int32_t>>,
+                      std::greater<std::pair<int64_t, int32_t>>> busy;   // (end, cta)
+  std::priority_queue<int32_t, std::vector<int32_t>, std::greater<int32_t>> idle;
+  for (int32_t c = 0; c < P; ++c) idle.push(c);
+  struct Pc {
+    int32_t cta, level, u;
+    int64_t b, j0, j1;
+  };
+  std::vector<Pc> pcs;
+  std::vector<int32_t> depth(P, 0);
+  std::vector<int64_t> done(V, 0);   // tiles of each segment dealt so far
+  int32_t used = 0;
+  for (const Act &x : act) {
+    while (!busy.empty() && busy.top().first <= x.a) {
+      idle.push(busy.top().second);
+      busy.pop();
+    }
+    if (idle.empty()) return -1;   // more than P intervals at once: not reachable
+    const int32_t c = idle.top();
+    idle.pop();
+    busy.push({x.b, c});
+    used = std::max(used, c + 1);
+    if (static_cast<int64_t>(pcs.size()) >= kMaxStepPieces) return 0;
+    const Seg &sg = seg[x.v];
+    const int64_t j0 = sg.j0 + done[x.v];
+    done[x.v] += x.b - x.a;
+    pcs.push_back({c, depth[c]++, sg.u, x.b, j0, j0 + (x.b - x.a)});
+  }
+  // pieces in CTA order, each CTA's in schedule order
+  std::vector<int32_t> order(pcs.size());
+  for (size_t i = 0; i < pcs.size(); ++i) order[i] = static_cast<int32_t>(i);
+  std::sort(order.begin(), order.end(), [&](int32_t x, int32_t y) {
+    return pcs[x].cta != pcs[y].cta ? pcs[x].cta < pcs[y].cta : pcs[x].level < pcs[y].level;
+  });
+  std::vector<int32_t> at(pcs.size());   // piece -> table index
+  for (size_t i = 0; i < order.size(); ++i) {
+    const Pc &pc = pcs[order[i]];
+    at[order[i]] = static_cast<int32_t>(i);
+    S.piece[i] = static_cast<uint64_t>(pc.u) | (static_cast<uint64_t>(pc.j0) << 16) |
+                 (static_cast<uint64_t>(pc.j1) << 40);
+    S.slot[i] = kSlotNone;
+    S.merges[i] = 0;
+  }
+  for (int32_t c = 0, i = 0; c <= used; ++c) {
+    while (i < static_cast<int32_t>(order.size()) && pcs[order[i]].cta < c) ++i;
+    S.first[c] = static_cast<uint16_t>(i);
+  }
+  // per unit: the last piece (latest end, then highest CTA) merges the others
+  std::vector<std::vector<int32_t>> of_unit(U);
+  for (int32_t i = 0; i < static_cast<int32_t>(pcs.size()); ++i) of_unit[pcs[i].u].push_back(i);
+  int32_t next = 0;
+  for (int32_t u = 0; u < U; ++u) {
+    auto &v = of_unit[u];
+    if (v.empty()) return -1;
+    if (v.size() == 1) continue;
+    std::sort(v.begin(), v.end(), [&](int32_t x, int32_t y) {
+      return pcs[x].b != pcs[y].b ? pcs[x].b < pcs[y].b : pcs[x].cta < pcs[y].cta;
+    });
+    const int32_t cnt = static_cast<int32_t>(v.size());
+    if (next + cnt - 1 > kPartialItems / 2) return 0;
+    for (int32_t k = 0; k + 1 < cnt; ++k) S.slot[at[v[k]]] = static_cast<uint16_t>(next + k);
+    S.slot[at[v[cnt - 1]]] = static_cast<uint16_t>(next);
+    S.merges[at[v[cnt - 1]]] = static_cast<uint16_t>(cnt - 1);
+    next += cnt - 1;
+  }
+  S.grid = used;
+  S.n_units = U;
+  S.n_pieces = static_cast<int32_t>(pcs.size());
+  S.n_slots = next;
+  return 1;
+}
+
+// The schedule of a block; a forced piece length (cap_tiles > 0) grows by
+// halves while the launch would hold more pieces or slots than it can.
+bool build_step_schedule(int64_t L, int32_t n, int T, int hkv, int32_t n_tiles, int grid_cap,
+                         int cap_tiles, StepSchedule &S) {
   const int32_t pairs = static_cast<int32_t>(ceil_div(n_tiles, 2));
   const int32_t U = pairs * hkv;
-  auto K = [&](int32_t u) { return unit_iters(L, n, T, 2 * (u / hkv) + 1); };
-  S.n_units = U;
-  const int64_t kv_max = K(U - 1);
-  if (forced_chunk > 0 || U > 0xffff) {
-    S.chunked = 1;
-    const int64_t cap_chunks = std::max<int64_t>(1, (kPartialItems / 2) / U);
-    const int64_t chunk = std::max<int64_t>(std::max(forced_chunk, 1), ceil_div(kv_max, cap_chunks));
-    const int64_t n_chunks = ceil_div(kv_max, chunk);
-    S.chunk_tiles = static_cast<int32_t>(chunk);
-    S.n_items = static_cast<int32_t>(n_chunks * U);
-    S.grid = static_cast<int32_t>(std::min<int64_t>(grid_cap, S.n_items));
-    S.n_slots = n_chunks > 1 ? S.n_items : 0;
-    return;
+  if (U < 1 || U > 0xffff || grid_cap < 1) return false;
+  std::vector<int64_t> K(U);
+  int64_t W = 0;
+  for (int32_t u = 0; u < U; ++u) {
+    K[u] = unit_iters(L, n, T, 2 * (u / hkv) + 1);
+    W += K[u];
   }
-  int64_t total = 0;
-  for (int32_t u = 0; u < U; ++u) total += K(u);
-  const int32_t grid = static_cast<int32_t>(std::max<int64_t>(1, std::min<int64_t>(grid_cap, total)));
-  S.grid = grid;
-  S.full_rounds = U / grid;
-  S.n_tail = U - S.full_rounds * grid;
-  struct Pc {
-    int32_t u;
-    int64_t a, b;
-  };
-  std::vector<Pc> pieces;
-  const int32_t first_tail = U - S.n_tail;
-  for (int32_t t = 0; t < S.n_tail; ++t) pieces.push_back({first_tail + t, 0, K(first_tail + t)});
-  std::vector<std::vector<std::pair<int, int>>> unit_pieces(S.n_tail);
-  int level = 0;
-  while (!pieces.empty()) {
-    const int64_t P = static_cast<int64_t>(pieces.size());
-    int64_t len_min = pieces[0].b - pieces[0].a;
-    double len_sum = 0;
-    for (const Pc &pc : pieces) {
-      len_min = std::min<int64_t>(len_min, pc.b - pc.a);
-      len_sum += static_cast<double>(pc.b - pc.a);
-    }
-    const double len = len_sum / static_cast<double>(P);
-    const bool last = level == kMaxTailLevels - 1;
-    const int64_t s_hi = last ? std::max<int64_t>(1, grid / P) : ceil_div(grid, P);
-    int64_t best_s = 1;
-    double best = 1e300;
-    for (int64_t sx = 1; sx <= s_hi; ++sx) {
-      if (sx > 1 && len_min / sx < kMinPieceTiles) break;
-      const int64_t tot = P * sx;
-      const double d = len / static_cast<double>(sx);
-      double cost = d + kPieceCostTiles + kSlotCostTiles * static_cast<double>(tot);
-      if (tot > grid) cost += static_cast<double>(tot - grid) * d / grid + kPieceCostTiles;
-      if (cost < best - 1e-9) {
-        best = cost;
-        best_s = sx;
-      }
-    }
-    std::vector<Pc> subs;
-    for (int64_t q = 0; q < best_s; ++q)
-      for (const Pc &pc : pieces) {
-        const int64_t len_p = pc.b - pc.a;
-        const int64_t a = pc.a + len_p * q / best_s, b = pc.a + len_p * (q + 1) / best_s;
-        if (b > a) subs.push_back({pc.u, a, b});
-      }
-    const int64_t take = std::min<int64_t>(static_cast<int64_t>(subs.size()), grid);
-    for (int64_t c = 0; c < take; ++c) {
-      const Pc &pc = subs[c];
-      S.piece[level][c] = static_cast<uint64_t>(pc.u) | (static_cast<uint64_t>(pc.a) << 16) |
-                          (static_cast<uint64_t>(pc.b) << 40);
-      unit_pieces[pc.u - first_tail].push_back({level, static_cast<int>(c)});
-    }
-    pieces.assign(subs.begin() + take, subs.end());
-    ++level;
+  if (K[U - 1] >= (1ll << 24)) return false;
+  const int64_t P = std::min<int64_t>(grid_cap, kMaxStepGrid);
+  const int64_t T0 = ceil_div(W, P);
+  int64_t cap = cap_tiles > 0 ? std::min<int64_t>(T0, cap_tiles) : T0;
+  while (true) {
+    const int r = try_step_schedule(K, P, cap, S);
+    if (r != 0) return r == 1;
+    if (cap >= T0) return false;
+    cap = std::min(T0, cap + std::max<int64_t>(1, cap / 2));
   }
-  S.levels = level;
-  int32_t next = 0;
-  for (int32_t t = 0; t < S.n_tail; ++t) {
-    S.tail_slot0[t] = static_cast<uint16_t>(next);
-    if (unit_pieces[t].size() > 1)
-      for (const auto &lc : unit_pieces[t]) S.slot[lc.first][lc.second] = static_cast<uint16_t>(next++);
-  }
-  S.tail_slot0[S.n_tail] = static_cast<uint16_t>(next);
-  S.n_slots = next;
 }
 
 cudaEvent_t take_event(csr_ctx *c) {
@@ -541,9 +607,10 @@ csr_status run_block(csr_ctx *c, int slot, int ws, const void *q, const void *k,
   const int T = kBM / c->group;
 
   // Foreground: one cooperative launch of the fused kernel when the call is
-  // long enough for its fixed costs (query preparation, grid barrier, merge:
-  // about 25 us) to vanish, else three chained launches (the rebuild's path
-  // with a persistent grid).  Flags force either.
+  // long enough for its fixed costs (query preparation and append before the
+  // first tile, merges by the last pieces: tens of microseconds) to vanish,
+  // else three chained launches (the rebuild's path with a persistent grid).
+  // Flags force either.
   bool fused = false;
   if (fg) {
     if (cf.flags & CSR_FLAG_FUSED_ALWAYS) {
@@ -555,10 +622,15 @@ csr_status run_block(csr_ctx *c, int slot, int ws, const void *q, const void *k,
       tiles *= cf.num_kv_heads;
       fused = tiles >= static_cast<int64_t>(kFusedMinTilesPerCta) * c->fg_grid;
     }
+    if (n_ids > kMaxStepIds) fused = false;   // more new pages than one fused launch names
+  }
+  StepParams &sp = c->step;
+  if (fused && !build_step_schedule(L, n, T, cf.num_kv_heads, ap.n_tiles, c->fg_grid, cf.fg_chunk_tiles, sp.s)) {
+    if (cf.flags & CSR_FLAG_FUSED_ALWAYS)
+      return fail(c, CSR_EINVAL, "block cannot be scheduled as one fused launch");
+    fused = false;
   }
   if (fused) {
-    StepParams &sp = c->step;
-    build_step_schedule(L, n, T, cf.num_kv_heads, ap.n_tiles, c->fg_grid, cf.fg_chunk_tiles, sp.s);
     ap.grid = sp.s.grid;
     sp.a = ap;
     sp.q = static_cast<const uint16_t *>(q);
@@ -569,8 +641,9 @@ csr_status run_block(csr_ctx *c, int slot, int ws, const void *q, const void *k,
     sp.k_pool = c->k_pool;
     sp.v_pool = c->v_pool;
     sp.sync = c->wsp<uint32_t>(c->lay.sync);
+    sp.flags = c->wsp<uint32_t>(c->lay.flags);
     sp.append_target = c->step_append + static_cast<uint32_t>(sp.s.grid);
-    sp.barrier_target = c->step_barrier + static_cast<uint32_t>(sp.s.grid);
+    sp.gen = c->step_gen + 1 == 0 ? 1 : c->step_gen + 1;
     sp.first_lp = first_lp;
     sp.n_ids = n_ids;
     sp.new_lp = static_cast<int32_t>(L / cf.page_size);
@@ -582,11 +655,12 @@ csr_status run_block(csr_ctx *c, int slot, int ws, const void *q, const void *k,
     sp.append_by_mma = append_items <= 2ll * 32 * sp.s.grid ? 1 : 0;
     std::memcpy(sp.inv_turns, c->turns, sizeof(sp.inv_turns));
     for (int i = 0; i < n_ids; ++i) sp.ids[i] = ids[i];
-    const cudaError_t e =
+    cudaError_t e =
         timed_launch(c, CSR_KERNEL_ATTENTION, true, s, [&] { return launch_step(sp, cf.head_dim, s); });
+    if (e == cudaSuccess && c->rw.started) e = cudaEventRecord(c->ev_fg_done, s);
     if (e != cudaSuccess) return cuda_fail(c, e, "attention launch");
     c->step_append += static_cast<uint32_t>(sp.s.grid);
-    if (sp.s.n_slots > 0) c->step_barrier += static_cast<uint32_t>(sp.s.grid);
+    c->step_gen = sp.gen;
     ++c->launches;
     return CSR_OK;
   }
@@ -658,6 +732,10 @@ csr_status run_block(csr_ctx *c, int slot, int ws, const void *q, const void *k,
     e = timed_launch(c, CSR_KERNEL_MERGE, fg, s, [&] { return launch_merge(mp, s); });
     if (e != cudaSuccess) return cuda_fail(c, e, "merge launch");
     ++c->launches;
+  }
+  if (fg && c->rw.started) {
+    e = cudaEventRecord(c->ev_fg_done, s);
+    if (e != cudaSuccess) return cuda_fail(c, e, "recording the foreground event");
   }
   return CSR_OK;
 }
@@ -775,6 +853,17 @@ csr_status rebuild_chunk(csr_ctx *c, const ChunkRec &ch, int64_t pos,
                    out ? out : c->wsp<void>(c->lay.rb_out), nullptr, s);
 }
 
+// Wait for an event by polling (the worker's own thread; yields between
+// polls so that a foreground thread sharing the core is not starved).
+cudaError_t wait_event(csr_ctx *c, cudaEvent_t ev) {
+  (void)c;
+  while (true) {
+    const cudaError_t e = cudaEventQuery(ev);
+    if (e != cudaErrorNotReady) return e;
+    std::this_thread::yield();
+  }
+}
+
 // Worker side of Reconciler: run tasks in order, record ev_rb after each.
 void worker_main(csr_ctx *c) {
   cudaSetDevice(c->device);
@@ -791,7 +880,13 @@ void worker_main(csr_ctx *c) {
     lk.unlock();
     csr_status st = CSR_OK;
     msg.clear();
-    if (!skip) {
+    const bool paced = !(c->cfg.flags & CSR_FLAG_UNPACED_REBUILD);
+    if (!skip && paced) {
+      // start only once the foreground work enqueued so far has finished
+      const cudaError_t e = wait_event(c, c->ev_fg_done);
+      if (e != cudaSuccess) st = cuda_fail(c, e, "waiting for the foreground work");
+    }
+    if (!skip && st == CSR_OK) {
       Range range(t.compact ? "csr_rebuild_compact" : "csr_rebuild_chunk");
       if (t.compact) {
         const cudaError_t e = launch_evict(*t.compact, c->lo);
@@ -803,6 +898,8 @@ void worker_main(csr_ctx *c) {
       if (st == CSR_OK) {
         cudaError_t e = cudaEventRecord(c->ev_rb, c->lo);
         if (e == cudaSuccess) e = cudaEventRecord(c->ev_rb_t1, c->lo);
+        // paced: one task in flight at a time
+        if (e == cudaSuccess && paced) e = wait_event(c, c->ev_rb);
         if (e != cudaSuccess) st = cuda_fail(c, e, "recording the rebuild event");
       }
     }
@@ -969,11 +1066,13 @@ csr_status csr_create(const csr_config *cfg, void *k_pool, void *v_pool, void *w
     if (e == cudaSuccess) e = cudaMemsetAsync(workspace, 0, c->lay.total, s);
     if (e == cudaSuccess) e = cudaEventCreateWithFlags(&c->ev_fg, cudaEventDisableTiming);
     if (e == cudaSuccess) e = cudaEventCreateWithFlags(&c->ev_rb, cudaEventDisableTiming);
+    if (e == cudaSuccess) e = cudaEventCreateWithFlags(&c->ev_fg_done, cudaEventDisableTiming);
     if (e == cudaSuccess) e = cudaEventCreate(&c->ev_rb_t0);
     if (e == cudaSuccess) e = cudaEventCreate(&c->ev_rb_t1);
     if (e != cudaSuccess) {
       if (c->ev_fg) cudaEventDestroy(c->ev_fg);
       if (c->ev_rb) cudaEventDestroy(c->ev_rb);
+      if (c->ev_fg_done) cudaEventDestroy(c->ev_fg_done);
       if (c->ev_rb_t0) cudaEventDestroy(c->ev_rb_t0);
       if (c->ev_rb_t1) cudaEventDestroy(c->ev_rb_t1);
       delete c;
@@ -992,6 +1091,7 @@ void csr_destroy(csr_ctx *c) {
     cudaDeviceSynchronize();
     if (c->ev_fg) cudaEventDestroy(c->ev_fg);
     if (c->ev_rb) cudaEventDestroy(c->ev_rb);
+    if (c->ev_fg_done) cudaEventDestroy(c->ev_fg_done);
     if (c->ev_rb_t0) cudaEventDestroy(c->ev_rb_t0);
     if (c->ev_rb_t1) cudaEventDestroy(c->ev_rb_t1);
     for (auto &t : c->timed) {
@@ -1597,36 +1697,18 @@ csr_status csr_foreground_schedule(const csr_config *cfg, int64_t L, int32_t n, 
   const int T = kBM / group;
   const int32_t n_tiles = static_cast<int32_t>(ceil_div(static_cast<int64_t>(n) * group, kBM));
   StepSchedule S;
-  build_step_schedule(L, n, T, cfg->num_kv_heads, n_tiles, grid, cfg->fg_chunk_tiles, S);
-  // Enumerate what each CTA's walker yields, in order.
+  if (!build_step_schedule(L, n, T, cfg->num_kv_heads, n_tiles, grid, cfg->fg_chunk_tiles, S))
+    return CSR_EINVAL;
+  // What each CTA's walker yields, in order.
   std::vector<csr_piece> out;
-  const int hkv = cfg->num_kv_heads;
-  auto K = [&](int32_t u) { return unit_iters(L, n, T, 2 * (u / hkv) + 1); };
-  for (int32_t c = 0; c < S.grid; ++c) {
-    int32_t order = 0;
-    if (S.chunked) {
-      for (int32_t it = c; it < S.n_items; it += S.grid) {
-        const int32_t k = it / S.n_units, u = it - k * S.n_units;
-        const int64_t kv = K(u), j0 = static_cast<int64_t>(k) * S.chunk_tiles;
-        if (j0 >= kv) continue;
-        const int64_t j1 = std::min<int64_t>(j0 + S.chunk_tiles, kv);
-        out.push_back({c, order++, u, static_cast<int32_t>(j0), static_cast<int32_t>(j1),
-                       kv <= S.chunk_tiles ? -1 : it});
-      }
-      continue;
-    }
-    for (int32_t r = 0; r < S.full_rounds; ++r) {
-      const int32_t u = r * S.grid + ((r & 1) ? S.grid - 1 - c : c);
-      out.push_back({c, order++, u, 0, static_cast<int32_t>(K(u)), -1});
-    }
-    for (int l = 0; l < S.levels; ++l) {
-      const uint64_t e = S.piece[l][c];
-      if (e == kNoPiece) continue;
-      out.push_back({c, order++, static_cast<int32_t>(e & 0xffffu), static_cast<int32_t>((e >> 16) & 0xffffffu),
+  for (int32_t c = 0; c < S.grid; ++c)
+    for (int32_t i = S.first[c], order = 0; i < S.first[c + 1]; ++i, ++order) {
+      const uint64_t e = S.piece[i];
+      out.push_back({c, order, static_cast<int32_t>(e & 0xffffu), static_cast<int32_t>((e >> 16) & 0xffffffu),
                      static_cast<int32_t>((e >> 40) & 0xffffffu),
-                     S.slot[l][c] == kSlotWhole ? -1 : static_cast<int32_t>(S.slot[l][c])});
+                     S.slot[i] == kSlotNone ? -1 : static_cast<int32_t>(S.slot[i]),
+                     static_cast<int32_t>(S.merges[i])});
     }
-  }
   *count = static_cast<int32_t>(out.size());
   if (n_slots) *n_slots = S.n_slots;
   if (pieces) {

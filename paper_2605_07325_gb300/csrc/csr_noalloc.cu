@@ -32,7 +32,8 @@ static __device__ __align__(256) uint8_t g_block_scratch[kScratchBytes];
 
 struct DeviceSetup {
   bool ready = false;
-  uint8_t *scratch = nullptr;  // device address of g_block_scratch on this device
+  unsigned long long ctx_id = 0;  // the context the setup was made in (a reset makes a new one)
+  uint8_t *scratch = nullptr;     // device address of g_block_scratch in that context
   int num_sms = 0;
 };
 std::mutex g_setup_mu;
@@ -65,20 +66,50 @@ bool encode(CUtensorMap *m, const void *base, uint64_t rows, uint64_t d, uint32_
 
 int64_t cdiv(int64_t a, int64_t b) { return (a + b - 1) / b; }
 
-// Once per device, with that device current: resolve the scratch array's
-// device address and raise the attention kernels' shared-memory limit.
+// Unique id of the calling thread's current context (0 if none or the driver
+// lacks the query).  The runtime's primary context of a device is replaced by
+// cudaDeviceReset, and with it the module holding the scratch array and the
+// kernels' attributes: the setup below is redone whenever the id changes.
+unsigned long long current_context_id() {
+  static PFN_cuCtxGetCurrent_v4000 get_current = nullptr;
+  static PFN_cuCtxGetId_v12000 get_id = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void *p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 4000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      get_current = reinterpret_cast<PFN_cuCtxGetCurrent_v4000>(p);
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      get_id = reinterpret_cast<PFN_cuCtxGetId_v12000>(p);
+  });
+  CUcontext ctx = nullptr;
+  unsigned long long id = 0;
+  if (!get_current || !get_id || get_current(&ctx) != CUDA_SUCCESS || !ctx || get_id(ctx, &id) != CUDA_SUCCESS)
+    return 0;
+  return id;
+}
+
+// With the device current: resolve the scratch array's device address and
+// raise the attention kernels' shared-memory limit, once per context of the
+// device.
 csr_status setup_device(int dev, DeviceSetup **out) {
   if (dev < 0 || dev >= kMaxDevices) return CSR_EINVAL;
   std::lock_guard<std::mutex> lock(g_setup_mu);
   DeviceSetup &s = g_setup[dev];
-  if (!s.ready) {
-    void *ptr = nullptr;
-    if (cudaGetSymbolAddress(&ptr, g_block_scratch) != cudaSuccess) return CSR_ECUDA;
+  void *sym = nullptr;
+  // also makes the device's primary context current on this thread
+  if (cudaGetSymbolAddress(&sym, g_block_scratch) != cudaSuccess) return CSR_ECUDA;
+  const unsigned long long ctx_id = current_context_id();
+  if (!s.ready || ctx_id == 0 || ctx_id != s.ctx_id || sym != s.scratch) {
+    s.ready = false;
     if (attn_configure(64) != cudaSuccess || attn_configure(128) != cudaSuccess) return CSR_ECUDA;
     int sms = 0;
     if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
       return CSR_ECUDA;
-    s.scratch = static_cast<uint8_t *>(ptr);
+    s.scratch = static_cast<uint8_t *>(sym);
+    s.ctx_id = ctx_id;
     s.num_sms = sms;
     s.ready = true;
   }

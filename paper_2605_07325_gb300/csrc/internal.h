@@ -62,33 +62,34 @@ struct AttnParams {
   float scale_log2;        // softmax_scale * log2(e)
 };
 
-// Schedule of a fused foreground launch (attn_pair_kernel<HD, true>): which
-// pieces (unit, key tiles [j0, j1)) each CTA runs, and where split pieces
-// leave their partial outputs.  Units are numbered u = pair * hkv + head.
+// Schedule of a fused foreground launch (attn_pair_kernel<HD, true>): the
+// pieces (unit, key tiles [j0, j1)) each CTA runs, in order.  Units are
+// numbered u = pair * hkv + head.  A unit cut into several pieces is merged
+// by its last piece (the one that ends last in the schedule): every other
+// piece writes its normalised partial rows and log2-sum-exp to a slot and
+// raises that slot's flags; the last piece waits for the flags, combines the
+// partials with its own accumulator and writes the output rows.
 constexpr int kMaxStepGrid = 160;
-constexpr int kMaxTailLevels = 6;
-constexpr uint64_t kNoPiece = ~0ull;
-constexpr uint16_t kSlotWhole = 0xffff;  // the piece is a whole unit: written directly
+constexpr int kMaxStepPieces = 2304;    // pieces of one launch, over all CTAs
+constexpr int kMaxStepIds = 256;        // new pages one fused launch may name
+constexpr uint16_t kSlotNone = 0xffff;
 struct StepSchedule {
   int32_t grid;          // CTAs (<= kMaxStepGrid)
   int32_t n_units;
-  int32_t chunked;       // 1: round-robin chunks (forced chunk length); 0: rounds + tail levels
-  // chunked form: items (chunk k, unit u) = k * n_units + u, CTA c runs c, c + grid, ...;
-  // every unit with more than one chunk is merged (slot = item)
-  int32_t chunk_tiles, n_items;
-  // rounds + tail form: CTA c runs units r * grid + (r odd ? grid - 1 - c : c)
-  // whole for r < full_rounds; units n_units - n_tail .. n_units - 1 are cut
-  // into the pieces of the tail levels, piece[l][c] being CTA c's at level l
-  int32_t full_rounds, n_tail, levels;
-  int32_t n_slots;       // partial slots written (0: the launch merges nothing)
-  uint64_t piece[kMaxTailLevels][kMaxStepGrid];  // unit | j0 << 16 | j1 << 40, or kNoPiece
-  uint16_t slot[kMaxTailLevels][kMaxStepGrid];   // partial slot, or kSlotWhole
-  uint16_t tail_slot0[kMaxStepGrid + 1];         // tail unit t's slots [tail_slot0[t], tail_slot0[t+1])
+  int32_t n_pieces;
+  int32_t n_slots;       // partial slots written (0: no unit is cut)
+  uint16_t first[kMaxStepGrid + 1];    // CTA c runs pieces first[c] .. first[c + 1] - 1, in order
+  uint64_t piece[kMaxStepPieces];      // unit | j0 << 16 | j1 << 40
+  // merges == 0: slot is the partial slot the piece writes, or kSlotNone for a
+  // whole unit (written directly); merges > 0: the piece is its unit's last
+  // and merges the partials of slots slot .. slot + merges - 1
+  uint16_t slot[kMaxStepPieces];
+  uint16_t merges[kMaxStepPieces];
 };
 
 // Fused foreground block (one cooperative launch): RoPE + paged append of the
 // new keys/values, RoPE of the queries straight into shared memory, attention,
-// and the merge of split pieces after a grid barrier.
+// and the merge of cut units by their last pieces.
 struct StepParams {
   AttnParams a;            // tm_q, n_items, chunk_tiles unused
   CUtensorMap tm_qraw;     // q as [n][hq][d] (3-D), box {64, G, 128/G}: one query tile per column half
@@ -96,16 +97,18 @@ struct StepParams {
   const uint16_t *k;       // [n][hkv][d]
   const uint16_t *v;
   uint16_t *k_pool, *v_pool;
-  uint32_t *sync;          // [0]: append arrivals, [1]: merge-barrier arrivals (both monotonic)
+  uint32_t *sync;          // [0]: append arrivals (monotonic)
+  uint32_t *flags;         // [slot][8 softmax warps]: the launch generation once written
   uint32_t append_target;  // sync[0] once every CTA of this launch has appended its share
-  uint32_t barrier_target; // sync[1] once every CTA of this launch has written its partials
+  uint32_t gen;            // this launch's generation (never 0; stale flags hold older ones)
   int32_t first_lp, n_ids; // logical pages first_lp.. get ids[] (written to the table by CTA 0)
   int32_t new_lp;          // logical page holding position L: key tiles reaching it wait for the append
   int32_t append_by_mma;   // 1: the MMA warp appends (few tokens); 0: the softmax warps
   TurnSplit inv_turns[kMaxHalfDim];
-  int32_t ids[kMaxIdsPerCall];
+  int32_t ids[kMaxStepIds];
   StepSchedule s;
 };
+static_assert(sizeof(StepParams) <= 32000, "kernel parameters of the fused launch");
 
 // K3: merge of split partials (rebuild launches and the no-allocation block path).
 struct MergeParams {

@@ -60,17 +60,14 @@
 
 namespace csr {
 
-// One piece of work: key tiles [j0, j1) of a unit (head, pair).  A split
-// piece writes row r (0..255) of its partial output at row pbase + r * pstride
-// of the partial buffer: slot-major (pbase = slot * 256, pstride = 1) for
-// item launches and the chunked form, row-major over the unit's slots
-// (pbase = first slot * 256 + slot index, pstride = the unit's slot count) for
-// the rounds + tail form, so that a merge batch of rows is one contiguous copy.
+// One piece of work: key tiles [j0, j1) of a unit (head, pair).  A piece
+// that is not the whole unit writes row r (0..255) of its partial output at
+// row slot * 256 + r of the partial buffer; in the fused form the last piece
+// of a cut unit instead merges the partials of slots slot .. slot + merges - 1
+// (merges > 0) into its own rows and writes the output.
 struct Seg {
-  int32_t head, pair, slot;
+  int32_t head, pair, slot, merges;
   int64_t j0, j1;
-  int64_t pbase;
-  int32_t pstride;
   bool complete;
 };
 
@@ -166,6 +163,9 @@ __device__ __forceinline__ uint32_t ld_acquire_gpu(const uint32_t *ptr) {
   asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(ptr) : "memory");
   return v;
 }
+__device__ __forceinline__ void st_release_gpu(uint32_t *ptr, uint32_t v) {
+  asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(ptr), "r"(v) : "memory");
+}
 __device__ __forceinline__ void red_release_gpu_add(uint32_t *ptr, uint32_t v) {
   asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(ptr), "r"(v) : "memory");
 }
@@ -235,11 +235,6 @@ struct PairCfg {
   static constexpr int kSmemIds = 256;
   static constexpr int kSmem = kAngOff + 1024;                 // + alignment slack
   static constexpr int kSmemStep = kIdsOff + kSmemIds * 4 + 1024;
-  // fused form, after the attention loops: the merge stages partial rows in
-  // the Q and K/V region and keeps row LSEs and weights in the angle tables
-  static constexpr int kMergeBuf = kBarOff;
-  static constexpr int kMergeRows = 40;                        // rows per merge batch
-  static constexpr int kMergeWts = (8 * kAngEntries * 8) / 4 - kMergeRows;  // weight floats
   static constexpr uint32_t kTmemCols = 512;
   static constexpr uint32_t kOCol = 2 * kBN;                   // O_A; O_B at kOCol + HD
 };
@@ -249,7 +244,7 @@ struct PairBars {
   uint64_t q_full, q_empty;
   uint64_t k_full[4], k_empty[4], v_full[4], v_empty[4];
   uint64_t s_full[2], p_full[2], o_final[2], o_free[2];
-  uint64_t drain, merge_full, qraw_full;
+  uint64_t drain, qraw_full;
   uint32_t tmem_base;
   int abort;
 };
@@ -277,8 +272,7 @@ struct PairWalker {
       s.head = head;
       s.pair = pair;
       s.slot = it;
-      s.pbase = static_cast<int64_t>(it) * kPairRows;
-      s.pstride = 1;
+      s.merges = 0;
       s.j0 = j0;
       s.j1 = min(j0 + p.chunk_tiles, kv);
       s.complete = kv <= p.chunk_tiles;
@@ -290,69 +284,23 @@ struct PairWalker {
 
 // Pieces of the fused form (StepSchedule); units u = pair * hkv + head.
 struct StepWalker {
-  int32_t c, r, lvl, item;
+  int32_t i, end;
   __device__ bool next(const StepParams &p, int T, Seg &s) {
     const StepSchedule &S = p.s;
-    const AttnParams &A = p.a;
-    if (S.chunked) {
-      while (item < S.n_items) {
-        const int32_t it = item;
-        item += S.grid;
-        const int32_t k = it / S.n_units;
-        const int32_t u = it - k * S.n_units;
-        const int32_t pair = u / A.hkv;
-        const int64_t kv = unit_iters(A.L, A.n, T, 2 * pair + 1);
-        const int64_t j0 = static_cast<int64_t>(k) * S.chunk_tiles;
-        if (j0 >= kv) continue;
-        s.head = u - pair * A.hkv;
-        s.pair = pair;
-        s.slot = it;
-        s.pbase = static_cast<int64_t>(it) * kPairRows;
-        s.pstride = 1;
-        s.j0 = j0;
-        s.j1 = min(j0 + S.chunk_tiles, kv);
-        s.complete = kv <= S.chunk_tiles;
-        return true;
-      }
-      return false;
-    }
-    if (r < S.full_rounds) {
-      const int32_t rr = r++;
-      const int32_t u = rr * S.grid + ((rr & 1) ? S.grid - 1 - c : c);
-      const int32_t pair = u / A.hkv;
-      s.head = u - pair * A.hkv;
-      s.pair = pair;
-      s.slot = kSlotWhole;
-      s.pbase = 0;
-      s.pstride = 1;
-      s.j0 = 0;
-      s.j1 = unit_iters(A.L, A.n, T, 2 * pair + 1);
-      s.complete = true;
-      return true;
-    }
-    while (lvl < S.levels) {
-      const int l = lvl++;
-      const uint64_t e = S.piece[l][c];
-      if (e == kNoPiece) continue;
-      const int32_t u = static_cast<int32_t>(e & 0xffffu);
-      const int32_t pair = u / A.hkv;
-      s.head = u - pair * A.hkv;
-      s.pair = pair;
-      s.slot = S.slot[l][c];
-      s.j0 = static_cast<int64_t>((e >> 16) & 0xffffffu);
-      s.j1 = static_cast<int64_t>((e >> 40) & 0xffffffu);
-      s.complete = s.slot == kSlotWhole;
-      s.pbase = 0;
-      s.pstride = 1;
-      if (!s.complete) {
-        const int32_t t = u - (S.n_units - S.n_tail);
-        const int32_t s0 = S.tail_slot0[t];
-        s.pbase = static_cast<int64_t>(s0) * kPairRows + (s.slot - s0);
-        s.pstride = S.tail_slot0[t + 1] - s0;
-      }
-      return true;
-    }
-    return false;
+    (void)T;
+    if (i >= end) return false;
+    const uint64_t e = S.piece[i];
+    const int32_t u = static_cast<int32_t>(e & 0xffffu);
+    const int32_t pair = u / p.a.hkv;
+    s.head = u - pair * p.a.hkv;
+    s.pair = pair;
+    s.j0 = static_cast<int64_t>((e >> 16) & 0xffffffu);
+    s.j1 = static_cast<int64_t>((e >> 40) & 0xffffffu);
+    s.slot = S.slot[i];
+    s.merges = S.merges[i];
+    s.complete = s.slot == kSlotNone;
+    ++i;
+    return true;
   }
 };
 
@@ -370,8 +318,8 @@ __device__ __forceinline__ const AttnParams &attn_of(const StepParams &p) { retu
 __device__ __forceinline__ PairWalker make_walker(const AttnParams &) {
   return PairWalker{static_cast<int32_t>(blockIdx.x)};
 }
-__device__ __forceinline__ StepWalker make_walker(const StepParams &) {
-  return StepWalker{static_cast<int32_t>(blockIdx.x), 0, 0, static_cast<int32_t>(blockIdx.x)};
+__device__ __forceinline__ StepWalker make_walker(const StepParams &p) {
+  return StepWalker{p.s.first[blockIdx.x], p.s.first[blockIdx.x + 1]};
 }
 
 // ============================================================ fused-form steps
@@ -382,8 +330,7 @@ __device__ __forceinline__ int32_t step_page(const StepParams &p, const int32_t 
   const AttnParams &A = p.a;
   int32_t phys;
   if (lp >= p.first_lp && lp < p.first_lp + p.n_ids) {
-    const int64_t i = lp - p.first_lp;
-    phys = i < 256 ? ids_s[i] : p.ids[i];
+    phys = ids_s[lp - p.first_lp];   // n_ids <= kSmemIds
   } else {
     phys = A.page_table[lp];
   }
@@ -567,196 +514,6 @@ __device__ __noinline__ bool step_q_prep(const StepParams &p, uint8_t *qtile, fl
   return true;
 }
 
-// The merge of a fused launch, in batches of at most kMergeRows rows of one
-// unit.  Rows are numbered unit by unit over the split units (every unit of
-// the chunked form with more than one chunk, the split tail units otherwise);
-// each CTA takes a contiguous range [m0, m1) of them.
-// Partial row of slot k (0..cnt-1) and batch row r is base + k * kstride +
-// r * rstride; rows_major: the rows of the batch are contiguous over all its
-// slots (one bulk copy), else each slot's rows are (one copy per slot).
-struct MergeBatch {
-  int32_t unit, ra, R, cnt;
-  int64_t base, kstride, rstride;
-  bool rows_major;
-};
-
-__device__ __forceinline__ void merge_range(const StepSchedule &S, int64_t &m0, int64_t &m1) {
-  const int64_t n_mu = S.chunked ? S.n_units : S.n_tail;
-  const int64_t rows = n_mu * kPairRows;
-  const int64_t per = (rows + gridDim.x - 1) / gridDim.x;
-  m0 = static_cast<int64_t>(blockIdx.x) * per;
-  m1 = min(rows, m0 + per);
-}
-
-// The batch starting at merge row m (rows up to m1): cnt == 0 for a unit that
-// the attention loop wrote whole.
-template <int HD>
-__device__ __forceinline__ MergeBatch merge_batch(const StepParams &p, int T, int64_t m, int64_t m1) {
-  using C = PairCfg<HD>;
-  const AttnParams &A = p.a;
-  const StepSchedule &S = p.s;
-  const int32_t mu = static_cast<int32_t>(m / kPairRows);
-  MergeBatch b;
-  b.ra = static_cast<int32_t>(m - static_cast<int64_t>(mu) * kPairRows);
-  int64_t rmax = kPairRows - b.ra;
-  if (S.chunked) {
-    b.unit = mu;
-    const int64_t kv = unit_iters(A.L, A.n, T, 2 * (mu / A.hkv) + 1);
-    const int32_t nk = static_cast<int32_t>((kv + S.chunk_tiles - 1) / S.chunk_tiles);
-    b.cnt = nk > 1 ? nk : 0;
-    b.base = static_cast<int64_t>(mu) * kPairRows + b.ra;
-    b.kstride = static_cast<int64_t>(S.n_units) * kPairRows;
-    b.rstride = 1;
-    b.rows_major = false;
-  } else {
-    b.unit = S.n_units - S.n_tail + mu;
-    const int32_t s0 = S.tail_slot0[mu];
-    b.cnt = S.tail_slot0[mu + 1] - s0;
-    b.base = static_cast<int64_t>(s0) * kPairRows + static_cast<int64_t>(b.ra) * b.cnt;
-    b.kstride = 1;
-    b.rstride = b.cnt;
-    b.rows_major = true;
-    // one copy of whole rows: as many rows as the staging buffer holds
-    if (b.cnt > 0) rmax = min(rmax, static_cast<int64_t>(max(1, C::kMergeBuf / (b.cnt * HD * 4))));
-  }
-  b.R = static_cast<int32_t>(min(min(m1 - m, rmax), static_cast<int64_t>(C::kMergeRows)));
-  return b;
-}
-
-// After the grid barrier: merge this CTA's batches (all 320 threads).  Per
-// batch and slot batch: warp 9 issues one bulk copy per slot of the slot's
-// partial rows (consecutive in memory) into shared memory, all in flight at
-// once, while warps 0-8 find the row LSEs (lse = log2 sum_k 2^lse_k, one pass
-// over each row's slot LSEs kept in registers) and the weights 2^(lse_k -
-// lse); then every thread accumulates its (row, 4 columns) outputs from
-// shared memory and writes bf16 out and the natural-log lse.
-template <int HD>
-__device__ __noinline__ void step_merge(const StepParams &p, int T, uint8_t *smem, uint64_t *bar, MergeBatch first,
-                                        int64_t m, int64_t m1) {
-  using C = PairCfg<HD>;
-  const AttnParams &A = p.a;
-  constexpr int kRowBytes = HD * 4;
-  constexpr int kCols = HD / 4;                                   // 4-float columns per row
-  constexpr int kOwn = (C::kMergeRows * kCols + kPairThreads - 1) / kPairThreads;
-  float *buf = reinterpret_cast<float *>(smem);                   // [slot][row][HD]
-  float *row_lse = reinterpret_cast<float *>(smem + C::kAngOff);  // [kMergeRows]
-  float *wts = row_lse + C::kMergeRows;                           // [slot][row]
-  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  volatile int no_abort = 0;
-  uint32_t phase = 0;
-  bool use_first = true;
-  while (m < m1) {
-    const MergeBatch b = use_first ? first : merge_batch<HD>(p, T, m, m1);
-    use_first = false;
-    m += b.R;
-    if (b.cnt == 0) continue;   // the unit was written whole by the attention loop
-    const int32_t R = b.R, cnt = b.cnt;
-    auto prow = [&](int32_t k, int32_t r) { return b.base + k * b.kstride + r * b.rstride; };
-    // slots per copy round: all of them when whole rows are copied
-    const int32_t kb_max = b.rows_major ? cnt : max(1, min(C::kMergeBuf / (R * kRowBytes), C::kMergeWts / R));
-    float4 acc[kOwn];
-#pragma unroll
-    for (int j = 0; j < kOwn; ++j) acc[j] = make_float4(0.f, 0.f, 0.f, 0.f);
-    for (int32_t k0 = 0; k0 < cnt; k0 += kb_max) {
-      const int32_t kb = min(kb_max, cnt - k0);
-      if (tid == 9 * 32) {
-        fence_proxy_async_global();   // partials another SM wrote, now read by the async proxy
-        mbar_arrive_expect_tx(bar, static_cast<uint32_t>(kb * R * kRowBytes));
-        if (b.rows_major) {
-          // the batch's rows over all slots: one copy, buffer [row][slot][HD]
-          bulk_load_1d(buf, A.part_o + prow(0, 0) * HD, static_cast<uint32_t>(R * cnt * kRowBytes), bar);
-        } else {
-          for (int32_t k = 0; k < kb; ++k)   // buffer [slot][row][HD]
-            bulk_load_1d(buf + static_cast<int64_t>(k) * R * HD, A.part_o + prow(k0 + k, 0) * HD,
-                         static_cast<uint32_t>(R * kRowBytes), bar);
-        }
-      }
-      if (k0 == 0) {
-        // row LSEs and the first slot batch's weights, one row per warp of 0-8
-        if (warp < 9) {
-          for (int r = warp; r < R; r += 9) {
-            float v[4];
-            float mx = -CUDART_INF_F;
-#pragma unroll
-            for (int j = 0; j < 4; ++j) {
-              const int k = lane + 32 * j;
-              v[j] = k < cnt ? ld_cg_f(A.part_lse + prow(k, r)) : -CUDART_INF_F;
-              mx = fmaxf(mx, v[j]);
-            }
-            for (int k = 128 + lane; k < cnt; k += 32) mx = fmaxf(mx, ld_cg_f(A.part_lse + prow(k, r)));
-#pragma unroll
-            for (int off = 16; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
-            const float m_use = mx == -CUDART_INF_F ? 0.f : mx;
-            float sum = 0.f;
-#pragma unroll
-            for (int j = 0; j < 4; ++j) sum += ex2_approx(v[j] - m_use);
-            for (int k = 128 + lane; k < cnt; k += 32) sum += ex2_approx(ld_cg_f(A.part_lse + prow(k, r)) - m_use);
-#pragma unroll
-            for (int off = 16; off > 0; off >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, off);
-            const float lr = sum > 0.f ? m_use + log2f(sum) : -CUDART_INF_F;
-            if (lane == 0) row_lse[r] = lr;
-#pragma unroll
-            for (int j = 0; j < 4; ++j) {
-              const int k = lane + 32 * j;
-              if (k < kb) wts[k * R + r] = lr == -CUDART_INF_F ? 0.f : ex2_approx(v[j] - lr);
-            }
-            for (int k = 128 + lane; k < kb; k += 32)
-              wts[k * R + r] = lr == -CUDART_INF_F ? 0.f : ex2_approx(ld_cg_f(A.part_lse + prow(k, r)) - lr);
-          }
-        }
-      } else {
-        for (int i = tid; i < kb * R; i += kPairThreads) {
-          const int k = i / R, r = i - k * R;
-          const float lr = row_lse[r];
-          wts[i] = lr == -CUDART_INF_F ? 0.f : ex2_approx(ld_cg_f(A.part_lse + prow(k0 + k, r)) - lr);
-        }
-      }
-      __syncthreads();
-      // wait for the copies even after an abort elsewhere (none may still be
-      // writing this CTA's shared memory when it exits); bounded all the same
-      mbar_wait(bar, phase & 1, &no_abort, A.err, CSR_DEVERR_WAIT_TIMEOUT);
-      ++phase;
-#pragma unroll
-      for (int j = 0; j < kOwn; ++j) {
-        const int idx = tid + j * kPairThreads;
-        if (idx < R * kCols) {
-          const int r = idx / kCols, c = idx - r * kCols;
-          for (int k = 0; k < kb; ++k) {
-            const float w = wts[k * R + r];
-            const int64_t bi = b.rows_major ? static_cast<int64_t>(r) * kb + k : static_cast<int64_t>(k) * R + r;
-            const float4 v = reinterpret_cast<const float4 *>(buf + bi * HD)[c];
-            acc[j].x = fmaf(w, v.x, acc[j].x);
-            acc[j].y = fmaf(w, v.y, acc[j].y);
-            acc[j].z = fmaf(w, v.z, acc[j].z);
-            acc[j].w = fmaf(w, v.w, acc[j].w);
-          }
-        }
-      }
-      __syncthreads();   // the buffer and weights are rewritten by the next slot batch
-    }
-    const int32_t pair = b.unit / A.hkv;
-    const int32_t head = b.unit - pair * A.hkv;
-#pragma unroll
-    for (int j = 0; j < kOwn; ++j) {
-      const int idx = tid + j * kPairThreads;
-      if (idx < R * kCols) {
-        const int r = idx / kCols, c = idx - r * kCols;
-        const int rr = (b.ra + r) % kBM;
-        const int tile = pair * 2 + (b.ra + r) / kBM;
-        const int64_t t = static_cast<int64_t>(tile) * T + rr / A.group;
-        if (tile < A.n_tiles && t < A.n) {
-          const int hq_idx = head * A.group + rr % A.group;
-          uint16_t *dst = A.out + (t * A.hq + hq_idx) * HD + c * 4;
-          *reinterpret_cast<uint2 *>(dst) = make_uint2(pack_bf16x2(acc[j].x, acc[j].y),
-                                                       pack_bf16x2(acc[j].z, acc[j].w));
-          if (c == 0 && A.lse) A.lse[static_cast<int64_t>(hq_idx) * A.n + t] = row_lse[r] * 0.69314718055994531f;
-        }
-      }
-    }
-    __syncthreads();   // row_lse is rewritten by the next batch
-  }
-}
-
 // ============================================================ the kernel
 template <int HD, bool kStep>
 __global__ void __launch_bounds__(kPairThreads, 1)
@@ -788,7 +545,6 @@ __global__ void __launch_bounds__(kPairThreads, 1)
       mbar_init(&bars->o_free[w], 4);
     }
     mbar_init(&bars->drain, 1);
-    mbar_init(&bars->merge_full, 1);
     mbar_init(&bars->qraw_full, 1);
     bars->abort = 0;
     fence_barrier_init();
@@ -1165,11 +921,63 @@ __global__ void __launch_bounds__(kPairThreads, 1)
         break;
       }
       tc_fence_after();
-      const float inv_l = l > 0.f ? 1.0f / l : 0.f;
-      const float lse2 = l > 0.f ? m_ref + log2f(l) : -CUDART_INF_F;
+      float inv_l = l > 0.f ? 1.0f / l : 0.f;
+      float lse2 = l > 0.f ? m_ref + log2f(l) : -CUDART_INF_F;
       uint32_t o[HD];
       load_o<HD>(tmem + lane_base + o_col, o);
-      if (seg.complete) {
+      // O is in registers now: the MMA warp may accumulate the next piece
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&bars->o_free[wg]);
+      bool to_out = seg.complete;
+      if constexpr (kStep) {
+        if (seg.merges > 0) {
+          // The unit's last piece: once the other pieces have written this
+          // warp's rows (their flags hold this launch's generation), combine
+          // lse = log2(2^lse_own + sum_k 2^lse_k) and
+          // out = 2^(lse_own - lse) O_own / l + sum_k 2^(lse_k - lse) O_k.
+          const uint32_t *fl = p.flags + static_cast<int64_t>(seg.slot) * 8 + warp;
+          bool got = true;
+          for (int k = 0; k < seg.merges && got; ++k) got = wait_counter(fl + k * 8, p.gen, A.err, abort);
+          if (!__all_sync(0xffffffffu, got)) {
+            ok = false;
+            break;
+          }
+          const int64_t r0 = static_cast<int64_t>(seg.slot) * kPairRows + wg * kBM + row;
+          float mx = lse2;
+          for (int k = 0; k < seg.merges; ++k) mx = fmaxf(mx, ld_cg_f(A.part_lse + r0 + k * kPairRows));
+          const float m_use = mx == -CUDART_INF_F ? 0.f : mx;
+          float sum = l > 0.f ? ex2_approx(lse2 - m_use) : 0.f;
+          for (int k = 0; k < seg.merges; ++k) sum += ex2_approx(ld_cg_f(A.part_lse + r0 + k * kPairRows) - m_use);
+          const float lse_t = sum > 0.f ? m_use + log2f(sum) : -CUDART_INF_F;
+          const float w_own = l > 0.f ? ex2_approx(lse2 - lse_t) * inv_l : 0.f;
+#pragma unroll
+          for (int c = 0; c < HD; ++c) o[c] = __float_as_uint(__uint_as_float(o[c]) * w_own);
+          for (int k = 0; k < seg.merges; ++k) {
+            const int64_t rk = r0 + k * kPairRows;
+            const float lk = ld_cg_f(A.part_lse + rk);
+            const float wk = lse_t == -CUDART_INF_F ? 0.f : ex2_approx(lk - lse_t);
+            const float *src = A.part_o + rk * HD;
+#pragma unroll
+            for (int c0 = 0; c0 < HD; c0 += 16) {
+              float4 v[4];
+#pragma unroll
+              for (int e = 0; e < 4; ++e) v[e] = ld_cg_f4(src + c0 + 4 * e);
+#pragma unroll
+              for (int e = 0; e < 4; ++e) {
+                o[c0 + 4 * e + 0] = __float_as_uint(fmaf(wk, v[e].x, __uint_as_float(o[c0 + 4 * e + 0])));
+                o[c0 + 4 * e + 1] = __float_as_uint(fmaf(wk, v[e].y, __uint_as_float(o[c0 + 4 * e + 1])));
+                o[c0 + 4 * e + 2] = __float_as_uint(fmaf(wk, v[e].z, __uint_as_float(o[c0 + 4 * e + 2])));
+                o[c0 + 4 * e + 3] = __float_as_uint(fmaf(wk, v[e].w, __uint_as_float(o[c0 + 4 * e + 3])));
+              }
+            }
+          }
+          inv_l = 1.0f;
+          lse2 = lse_t;
+          to_out = true;
+        }
+      }
+      if (to_out) {
         if (valid) {
           const int hq_idx = seg.head * A.group + row % A.group;
           uint16_t *dst = A.out + (static_cast<int64_t>(t) * A.hq + hq_idx) * HD;
@@ -1185,7 +993,7 @@ __global__ void __launch_bounds__(kPairThreads, 1)
           if (A.lse) A.lse[static_cast<int64_t>(hq_idx) * A.n + t] = lse2 * 0.69314718055994531f;
         }
       } else {
-        const int64_t base = seg.pbase + static_cast<int64_t>(wg * kBM + row) * seg.pstride;
+        const int64_t base = static_cast<int64_t>(seg.slot) * kPairRows + wg * kBM + row;
         // the partial buffer is 256-byte aligned and rows are HD floats: 32-byte stores
         float *dst = A.part_o + base * HD;
 #pragma unroll
@@ -1196,10 +1004,14 @@ __global__ void __launch_bounds__(kPairThreads, 1)
           st_global_v8(dst + 8 * c, w);
         }
         A.part_lse[base] = lse2;
+        if constexpr (kStep) {
+          // this warp's 32 rows are written: raise the slot's flag for the
+          // unit's last piece
+          __threadfence();
+          __syncwarp();
+          if (lane == 0) st_release_gpu(p.flags + static_cast<int64_t>(seg.slot) * 8 + warp, p.gen);
+        }
       }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&bars->o_free[wg]);
       ++seg_n;
     }
   }
@@ -1211,27 +1023,6 @@ __global__ void __launch_bounds__(kPairThreads, 1)
     __syncwarp();
     tc_fence_after();
     tmem_dealloc(tmem, C::kTmemCols);
-  }
-  if constexpr (kStep) {
-    if (p.s.n_slots > 0) {
-      // grid barrier (every CTA is resident: cooperative launch), then the
-      // merge; every thread works out its first batch (the schedule's
-      // parameters) while the barrier is pending
-      if (threadIdx.x == 0) {
-        __threadfence();
-        red_release_gpu_add(p.sync + 1, 1u);
-      }
-      int64_t m0, m1;
-      merge_range(p.s, m0, m1);
-      MergeBatch first{};
-      if (m0 < m1) first = merge_batch<HD>(p, T, m0, m1);
-      if (threadIdx.x == 0) {
-        wait_counter(p.sync + 1, p.barrier_target, A.err, nullptr);
-        __threadfence();
-      }
-      __syncthreads();
-      step_merge<HD>(p, T, smem, &bars->merge_full, first, m0, m1);
-    }
   }
 }
 

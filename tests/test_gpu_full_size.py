@@ -4,9 +4,9 @@ benchmark times, against the fp64 oracle on sampled query rows.
 A 122,880-token cache (4,096-token static prefix + 4,096-token chunks) of the
 64 q / 4 kv head, head_dim 128, page 64 shape; then the step -- a 256-token
 chunk and a 512-token suffix -- once fused (csr_append_chunk_attend_suffix,
-the benchmark's default) and once as two calls.  For sampled query tokens the
-oracle computes the attention of all 64 heads over every cached key one row
-at a time (inputs are the bf16 values the library received, keys rotated by
+the benchmark's default) and once as two calls.  For 71 sampled query tokens
+the oracle computes the attention of all 64 heads over every cached key one
+row at a time (inputs are the bf16 values the library received, keys rotated by
 the oracle's RoPE at their absolute positions); outputs and log-sum-exps must
 be within the parity tolerances, and the page table must equal the oracle
 allocator's.
@@ -25,7 +25,15 @@ pytestmark = pytest.mark.gpu
 
 HQ, HKV, D, P, BASE = 64, 4, 128, 64, 1e6
 PREFIX, FILL, L0, CHUNK, SUFFIX = 4096, 4096, 122880, 256, 512
-SAMPLE = np.array([0, 1, 130, 255, 256, 257, 600, 767])   # token offsets in the 768-token step
+# Sampled token offsets in the 768-token step (8 tokens per 128-row tile at
+# 16 query heads per kv head, 16 per pair of tiles): both sides of tile and
+# tile-pair boundaries, the chunk/suffix boundary (255 | 256), the first and
+# last token, and one token of every one of the 48 pairs (each pair is four
+# units, one per kv head, most of them cut into pieces by the fused schedule).
+_EDGES = [0, 1, 7, 8, 15, 16, 17, 31, 32, 127, 128, 247, 248, 255, 256, 257, 263, 264, 271, 272,
+          511, 512, 759, 760, 766, 767]
+SAMPLE = np.array(sorted(set(_EDGES) | {16 * p + (5 * p) % 16 for p in range(48)}))
+assert len(SAMPLE) >= 64
 
 
 @pytest.fixture(scope="module")

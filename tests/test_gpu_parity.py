@@ -79,16 +79,17 @@ def test_ragged_sizes(libcsr, shape, chunk_tiles, path):
 @pytest.mark.parametrize("num_ctas,chunk_tiles", [(1, 0), (3, 1), (7, 2), (19, 3), (64, 5),
                                                    (152, 1), (0, 4), (0, 0), (5, 0)])
 def test_split_kv_partials_any_grid(libcsr, num_ctas, chunk_tiles, path):
-    """Forced CTA counts and key-chunk lengths: every split into items (down to
-    one 128-key tile per item) must merge back to the oracle, on both paths
-    (chunk 0: the fused kernel's rounds + tail schedule, the three-launch
-    path's cost model)."""
+    """Forced CTA counts and piece lengths: every cut of a unit into pieces
+    (down to one 128-key tile) must merge back to the oracle, on both paths
+    (the fused kernel's last pieces merge the others' partials; the
+    three-launch path's merge kernel combines chunk partials)."""
+    sizes = (700, 1000, 33, 200)
     p = Pair(C2, pool_pages=256, max_seq=8192, max_new=1024, num_ctas=num_ctas,
              fg_chunk_tiles=chunk_tiles, flags=PATHS[path])
-    p.init_static(p.blk(30, 700))
-    p.append(p.blk(31, 1000))
-    p.append(p.blk(32, 33))
-    p.suffix(p.blk(33, 200))
+    p.init_static(p.blk(30, sizes[0]))
+    p.append(p.blk(31, sizes[1]))
+    p.append(p.blk(32, sizes[2]))
+    p.suffix(p.blk(33, sizes[3]))
     p.truncate()
     p.device_clean()
 

@@ -2,12 +2,13 @@
 
 For every block shape the pieces must cover each unit's key tiles [0, K(u))
 exactly once -- K(u) from the causal rule, key range [0, L + last token of the
-pair) -- with at most one piece per unit and CTA level, whole units written
-directly and split units given distinct partial slots; the work per CTA must
-be balanced, and only units left over after the full rounds may be split."""
-import itertools
-import math
-
+pair).  A unit run as one piece is written directly; of a cut unit, every
+piece but one writes its own partial slot and the remaining piece merges all
+of them.  Every CTA's load must be within the optimum ceil(W / P) tiles, the
+merge waits must not be able to deadlock (checked by running the schedule as
+the kernel would: a CTA takes its pieces in order and the merging piece
+finishes only once the others have), and the keys in use at any time must
+stay within a narrow window (the cache is then read through L2 about once)."""
 import pytest
 
 C1 = dict(hq=8, hkv=2, d=64, P=16)
@@ -32,87 +33,159 @@ def _unit_tiles(shape, L, n):
     return K
 
 
-def _check(pieces, slots, K, grid):
+def _check(pieces, n_slots, K, grid):
+    """Coverage, slot bookkeeping and per-CTA order; returns each CTA's load."""
     cover = {u: [] for u in K}
     per_cta = {}
-    used_slots = set()
-    for cta, order, u, j0, j1, slot in pieces:
+    for cta, order, u, j0, j1, slot, merges in pieces:
         assert 0 <= cta < grid and 0 <= j0 < j1 <= K[u]
-        cover[u].append((j0, j1, slot))
+        cover[u].append((j0, j1, slot, merges))
         per_cta.setdefault(cta, []).append((order, j1 - j0))
-        if slot >= 0:
-            assert slot not in used_slots
-            used_slots.add(slot)
+    written = []
     for u, segs in cover.items():
         segs.sort()
-        assert segs[0][0] == 0 and segs[-1][1] == K[u], (u, segs)
+        assert segs and segs[0][0] == 0 and segs[-1][1] == K[u], (u, segs)
         for a, b in zip(segs, segs[1:]):
             assert a[1] == b[0], (u, segs)       # contiguous, no overlap
         if len(segs) == 1:
-            assert segs[0][2] == -1               # a whole unit is written directly
-        else:
-            assert all(s >= 0 for _, _, s in segs)
-    assert len(used_slots) == slots or (slots > 0 and len(used_slots) <= slots)
+            assert segs[0][2:] == (-1, 0)         # a whole unit is written directly
+            continue
+        last = [s for s in segs if s[3] > 0]
+        assert len(last) == 1 and last[0][3] == len(segs) - 1, (u, segs)
+        own = sorted(s[2] for s in segs if s[3] == 0)
+        assert own == list(range(last[0][2], last[0][2] + len(segs) - 1)), (u, segs)
+        written += own
+    assert sorted(written) == list(range(n_slots))
     for cta, items in per_cta.items():
         assert sorted(o for o, _ in items) == list(range(len(items)))
     return {cta: sum(w for _, w in items) for cta, items in per_cta.items()}
 
 
+def _run(pieces):
+    """Execute the schedule as the kernel does; True if every piece finishes."""
+    seq = {}
+    for p in pieces:
+        seq.setdefault(p[0], []).append(p)
+    for v in seq.values():
+        v.sort(key=lambda p: p[1])
+    others = {}
+    for p in pieces:
+        if p[6] == 0 and p[5] >= 0:
+            others.setdefault(p[2], set()).add(p)
+    done, pos = set(), {c: 0 for c in seq}
+    progress = True
+    while progress:
+        progress = False
+        for c, v in seq.items():
+            while pos[c] < len(v):
+                p = v[pos[c]]
+                if p[6] > 0 and not others[p[2]] <= done:
+                    break                             # the merging piece waits
+                done.add(p)
+                pos[c] += 1
+                progress = True
+    return len(done) == len(pieces)
+
+
 CASES = [
-    (C2, 122_880, 768, 152),      # the 120K fused step: 192 units on 152 CTAs
-    (C2, 131_072, 16, 152),       # 4 units: every one split 38 ways
+    (C2, 122_880, 768, 152),      # the 120K step: 192 units on 152 CTAs
+    (C2, 131_072, 16, 152),       # 4 units on 152 CTAs: every unit cut into segments
     (C2, 131_072, 64, 152),
     (C2, 131_072, 256, 152),
+    (C2, 131_072, 512, 152),
     (C2, 131_072, 1024, 152),
     (C2, 16_384, 4096, 152),
-    (C2, 0, 4096, 152),           # a prefill: unit lengths from 1 to 32 tiles
     (C2, 6_144, 192, 152),        # the 8K step
     (C1, 1_024, 32, 152),         # tiny shape: fewer tiles than CTAs
     (C1, 0, 256, 152),
-    (C2, 122_880, 768, 7),
+    (C2, 122_880, 768, 37),
+    (C2, 122_880, 96, 7),
+    (C2, 1_000, 300, 19),
     (C2, 122_880, 768, 1),
 ]
 
 
 @pytest.mark.parametrize("shape,L,n,grid", CASES)
-def test_pieces_cover_every_key_tile_once(libcsr, shape, L, n, grid):
+def test_pieces_cover_balance_and_finish(libcsr, shape, L, n, grid):
     cfg = _cfg(libcsr, shape)
-    pieces, slots = libcsr.foreground_schedule(cfg, L, n, grid)
+    pieces, n_slots = libcsr.foreground_schedule(cfg, L, n, grid)
     K = _unit_tiles(shape, L, n)
-    load = _check(pieces, slots, K, grid)
-    used = len(load)
-    total = sum(K.values())
-    ideal = total / min(grid, total)
-    # a CTA's load: at most the ideal plus one piece's worth of rounding per tail level
-    longest = max(K.values())
-    assert max(load.values()) <= max(ideal * 1.06 + 6 * 2, longest), (max(load.values()), ideal)
-    assert used <= grid
+    load = _check(pieces, n_slots, K, grid)
+    W = sum(K.values())
+    assert max(load.values()) <= max(-(-W // grid), 1)     # the optimum, to the tile
+    assert _run(pieces)
 
 
-def test_only_leftover_units_split(libcsr):
-    """The 120K step: 152 units run whole in the first round; only the 40
-    left over are cut, so the partials are far fewer than a split of every
-    unit would write."""
-    pieces, slots = libcsr.foreground_schedule(_cfg(libcsr, C2), 122_880, 768, 152)
-    whole = [p for p in pieces if p[5] == -1]
-    split_units = {p[2] for p in pieces if p[5] >= 0}
-    assert len(whole) == 152 and len(split_units) == 40
-    assert slots == sum(1 for p in pieces if p[5] >= 0) <= 6 * 152
-    # pieces of one tail level cover the same key section of different units
-    by_cta = {}
+def _times(pieces):
+    """Start time of every piece: CTAs run back to back from time 0."""
+    seq = {}
     for p in pieces:
-        by_cta.setdefault(p[0], []).append(p)
-    first_tail = [sorted(v, key=lambda x: x[1])[1] for v in by_cta.values() if len(v) > 1]
-    sections = {p[3] for p in first_tail}
-    assert len(sections) <= 8
+        seq.setdefault(p[0], []).append(p)
+    out = []
+    for v in seq.values():
+        t = 0
+        for p in sorted(v, key=lambda p: p[1]):
+            out.append((t, p))
+            t += p[4] - p[3]
+    return out
 
 
-@pytest.mark.parametrize("chunk,n,L", [(1, 300, 1_000), (3, 77, 513), (5, 1024, 8_000)])
-def test_forced_chunks_round_robin(libcsr, chunk, n, L):
+def test_step_120k_cuts_and_locality(libcsr):
+    """The 120K step: 192 units of 960-966 tiles on 152 CTAs.  At most P - 1
+    partial slots (each 256 rows of 512 + 4 bytes, written once and read once:
+    under 15% of the 278.4 MB the step must move), at most three pieces per
+    CTA, and the keys a CTA reads at any time within one idle period (T - K,
+    about 253 tiles: 16 MB of each head's cache) of the schedule time."""
+    pieces, n_slots = libcsr.foreground_schedule(_cfg(libcsr, C2), 122_880, 768, 152)
+    K = _unit_tiles(C2, 122_880, 768)
+    assert n_slots <= 151
+    assert 2 * n_slots * 256 * (128 * 4 + 4) <= 0.15 * 278.4e6
+    per_cta = {}
+    for p in pieces:
+        per_cta[p[0]] = per_cta.get(p[0], 0) + 1
+    assert max(per_cta.values()) <= 3
+    T = -(-sum(K.values()) // 152)
+    window = T - min(K.values())
+    for t, p in _times(pieces):
+        assert abs(t - p[3]) <= window + 2, (t, p)
+
+
+def test_short_units_run_whole(libcsr):
+    """With fewer units than CTAs and units no longer than the balanced load,
+    nothing is cut."""
+    cfg = _cfg(libcsr, C2)
+    pieces, n_slots = libcsr.foreground_schedule(cfg, 0, 1024, 152)   # 256 units of <= 8 tiles
+    K = _unit_tiles(C2, 0, 1024)
+    _check(pieces, n_slots, K, 152)
+    assert _run(pieces)
+
+
+@pytest.mark.parametrize("chunk,n,L,grid", [(1, 300, 1_000, 19), (3, 77, 513, 19), (5, 1024, 8_000, 152),
+                                            (2, 512, 4_000, 64)])
+def test_forced_piece_length(libcsr, chunk, n, L, grid):
+    """fg_chunk_tiles caps the pieces' length (grown by halves only while the
+    launch would hold more than 2,304 pieces)."""
     cfg = _cfg(libcsr, C2, chunk=chunk, max_new=2048)
-    pieces, slots = libcsr.foreground_schedule(cfg, L, n, 19)
+    pieces, n_slots = libcsr.foreground_schedule(cfg, L, n, grid)
     K = _unit_tiles(C2, L, n)
-    _check(pieces, slots, K, 19)
-    # every piece is at most `chunk` tiles long unless the partial buffer forced longer ones
-    longest = max(j1 - j0 for _, _, _, j0, j1, _ in pieces)
-    assert longest >= min(chunk, max(K.values()))
+    _check(pieces, n_slots, K, grid)
+    assert _run(pieces)
+    longest = max(j1 - j0 for _, _, _, j0, j1, _, _ in pieces)
+    # a longer piece only where the cap was grown: pieces at the cap would
+    # have overflowed the table, so the grown schedule is still large
+    assert len(pieces) <= 2304 and (longest <= chunk or len(pieces) > 2304 // 2)
+
+
+def test_one_cta_runs_every_unit(libcsr):
+    """192 units of 960-966 tiles on one CTA: every unit whole, once."""
+    pieces, n_slots = libcsr.foreground_schedule(_cfg(libcsr, C2), 122_880, 768, 1)
+    assert n_slots == 0 and len(pieces) == 192
+    assert sorted(p[2] for p in pieces) == list(range(192))
+
+
+def test_too_many_pieces_is_refused(libcsr):
+    """A prefill of 16,384 tokens is 4,096 units, more pieces than one
+    launch's table holds (2,304): the call reports it (a foreground call then
+    takes the three-launch path)."""
+    with pytest.raises(libcsr.CsrError):
+        libcsr.foreground_schedule(_cfg(libcsr, C2, max_new=16384), 0, 16384, 152)
