@@ -554,7 +554,8 @@ def run_asr(args):
                           max_seq_tokens=n_max, cap_tokens=cap,
                           evict_tokens=evict, n_catchup=0,
                           rebuild_tiles_per_cta=args.asr_rebuild_tiles,
-                          flags=csr.FLAG_UNPACED_REBUILD if args.asr_unpaced else 0)
+                          flags=csr.FLAG_UNPACED_REBUILD if args.asr_unpaced else 0,
+                          rebuild_duty=args.asr_duty)
     fg = torch.cuda.Stream(device=dev, priority=-1)     # high priority
     lo = torch.cuda.Stream(device=dev, priority=0)      # low priority (rebuild, R_2)
     gen = torch.Generator(device=dev).manual_seed(4321)
@@ -634,7 +635,7 @@ def run_asr(args):
         length = ctx.layout()[1]
         peak_len = max(peak_len, length)
         during = was or now
-        records.append((t1 - t0, e0.elapsed_time(e1) / 1e3, during))
+        records.append((t1 - t0, e0.elapsed_time(e1) / 1e3, during, length))
         step += 1
         if period:
             next_t += period
@@ -648,6 +649,13 @@ def run_asr(args):
     out = [r[0] for r in records if not r[2]]
     dev_dur = [r[1] for r in records if r[2]]
     dev_out = [r[1] for r in records if not r[2]]
+    # A rebuild runs while the cache is at its largest (from tau_mem until the
+    # swap), the steps outside it over every length down to the post-eviction
+    # one: the like-for-like baseline is the outside steps over caches at
+    # least as long as the shortest one a rebuild ran beside (less 2,048).
+    band = min((r[3] for r in records if r[2]), default=0) - 2048
+    out_m = [r[0] for r in records if not r[2] and r[3] >= band]
+    dev_out_m = [r[1] for r in records if not r[2] and r[3] >= band]
     line = {
         "workload": (f"ASR cycle run: cap {cap:,} tokens, 4,096-token prefix, {chunk}-token chunks + "
                      f"512-token suffix per step, evict oldest {evict:,} tokens, rebuild on a "
@@ -657,12 +665,16 @@ def run_asr(args):
         "cadence_hz": args.asr_cadence_hz, "rebuild_tiles_per_cta": args.asr_rebuild_tiles or 16,
         "rebuild_pacing": "all tasks at once" if args.asr_unpaced else
                           "one task in flight, started after the foreground work",
+        "rebuild_duty": args.asr_duty,
         "cycles": cycles, "steps": step,
         "steps_during_rebuild": len(dur),
         "fg_ms_host": {"p50_outside": pct(out, 50), "p99_outside": pct(out, 99),
                        "p50_during": pct(dur, 50), "p99_during": pct(dur, 99)},
         "fg_ms_device": {"p50_outside": pct(dev_out, 50), "p99_outside": pct(dev_out, 99),
                          "p50_during": pct(dev_dur, 50), "p99_during": pct(dev_dur, 99)},
+        "matched_outside": {"min_cached_tokens": band, "steps": len(out_m),
+                            "host_p50": pct(out_m, 50), "host_p99": pct(out_m, 99),
+                            "device_p50": pct(dev_out_m, 50), "device_p99": pct(dev_out_m, 99)},
         "rebuild_to_swap_s": {"mean": statistics.mean(rebuilds) if rebuilds else None,
                               "max": max(rebuilds) if rebuilds else None,
                               "note": "eviction to the poll (start of a step) that swapped"},
@@ -671,7 +683,10 @@ def run_asr(args):
         "device_error_flags": flags,
     }
     if out and dur:
-        line["p99_increase_during_rebuild"] = pct(dur, 99) / pct(out, 99) - 1.0
+        line["p99_increase_during_rebuild_all_lengths"] = pct(dur, 99) / pct(out, 99) - 1.0
+    if out_m and dur:
+        line["p99_increase_during_rebuild"] = pct(dur, 99) / pct(out_m, 99) - 1.0
+        line["p99_increase_during_rebuild_device"] = pct(dev_dur, 99) / pct(dev_out_m, 99) - 1.0
     # App. D viability: the rebuild (warm-up + catch-up, here eviction -> swap)
     # must end before the cache, growing at X_dot tokens/s from tau_mem, reaches N_max
     if rebuilds and period:
@@ -782,8 +797,10 @@ def run_sweep(args):
     torch.cuda.set_device(dev)
     hbm, peak, _, kind = _peaks()
     max_L = max(args.sweep_l or SWEEP_L)
+    path_flags = {"auto": 0, "fused": csr.FLAG_FUSED_ALWAYS, "three": csr.FLAG_FUSED_NEVER}[args.sweep_path]
     cfg = csr.make_config(HQ, HKV, D, P, BASE, max_new_tokens=4096,
-                          pool_pages=(max_L + 4096) // P + 16, max_seq_tokens=max_L + 4096 + P)
+                          pool_pages=(max_L + 4096) // P + 16, max_seq_tokens=max_L + 4096 + P,
+                          flags=path_flags)
     stream = torch.cuda.Stream(device=dev, priority=-1)
     gen = torch.Generator(device=dev).manual_seed(99)
 
@@ -862,7 +879,8 @@ def run_sweep(args):
     status = ctx.device_status()
     ctx.close()
     oracle_points = _sweep_oracle(args, points) if args.sweep_oracle else []
-    print(json.dumps({"sweep": "L x n, one attend call each", "peaks": {"bf16_tflops": peak, "hbm_gbs": hbm,
+    print(json.dumps({"sweep": "L x n, one attend call each", "path": args.sweep_path,
+                      "peaks": {"bf16_tflops": peak, "hbm_gbs": hbm,
                       "source": kind}, "points": len(points),
                       "min_frac": min(p["roofline_frac"] for p in points),
                       "oracle_points": len(oracle_points),
@@ -936,6 +954,8 @@ def main(argv=None):
     ap.add_argument("--asr-chunk", type=int, default=CHUNK, help="tokens per state chunk")
     ap.add_argument("--asr-rebuild-tiles", type=int, default=0,
                     help="key tiles per rebuild CTA (0: the library default, 16)")
+    ap.add_argument("--asr-duty", type=float, default=0.0,
+                    help="share of wall time the rebuild may occupy the GPU (0 = no limit)")
     ap.add_argument("--asr-unpaced", action="store_true",
                     help="enqueue every rebuild task at once (default: one in flight, started "
                          "after the foreground work)")
@@ -947,6 +967,8 @@ def main(argv=None):
                     help="cached lengths of the sweep (default: 16K 32K 64K 96K 128K)")
     ap.add_argument("--sweep-n", type=int, nargs="*", default=None,
                     help="new-token counts of the sweep (default: 16 64 256 1024 4096)")
+    ap.add_argument("--sweep-path", choices=["auto", "fused", "three"], default="auto",
+                    help="with --sweep: the library's choice of foreground path, or one forced")
     ap.add_argument("--sweep-oracle", action="store_true",
                     help="with --sweep: also time the fp64 oracle in full on every L at n = 16 and 256")
     ap.add_argument("--unordered", action="store_true",

@@ -109,6 +109,11 @@ typedef struct csr_config {
                              would not fit); 0 = the fused launch cuts only as balance
                              needs, the three-launch path picks the chunk length from a
                              cost estimate (the default) */
+  float rebuild_duty;     /* share of wall time the paced reconciliation thread lets the
+                             rebuild occupy the GPU (after a task it waits task time *
+                             (1 / duty - 1) before the next): a lower share keeps the
+                             chip's power, and with it the foreground's clock, down while
+                             a rebuild runs; 0 or >= 1 = no wait (the default) */
 } csr_config;
 
 /*
@@ -418,11 +423,16 @@ typedef struct csr_piece {
                      128 packed rows (tokens x group heads) */
   int32_t j0, j1; /* key tiles [j0, j1) of 128 keys */
   int32_t slot;   /* merges == 0: the partial slot the piece writes, or -1 when the piece
-                     is the whole unit (written directly); merges > 0: the first of the
-                     slots it merges */
-  int32_t merges; /* > 0: the piece is the last of a cut unit; it waits for the partials
-                     of slots slot .. slot + merges - 1, combines them with its own rows
-                     and writes the unit's output */
+                     is the whole unit (written directly); merges > 0 and group == 1: the
+                     first of the slots it merges; group > 1: the slot it writes */
+  int32_t merges; /* > 0: the piece is in the last group of a cut unit (the pieces that end
+                     last); the unit has this many partial slots */
+  int32_t group;  /* size g of that group (0 for other pieces).  g == 1: the piece waits for
+                     the partials of slots slot .. slot + merges - 1, combines them with
+                     its own rows and writes the unit's output.  g > 1: every piece of the
+                     unit writes a partial (the group's are the last g of the unit's
+                     consecutive slots); member k merges rows [k*256/g, (k+1)*256/g) */
+  int32_t member; /* k, the piece's index in its group */
 } csr_piece;
 
 /*

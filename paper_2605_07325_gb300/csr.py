@@ -55,6 +55,7 @@ class Config(ctypes.Structure):
         ("rebuild_tiles_per_cta", ctypes.c_int32),
         ("flags", ctypes.c_int32),
         ("fg_chunk_tiles", ctypes.c_int32),
+        ("rebuild_duty", ctypes.c_float),
     ]
 
 
@@ -68,7 +69,7 @@ class Timing(ctypes.Structure):
 class Piece(ctypes.Structure):
     _fields_ = [("cta", ctypes.c_int32), ("order", ctypes.c_int32), ("unit", ctypes.c_int32),
                 ("j0", ctypes.c_int32), ("j1", ctypes.c_int32), ("slot", ctypes.c_int32),
-                ("merges", ctypes.c_int32)]
+                ("merges", ctypes.c_int32), ("group", ctypes.c_int32), ("member", ctypes.c_int32)]
 
 
 class Viability(ctypes.Structure):
@@ -135,15 +136,17 @@ class CsrError(RuntimeError):
 def make_config(num_q_heads, num_kv_heads, head_dim, page_size, rope_base, max_new_tokens,
                 pool_pages, max_seq_tokens, softmax_scale=0.0, cap_tokens=0, evict_tokens=0,
                 n_catchup=0, num_ctas=0, rebuild_tiles_per_cta=0, flags=0,
-                fg_chunk_tiles=0) -> Config:
+                fg_chunk_tiles=0, rebuild_duty=0.0) -> Config:
     return Config(num_q_heads, num_kv_heads, head_dim, page_size, float(rope_base),
                   float(softmax_scale), max_new_tokens, pool_pages, max_seq_tokens, cap_tokens,
-                  evict_tokens, n_catchup, num_ctas, rebuild_tiles_per_cta, flags, fg_chunk_tiles)
+                  evict_tokens, n_catchup, num_ctas, rebuild_tiles_per_cta, flags, fg_chunk_tiles,
+                  float(rebuild_duty))
 
 
 def foreground_schedule(cfg: Config, L: int, n: int, grid: int = 0):
-    """Pieces (cta, order, unit, j0, j1, slot, merges) of a fused foreground
-    call of n tokens over L cached, and the number of partial slots written."""
+    """Pieces (cta, order, unit, j0, j1, slot, merges, group, member) of a
+    fused foreground call of n tokens over L cached, and the number of partial
+    slots written."""
     cnt, slots = ctypes.c_int32(0), ctypes.c_int32(0)
     st = _lib.csr_foreground_schedule(ctypes.byref(cfg), int(L), int(n), int(grid), None, 0,
                                       ctypes.byref(cnt), ctypes.byref(slots))

@@ -187,7 +187,7 @@ bool valid_config(const csr_config *c, std::string *why) {
   if (static_cast<int64_t>(c->pool_pages) * c->num_kv_heads * c->page_size >= (1ll << 31))
     return bad("pool rows exceed the 32-bit TMA coordinate range");
   if (c->cap_tokens < 0 || c->evict_tokens < 0 || c->n_catchup < 0 || c->num_ctas < 0 ||
-      c->rebuild_tiles_per_cta < 0 || c->fg_chunk_tiles < 0)
+      c->rebuild_tiles_per_cta < 0 || c->fg_chunk_tiles < 0 || !(c->rebuild_duty >= 0.f))
     return bad("negative cap_tokens/evict_tokens/n_catchup/num_ctas/chunk tiles");
   if (c->cap_tokens > 0 && c->evict_tokens <= 0) return bad("cap_tokens needs evict_tokens > 0");
   return true;
@@ -490,12 +490,18 @@ static int try_step_schedule(const std::vector<int64_t> &K, int64_t P, int64_t s
                  (static_cast<uint64_t>(pc.j1) << 40);
     S.slot[i] = kSlotNone;
     S.merges[i] = 0;
+    S.share[i] = 0;
   }
   for (int32_t c = 0, i = 0; c <= used; ++c) {
     while (i < static_cast<int32_t>(order.size()) && pcs[order[i]].cta < c) ++i;
     S.first[c] = static_cast<uint16_t>(i);
   }
-  // per unit: the last piece (latest end, then highest CTA) merges the others
+  // per unit: the pieces that end last (its last group) merge the others.  A
+  // group of one, or a unit of at most three pieces: its last member (then
+  // highest CTA) combines the others' partials with its own rows.  A larger
+  // group of g pieces running at the same time: all write partials and each
+  // merges 256 / g of the rows over every partial, so that no single CTA
+  // reads them all.
   std::vector<std::vector<int32_t>> of_unit(U);
   for (int32_t i = 0; i < static_cast<int32_t>(pcs.size()); ++i) of_unit[pcs[i].u].push_back(i);
   int32_t next = 0;
@@ -507,11 +513,25 @@ static int try_step_schedule(const std::vector<int64_t> &K, int64_t P, int64_t s
       return pcs[x].b != pcs[y].b ? pcs[x].b < pcs[y].b : pcs[x].cta < pcs[y].cta;
     });
     const int32_t cnt = static_cast<int32_t>(v.size());
-    if (next + cnt - 1 > kPartialItems / 2) return 0;
-    for (int32_t k = 0; k + 1 < cnt; ++k) S.slot[at[v[k]]] = static_cast<uint16_t>(next + k);
-    S.slot[at[v[cnt - 1]]] = static_cast<uint16_t>(next);
-    S.merges[at[v[cnt - 1]]] = static_cast<uint16_t>(cnt - 1);
-    next += cnt - 1;
+    int32_t g = 0;
+    while (g < cnt && pcs[v[cnt - 1 - g]].b == pcs[v[cnt - 1]].b) ++g;
+    if (cnt <= 3) g = 1;
+    const int32_t parts = g == 1 ? cnt - 1 : cnt;
+    if (next + parts > kPartialItems / 2) return 0;
+    for (int32_t k = 0; k < cnt - g; ++k) S.slot[at[v[k]]] = static_cast<uint16_t>(next + k);
+    if (g == 1) {
+      S.slot[at[v[cnt - 1]]] = static_cast<uint16_t>(next);
+      S.merges[at[v[cnt - 1]]] = static_cast<uint16_t>(parts);
+      S.share[at[v[cnt - 1]]] = static_cast<uint16_t>(1 << 8);
+    } else {
+      for (int32_t k = 0; k < g; ++k) {
+        const int32_t i = at[v[cnt - g + k]];
+        S.slot[i] = static_cast<uint16_t>(next + cnt - g + k);
+        S.merges[i] = static_cast<uint16_t>(parts);
+        S.share[i] = static_cast<uint16_t>(k | (g << 8));
+      }
+    }
+    next += parts;
   }
   S.grid = used;
   S.n_units = U;
@@ -886,6 +906,7 @@ void worker_main(csr_ctx *c) {
       const cudaError_t e = wait_event(c, c->ev_fg_done);
       if (e != cudaSuccess) st = cuda_fail(c, e, "waiting for the foreground work");
     }
+    const auto t_task = std::chrono::steady_clock::now();
     if (!skip && st == CSR_OK) {
       Range range(t.compact ? "csr_rebuild_compact" : "csr_rebuild_chunk");
       if (t.compact) {
@@ -901,6 +922,12 @@ void worker_main(csr_ctx *c) {
         // paced: one task in flight at a time
         if (e == cudaSuccess && paced) e = wait_event(c, c->ev_rb);
         if (e != cudaSuccess) st = cuda_fail(c, e, "recording the rebuild event");
+        // and at most the configured share of wall time
+        const float duty = c->cfg.rebuild_duty;
+        if (st == CSR_OK && paced && duty > 0.f && duty < 1.f) {
+          const double busy = std::chrono::duration<double>(std::chrono::steady_clock::now() - t_task).count();
+          std::this_thread::sleep_for(std::chrono::duration<double>(busy * (1.0 / duty - 1.0)));
+        }
       }
     }
     delete t.compact;
@@ -1707,7 +1734,8 @@ csr_status csr_foreground_schedule(const csr_config *cfg, int64_t L, int32_t n, 
       out.push_back({c, order, static_cast<int32_t>(e & 0xffffu), static_cast<int32_t>((e >> 16) & 0xffffffu),
                      static_cast<int32_t>((e >> 40) & 0xffffffu),
                      S.slot[i] == kSlotNone ? -1 : static_cast<int32_t>(S.slot[i]),
-                     static_cast<int32_t>(S.merges[i])});
+                     static_cast<int32_t>(S.merges[i]), static_cast<int32_t>(S.share[i] >> 8),
+                     static_cast<int32_t>(S.share[i] & 0xffu)});
     }
   *count = static_cast<int32_t>(out.size());
   if (n_slots) *n_slots = S.n_slots;

@@ -65,12 +65,14 @@ struct AttnParams {
 // Schedule of a fused foreground launch (attn_pair_kernel<HD, true>): the
 // pieces (unit, key tiles [j0, j1)) each CTA runs, in order.  Units are
 // numbered u = pair * hkv + head.  A unit cut into several pieces is merged
-// by its last piece (the one that ends last in the schedule): every other
+// by the pieces that end last in the schedule (its last group): every other
 // piece writes its normalised partial rows and log2-sum-exp to a slot and
-// raises that slot's flags; the last piece waits for the flags, combines the
-// partials with its own accumulator and writes the output rows.
+// raises that slot's flags.  A last group of one piece waits for the flags
+// and combines the partials with its own accumulator; the g > 1 pieces of a
+// larger last group (pieces that run at the same time) also write partials,
+// then each merges a share of the unit's 256 rows over all of them.
 constexpr int kMaxStepGrid = 160;
-constexpr int kMaxStepPieces = 2304;    // pieces of one launch, over all CTAs
+constexpr int kMaxStepPieces = 2048;    // pieces of one launch, over all CTAs
 constexpr int kMaxStepIds = 256;        // new pages one fused launch may name
 constexpr uint16_t kSlotNone = 0xffff;
 struct StepSchedule {
@@ -81,10 +83,15 @@ struct StepSchedule {
   uint16_t first[kMaxStepGrid + 1];    // CTA c runs pieces first[c] .. first[c + 1] - 1, in order
   uint64_t piece[kMaxStepPieces];      // unit | j0 << 16 | j1 << 40
   // merges == 0: slot is the partial slot the piece writes, or kSlotNone for a
-  // whole unit (written directly); merges > 0: the piece is its unit's last
-  // and merges the partials of slots slot .. slot + merges - 1
+  // whole unit (written directly).  merges > 0: the piece is in its unit's
+  // last group (share = k | g << 8, member k of g); g == 1: it merges the
+  // partials of slots slot .. slot + merges - 1 into its own rows; g > 1: it
+  // writes slot, and the unit's merges partials are slots
+  // slot - (merges - g) - k .. (the last g of them the group's), of which it
+  // merges rows [k * 256 / g, (k + 1) * 256 / g)
   uint16_t slot[kMaxStepPieces];
   uint16_t merges[kMaxStepPieces];
+  uint16_t share[kMaxStepPieces];
 };
 
 // Fused foreground block (one cooperative launch): RoPE + paged append of the

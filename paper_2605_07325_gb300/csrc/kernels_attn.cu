@@ -66,7 +66,7 @@ namespace csr {
 // of a cut unit instead merges the partials of slots slot .. slot + merges - 1
 // (merges > 0) into its own rows and writes the output.
 struct Seg {
-  int32_t head, pair, slot, merges;
+  int32_t head, pair, slot, merges, share;
   int64_t j0, j1;
   bool complete;
 };
@@ -212,6 +212,11 @@ __device__ __forceinline__ float ld_cg_f(const float *ptr) {
   asm volatile("ld.global.cg.f32 %0, [%1];" : "=f"(v) : "l"(ptr));
   return v;
 }
+__device__ __forceinline__ float2 ld_cg_f2(const float *ptr) {
+  float2 v;
+  asm volatile("ld.global.cg.v2.f32 {%0, %1}, [%2];" : "=f"(v.x), "=f"(v.y) : "l"(ptr));
+  return v;
+}
 
 // ============================================================ configuration
 // Shared memory: Q_A, Q_B, K and V stages, barriers, staged page ids; the
@@ -273,6 +278,7 @@ struct PairWalker {
       s.pair = pair;
       s.slot = it;
       s.merges = 0;
+      s.share = 0;
       s.j0 = j0;
       s.j1 = min(j0 + p.chunk_tiles, kv);
       s.complete = kv <= p.chunk_tiles;
@@ -298,6 +304,7 @@ struct StepWalker {
     s.j1 = static_cast<int64_t>((e >> 40) & 0xffffffu);
     s.slot = S.slot[i];
     s.merges = S.merges[i];
+    s.share = S.share[i];
     s.complete = s.slot == kSlotNone;
     ++i;
     return true;
@@ -514,6 +521,97 @@ __device__ __noinline__ bool step_q_prep(const StepParams &p, uint8_t *qtile, fl
   return true;
 }
 
+// Merge share of a member of a unit's last group (fused form, group of g > 1
+// pieces that run at the same time): rows [k * 256 / g, (k + 1) * 256 / g) of
+// the unit's 256, those of this warpgroup's tile, over the unit's cnt partial
+// slots (every piece's normalised rows and log2-sum-exps, the group's own
+// included): lse = log2 sum_k 2^lse_k, out = sum_k 2^(lse_k - lse) O_k.  One
+// row per warp at a time, HD / 32 columns per lane; the flags of the warp
+// that wrote the row in every piece are awaited first.  False after a failed
+// wait.
+template <int HD>
+__device__ __noinline__ bool step_merge_share(const StepParams &p, const Seg &seg, int T, int wg, int wq,
+                                              int lane, volatile int *abort) {
+  const AttnParams &A = p.a;
+  constexpr int kPer = HD / 32;
+  const int32_t g = seg.share >> 8, k = seg.share & 0xff, cnt = seg.merges;
+  const int64_t s0 = static_cast<int64_t>(seg.slot) - (cnt - g) - k;
+  const int r_a = max(k * kPairRows / g, wg * kBM), r_b = min((k + 1) * kPairRows / g, wg * kBM + kBM);
+  const int tile = seg.pair * 2 + wg;
+  int last_fw = -1;
+  for (int r = r_a + wq; r < r_b; r += 4) {
+    const int rr = r - wg * kBM;
+    const int64_t t = static_cast<int64_t>(tile) * T + rr / A.group;
+    if (tile >= A.n_tiles || t >= A.n) continue;
+    const int fw = r / 32;   // the softmax warp that wrote row r in every piece
+    if (fw != last_fw) {
+      bool got = true;
+      for (int kk = lane; kk < cnt && got; kk += 32)
+        got = wait_counter(p.flags + (s0 + kk) * 8 + fw, p.gen, A.err, abort);
+      if (!__all_sync(0xffffffffu, got)) return false;
+      last_fw = fw;
+    }
+    const float *lse_r = A.part_lse + s0 * kPairRows + r;
+    float mx = -CUDART_INF_F;
+    for (int kk = lane; kk < cnt; kk += 32) mx = fmaxf(mx, ld_cg_f(lse_r + static_cast<int64_t>(kk) * kPairRows));
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
+    const float m_use = mx == -CUDART_INF_F ? 0.f : mx;
+    float sum = 0.f;
+    for (int kk = lane; kk < cnt; kk += 32) sum += ex2_approx(ld_cg_f(lse_r + static_cast<int64_t>(kk) * kPairRows) - m_use);
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, off);
+    const float lse = sum > 0.f ? m_use + log2f(sum) : -CUDART_INF_F;
+    float acc[kPer];
+#pragma unroll
+    for (int c = 0; c < kPer; ++c) acc[c] = 0.f;
+    const float *o_r = A.part_o + (s0 * kPairRows + r) * HD + lane * kPer;
+    for (int k0 = 0; k0 < cnt; k0 += 8) {
+      float lk[8], v[8][kPer];
+#pragma unroll
+      for (int e = 0; e < 8; ++e) {
+        if (k0 + e < cnt) {
+          const int64_t off = static_cast<int64_t>(k0 + e) * kPairRows;
+          lk[e] = ld_cg_f(lse_r + off);
+          if constexpr (kPer == 4) {
+            const float4 x = ld_cg_f4(o_r + off * HD);
+            v[e][0] = x.x; v[e][1] = x.y; v[e][2] = x.z; v[e][3] = x.w;
+          } else {
+            const float2 x = ld_cg_f2(o_r + off * HD);
+            v[e][0] = x.x; v[e][1] = x.y;
+          }
+        }
+      }
+#pragma unroll
+      for (int e = 0; e < 8; ++e) {
+        if (k0 + e < cnt) {
+          const float w = lse == -CUDART_INF_F ? 0.f : ex2_approx(lk[e] - lse);
+#pragma unroll
+          for (int c = 0; c < kPer; ++c) acc[c] = fmaf(w, v[e][c], acc[c]);
+        }
+      }
+    }
+    const int hq_idx = seg.head * A.group + rr % A.group;
+    uint16_t *dst = A.out + (t * A.hq + hq_idx) * HD + lane * kPer;
+    if constexpr (kPer == 4)
+      *reinterpret_cast<uint2 *>(dst) = make_uint2(pack_bf16x2(acc[0], acc[1]), pack_bf16x2(acc[2], acc[3]));
+    else
+      *reinterpret_cast<uint32_t *>(dst) = pack_bf16x2(acc[0], acc[1]);
+    if (lane == 0 && A.lse) A.lse[static_cast<int64_t>(hq_idx) * A.n + t] = lse * 0.69314718055994531f;
+  }
+  return true;
+}
+
+template <int HD>
+__device__ __noinline__ void step_merge_shares(const StepParams &p, int T, int wg, int wq, int lane,
+                                               volatile int *abort) {
+  StepWalker walk = make_walker(p);
+  Seg seg;
+  while (walk.next(p, T, seg))
+    if (seg.merges > 0 && (seg.share >> 8) > 1)
+      if (!step_merge_share<HD>(p, seg, T, wg, wq, lane, abort)) return;
+}
+
 // ============================================================ the kernel
 template <int HD, bool kStep>
 __global__ void __launch_bounds__(kPairThreads, 1)
@@ -631,21 +729,36 @@ __global__ void __launch_bounds__(kPairThreads, 1)
         const int64_t je = min(jb + tiles_per_block, seg.j1);
         const int npages = static_cast<int>(je - jb) * ppt;
         __syncwarp();
-        for (int i = lane; i < npages; i += 32) {
+        // every lane's page-table loads are issued before any is used (one
+        // memory round trip per block instead of one per 32 pages)
+        constexpr int kPer = C::kPtStage / 32;
+        int32_t phys_v[kPer];
+#pragma unroll
+        for (int q = 0; q < kPer; ++q) {
+          const int i = lane + 32 * q;
           const int64_t lp = jb * ppt + i;
-          int32_t phys;
-          if constexpr (kStep) {
-            // the launch's new pages come from its id list: staging never
-            // waits for the append, only the TMA of the new keys does
-            phys = (lp < A.n_pages_valid) ? step_page(p, ids_s, lp) : A.page_table[0];
-          } else {
-            phys = (lp < A.n_pages_valid) ? A.page_table[lp] : A.page_table[0];
+          phys_v[q] = 0;
+          if (i < npages) {
+            if constexpr (kStep) {
+              // the launch's new pages come from its id list: staging never
+              // waits for the append, only the TMA of the new keys does
+              phys_v[q] = (lp < A.n_pages_valid) ? step_page(p, ids_s, lp) : A.page_table[0];
+            } else {
+              phys_v[q] = (lp < A.n_pages_valid) ? A.page_table[lp] : A.page_table[0];
+            }
           }
-          if (phys < 0 || phys >= A.pool_pages) {
-            atomicOr(A.err, CSR_DEVERR_BAD_PAGE);
-            phys = 0;
+        }
+#pragma unroll
+        for (int q = 0; q < kPer; ++q) {
+          const int i = lane + 32 * q;
+          if (i < npages) {
+            int32_t phys = phys_v[q];
+            if (phys < 0 || phys >= A.pool_pages) {
+              atomicOr(A.err, CSR_DEVERR_BAD_PAGE);
+              phys = 0;
+            }
+            stage[i] = phys;
           }
-          stage[i] = phys;
         }
         __syncwarp();
         for (int64_t j = jb; j < je; ++j) {
@@ -931,7 +1044,7 @@ __global__ void __launch_bounds__(kPairThreads, 1)
       if (lane == 0) mbar_arrive(&bars->o_free[wg]);
       bool to_out = seg.complete;
       if constexpr (kStep) {
-        if (seg.merges > 0) {
+        if (seg.merges > 0 && (seg.share >> 8) <= 1) {
           // The unit's last piece: once the other pieces have written this
           // warp's rows (their flags hold this launch's generation), combine
           // lse = log2(2^lse_own + sum_k 2^lse_k) and
@@ -1010,9 +1123,16 @@ __global__ void __launch_bounds__(kPairThreads, 1)
           __threadfence();
           __syncwarp();
           if (lane == 0) st_release_gpu(p.flags + static_cast<int64_t>(seg.slot) * 8 + warp, p.gen);
+          // a member of a last group of several pieces merges its share
+          // after this CTA's last piece
         }
       }
       ++seg_n;
+    }
+    if constexpr (kStep) {
+      // The merge shares of this CTA's pieces in larger last groups (every
+      // flag of this CTA is raised by now, so these waits hold up no one).
+      if (ok) step_merge_shares<HD>(p, T, wg, warp & 3, lane, abort);
     }
   }
 

@@ -59,7 +59,22 @@ def test_random_session_matches_oracle(libcsr, seed):
                 p.ctx.cancel_reconcile()
                 p.orc.cancel()
                 done["cancel"] += 1
-        elif op == "rewind" and not p.orc.is_reconciling and p.orc.chunk_ids():
+        elif op == "rewind" and p.orc.chunk_ids():
+            if p.orc.is_reconciling:
+                # a rewind needs a settled cache: finish the rebuild first (how
+                # many steps it spans depends on the GPU's pace)
+                assert p.ctx.wait_reconcile(60.0) == csr.RECON_SWAPPED
+                expect = p.orc.reconcile()
+                torch.cuda.synchronize()
+                for cid, (eo, _) in expect.items():
+                    assert_close(to_f64(outs[cid]), eo, f"rebuilt chunk {cid}")
+                version += 1
+                done["swap"] += 1
+                assert p.ctx.versions() == (version, version)
+                if not p.orc.chunk_ids():
+                    bseed += 1
+                    p.check_layout()
+                    continue
             ids, lens, pre = p.ctx.chunks(csr.VERSION_ACTIVE)
             keep = int(rng.integers(0, len(ids) + 1))
             length = pre + int(sum(lens[:keep]))

@@ -37,9 +37,9 @@ def _check(pieces, n_slots, K, grid):
     """Coverage, slot bookkeeping and per-CTA order; returns each CTA's load."""
     cover = {u: [] for u in K}
     per_cta = {}
-    for cta, order, u, j0, j1, slot, merges in pieces:
+    for cta, order, u, j0, j1, slot, merges, group, member in pieces:
         assert 0 <= cta < grid and 0 <= j0 < j1 <= K[u]
-        cover[u].append((j0, j1, slot, merges))
+        cover[u].append((j0, j1, slot, merges, group, member))
         per_cta.setdefault(cta, []).append((order, j1 - j0))
     written = []
     for u, segs in cover.items():
@@ -48,13 +48,25 @@ def _check(pieces, n_slots, K, grid):
         for a, b in zip(segs, segs[1:]):
             assert a[1] == b[0], (u, segs)       # contiguous, no overlap
         if len(segs) == 1:
-            assert segs[0][2:] == (-1, 0)         # a whole unit is written directly
+            assert segs[0][2:] == (-1, 0, 0, 0)   # a whole unit is written directly
             continue
         last = [s for s in segs if s[3] > 0]
-        assert len(last) == 1 and last[0][3] == len(segs) - 1, (u, segs)
-        own = sorted(s[2] for s in segs if s[3] == 0)
-        assert own == list(range(last[0][2], last[0][2] + len(segs) - 1)), (u, segs)
-        written += own
+        rest = sorted(s[2] for s in segs if s[3] == 0)
+        g = last[0][4]
+        assert all(s[4] == g for s in last) and len(last) == g >= 1, (u, segs)
+        assert sorted(s[5] for s in last) == list(range(g))
+        if g == 1:
+            # the last piece merges every other piece's slot into its own rows
+            assert last[0][3] == len(segs) - 1
+            assert rest == list(range(last[0][2], last[0][2] + len(segs) - 1)), (u, segs)
+            written += rest
+        else:
+            # every piece writes a slot; the group's are the last g of the unit's
+            assert all(s[3] == len(segs) for s in last) and len(segs) > 3
+            s0 = rest[0] if rest else min(s[2] for s in last)
+            assert rest == list(range(s0, s0 + len(segs) - g))
+            assert all(s[2] == s0 + len(segs) - g + s[5] for s in last), (u, segs)
+            written += rest + [s[2] for s in last]
     assert sorted(written) == list(range(n_slots))
     for cta, items in per_cta.items():
         assert sorted(o for o, _ in items) == list(range(len(items)))
@@ -62,29 +74,33 @@ def _check(pieces, n_slots, K, grid):
 
 
 def _run(pieces):
-    """Execute the schedule as the kernel does; True if every piece finishes."""
+    """Execute the schedule as the kernel does; True if every piece finishes.
+    A piece raises its flag when its attention is done (after any waits of
+    earlier pieces on its CTA); a piece of a last group then waits for the
+    flags of every other piece of its unit before its CTA moves on."""
     seq = {}
     for p in pieces:
         seq.setdefault(p[0], []).append(p)
     for v in seq.values():
         v.sort(key=lambda p: p[1])
-    others = {}
+    of_unit = {}
     for p in pieces:
-        if p[6] == 0 and p[5] >= 0:
-            others.setdefault(p[2], set()).add(p)
-    done, pos = set(), {c: 0 for c in seq}
+        of_unit.setdefault(p[2], set()).add(p)
+    flagged, pos = set(), {c: 0 for c in seq}
     progress = True
     while progress:
         progress = False
         for c, v in seq.items():
             while pos[c] < len(v):
                 p = v[pos[c]]
-                if p[6] > 0 and not others[p[2]] <= done:
+                if p not in flagged:
+                    flagged.add(p)
+                    progress = True
+                if p[6] > 0 and not (of_unit[p[2]] - {p}) <= flagged:
                     break                             # the merging piece waits
-                done.add(p)
                 pos[c] += 1
                 progress = True
-    return len(done) == len(pieces)
+    return all(pos[c] == len(v) for c, v in seq.items())
 
 
 CASES = [
@@ -170,10 +186,22 @@ def test_forced_piece_length(libcsr, chunk, n, L, grid):
     K = _unit_tiles(C2, L, n)
     _check(pieces, n_slots, K, grid)
     assert _run(pieces)
-    longest = max(j1 - j0 for _, _, _, j0, j1, _, _ in pieces)
+    longest = max(p[4] - p[3] for p in pieces)
     # a longer piece only where the cap was grown: pieces at the cap would
     # have overflowed the table, so the grown schedule is still large
     assert len(pieces) <= 2304 and (longest <= chunk or len(pieces) > 2304 // 2)
+
+
+def test_concurrent_pieces_share_the_merge(libcsr):
+    """n = 16 at 128K: four units of 1,025 tiles, each cut into 38 pieces that
+    run at the same time on 38 CTAs; all 38 write partials and the pieces that
+    end last (37 of 27 tiles; one has 26) each merge 6 or 7 of the unit's 256
+    rows, so no CTA reads all 38 partials."""
+    pieces, n_slots = libcsr.foreground_schedule(_cfg(libcsr, C2), 131_072, 16, 152)
+    assert len(pieces) == 152 and n_slots == 152
+    group = [p for p in pieces if p[6] > 0]
+    assert len(group) == 4 * 37 and all(p[7] == 37 and p[6] == 38 for p in group)
+    assert _run(pieces)
 
 
 def test_one_cta_runs_every_unit(libcsr):
