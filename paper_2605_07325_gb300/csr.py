@@ -32,6 +32,7 @@ FLAG_PLAN_ONLY = 0x1
 FLAG_FUSED_ALWAYS = 0x2
 FLAG_FUSED_NEVER = 0x4
 FLAG_UNPACED_REBUILD = 0x8
+FLAG_SCHEDULE_LOCAL = 0x10
 RECON_IDLE, RECON_RUNNING, RECON_SWAPPED = 0, 1, 2
 ROUTE_CONTINUE, ROUTE_BRIDGE, ROUTE_SWAPPED, ROUTE_STRAGGLER = 0, 1, 2, 3
 VERSION_ACTIVE, VERSION_PENDING = 0, 1

@@ -404,7 +404,8 @@ int32_t choose_chunk_tiles(int64_t units, int64_t kv_max, int max_tiles) {
 // pieces in schedule order, so the waits cannot form a cycle.
 // One attempt with segments of at most seg_cap tiles: 1 = scheduled, 0 = more
 // pieces or partial slots than one launch holds, -1 = not schedulable at all.
-static int try_step_schedule(const std::vector<int64_t> &K, int64_t P, int64_t seg_cap, StepSchedule &S) {
+static int try_step_schedule(const std::vector<int64_t> &K, int64_t P, int64_t seg_cap, int64_t quantum,
+                             StepSchedule &S) {
   S = StepSchedule{};
   const int32_t U = static_cast<int32_t>(K.size());
   int64_t W = 0;
@@ -420,61 +421,125 @@ static int try_step_schedule(const std::vector<int64_t> &K, int64_t P, int64_t s
     for (int64_t s = 0; s < m; ++s) seg.push_back({u, s * K[u] / m, (s + 1) * K[u] / m});
   }
   const int64_t V = static_cast<int64_t>(seg.size());
-  struct Act {
-    int64_t a, b;   // schedule times [a, b)
-    int32_t v;
-  };
-  std::vector<Act> act;
-  if (V <= P) {
-    for (int32_t v = 0; v < V; ++v) act.push_back({0, seg[v].j1 - seg[v].j0, v});
-  } else {
-    // idle intervals laid end to end on tracks of length T0
-    int64_t pos = 0;
-    for (int32_t v = 0; v < V; ++v) {
-      const int64_t k = seg[v].j1 - seg[v].j0, d = T0 - k;
-      if (d == 0) {
-        act.push_back({0, T0, v});
-      } else if (pos + d <= T0) {
-        if (pos > 0) act.push_back({0, pos, v});
-        if (pos + d < T0) act.push_back({pos + d, T0, v});
-        pos = pos + d == T0 ? 0 : pos + d;
-      } else {
-        act.push_back({pos + d - T0, pos, v});   // idle [pos, T0) and [0, pos + d - T0)
-        pos = pos + d - T0;
-      }
-    }
-  }
-  std::sort(act.begin(), act.end(), [](const Act &x, const Act &y) {
-    return x.a != y.a ? x.a < y.a : (x.b != y.b ? x.b < y.b : x.v < y.v);
-  });
-  // deal the intervals to CTAs in order of start time: the lowest free CTA
-  std::priority_queue<std::pair<int64_t, int32_t>, std::vector<std::pair<int64_t, int32_t>>,
-                      std::greater<std::pair<int64_t, int32_t>>> busy;   // (end, cta)
-  std::priority_queue<int32_t, std::vector<int32_t>, std::greater<int32_t>> idle;
-  for (int32_t c = 0; c < P; ++c) idle.push(c);
   struct Pc {
     int32_t cta, level, u;
     int64_t b, j0, j1;
   };
   std::vector<Pc> pcs;
   std::vector<int32_t> depth(P, 0);
-  std::vector<int64_t> done(V, 0);   // tiles of each segment dealt so far
   int32_t used = 0;
-  for (const Act &x : act) {
-    while (!busy.empty() && busy.top().first <= x.a) {
-      idle.push(busy.top().second);
-      busy.pop();
+  if (quantum > 0 && V > P) {
+    // Least-advanced first: in steps of at most `quantum` tiles, the P
+    // segments with the least progress run (ties: those already running,
+    // which keep their CTA and extend their piece); a segment that stops
+    // and later resumes on another CTA starts a new piece.
+    std::vector<int64_t> prog(V, 0);
+    std::vector<int32_t> on(P, -1), last_piece(P, -1);
+    std::vector<int32_t> cand;
+    int64_t t = 0;
+    while (true) {
+      cand.clear();
+      for (int32_t v = 0; v < V; ++v)
+        if (seg[v].j0 + prog[v] < seg[v].j1) cand.push_back(v);
+      if (cand.empty()) break;
+      std::vector<char> running(V, 0);
+      for (int32_t c = 0; c < P; ++c)
+        if (on[c] >= 0) running[on[c]] = 1;
+      const size_t m = std::min<size_t>(cand.size(), static_cast<size_t>(P));
+      std::partial_sort(cand.begin(), cand.begin() + m, cand.end(), [&](int32_t x, int32_t y) {
+        if (prog[x] != prog[y]) return prog[x] < prog[y];
+        if (running[x] != running[y]) return running[x] > running[y];
+        return x < y;
+      });
+      std::vector<char> chosen(V, 0);
+      int64_t step = quantum;
+      for (size_t i = 0; i < m; ++i) {
+        chosen[cand[i]] = 1;
+        step = std::min(step, seg[cand[i]].j1 - seg[cand[i]].j0 - prog[cand[i]]);
+      }
+      std::vector<int32_t> next_on(P, -1);
+      std::vector<char> placed(V, 0);
+      for (int32_t c = 0; c < P; ++c)
+        if (on[c] >= 0 && chosen[on[c]]) {
+          next_on[c] = on[c];
+          placed[on[c]] = 1;
+        }
+      int32_t c = 0;
+      for (size_t i = 0; i < m; ++i) {
+        const int32_t v = cand[i];
+        if (placed[v]) continue;
+        while (next_on[c] >= 0) ++c;
+        next_on[c] = v;
+      }
+      for (int32_t cc = 0; cc < P; ++cc) {
+        const int32_t v = next_on[cc];
+        if (v < 0) continue;
+        const int64_t j0 = seg[v].j0 + prog[v];
+        const int32_t lp = last_piece[cc];
+        if (lp >= 0 && on[cc] == v && pcs[lp].b == t) {
+          pcs[lp].j1 += step;   // the segment keeps running on this CTA
+          pcs[lp].b += step;
+        } else {
+          if (static_cast<int64_t>(pcs.size()) >= kMaxStepPieces) return 0;
+          last_piece[cc] = static_cast<int32_t>(pcs.size());
+          pcs.push_back({cc, depth[cc]++, seg[v].u, t + step, j0, j0 + step});
+          used = std::max(used, cc + 1);
+        }
+        prog[v] += step;
+      }
+      on = next_on;
+      t += step;
     }
-    if (idle.empty()) return -1;   // more than P intervals at once: not reachable
-    const int32_t c = idle.top();
-    idle.pop();
-    busy.push({x.b, c});
-    used = std::max(used, c + 1);
-    if (static_cast<int64_t>(pcs.size()) >= kMaxStepPieces) return 0;
-    const Seg &sg = seg[x.v];
-    const int64_t j0 = sg.j0 + done[x.v];
-    done[x.v] += x.b - x.a;
-    pcs.push_back({c, depth[c]++, sg.u, x.b, j0, j0 + (x.b - x.a)});
+  } else {
+    struct Act {
+      int64_t a, b;   // schedule times [a, b)
+      int32_t v;
+    };
+    std::vector<Act> act;
+    if (V <= P) {
+      for (int32_t v = 0; v < V; ++v) act.push_back({0, seg[v].j1 - seg[v].j0, v});
+    } else {
+      // idle intervals laid end to end on tracks of length T0
+      int64_t pos = 0;
+      for (int32_t v = 0; v < V; ++v) {
+        const int64_t k = seg[v].j1 - seg[v].j0, d = T0 - k;
+        if (d == 0) {
+          act.push_back({0, T0, v});
+        } else if (pos + d <= T0) {
+          if (pos > 0) act.push_back({0, pos, v});
+          if (pos + d < T0) act.push_back({pos + d, T0, v});
+          pos = pos + d == T0 ? 0 : pos + d;
+        } else {
+          act.push_back({pos + d - T0, pos, v});   // idle [pos, T0) and [0, pos + d - T0)
+          pos = pos + d - T0;
+        }
+      }
+    }
+    std::sort(act.begin(), act.end(), [](const Act &x, const Act &y) {
+      return x.a != y.a ? x.a < y.a : (x.b != y.b ? x.b < y.b : x.v < y.v);
+    });
+    // deal the intervals to CTAs in order of start time: the lowest free CTA
+    std::priority_queue<std::pair<int64_t, int32_t>, std::vector<std::pair<int64_t, int32_t>>,
+                        std::greater<std::pair<int64_t, int32_t>>> busy;   // (end, cta)
+    std::priority_queue<int32_t, std::vector<int32_t>, std::greater<int32_t>> idle;
+    for (int32_t c = 0; c < P; ++c) idle.push(c);
+    std::vector<int64_t> done(V, 0);   // tiles of each segment dealt so far
+    for (const Act &x : act) {
+      while (!busy.empty() && busy.top().first <= x.a) {
+        idle.push(busy.top().second);
+        busy.pop();
+      }
+      if (idle.empty()) return -1;   // more than P intervals at once: not reachable
+      const int32_t c = idle.top();
+      idle.pop();
+      busy.push({x.b, c});
+      used = std::max(used, c + 1);
+      if (static_cast<int64_t>(pcs.size()) >= kMaxStepPieces) return 0;
+      const Seg &sg = seg[x.v];
+      const int64_t j0 = sg.j0 + done[x.v];
+      done[x.v] += x.b - x.a;
+      pcs.push_back({c, depth[c]++, sg.u, x.b, j0, j0 + (x.b - x.a)});
+    }
   }
   // pieces in CTA order, each CTA's in schedule order
   std::vector<int32_t> order(pcs.size());
@@ -540,10 +605,17 @@ static int try_step_schedule(const std::vector<int64_t> &K, int64_t P, int64_t s
   return 1;
 }
 
+// Key tiles per step of the least-advanced-first schedule (on request): the
+// keys in use at any time stay within about this many tiles of each other
+// (8 MB per head at d = 128), at the cost of a cut wherever a segment stops
+// and resumes on another CTA.
+constexpr int64_t kStepQuantum = 128;
+int64_t step_quantum(const csr_config &cf) { return (cf.flags & CSR_FLAG_SCHEDULE_LOCAL) ? kStepQuantum : 0; }
+
 // The schedule of a block; a forced piece length (cap_tiles > 0) grows by
 // halves while the launch would hold more pieces or slots than it can.
 bool build_step_schedule(int64_t L, int32_t n, int T, int hkv, int32_t n_tiles, int grid_cap,
-                         int cap_tiles, StepSchedule &S) {
+                         int cap_tiles, int64_t quantum, StepSchedule &S) {
   const int32_t pairs = static_cast<int32_t>(ceil_div(n_tiles, 2));
   const int32_t U = pairs * hkv;
   if (U < 1 || U > 0xffff || grid_cap < 1) return false;
@@ -558,11 +630,33 @@ bool build_step_schedule(int64_t L, int32_t n, int T, int hkv, int32_t n_tiles, 
   const int64_t T0 = ceil_div(W, P);
   int64_t cap = cap_tiles > 0 ? std::min<int64_t>(T0, cap_tiles) : T0;
   while (true) {
-    const int r = try_step_schedule(K, P, cap, S);
-    if (r != 0) return r == 1;
+    const int r = try_step_schedule(K, P, cap, 0, S);
+    if (r == -1) return false;
+    if (r == 1) break;
     if (cap >= T0) return false;
     cap = std::min(T0, cap + std::max<int64_t>(1, cap / 2));
   }
+  // The least-advanced-first steps where they keep the load within 1 % of
+  // the idle-interval schedule's (the optimum) and cut at most twice as often:
+  // units of about equal length, a little more than one per CTA.
+  if (quantum > 0) {
+    static thread_local StepSchedule S2;
+    if (try_step_schedule(K, P, cap, quantum, S2) == 1) {
+      auto max_load = [](const StepSchedule &X) {
+        int64_t m = 0;
+        for (int32_t c = 0; c < X.grid; ++c) {
+          int64_t l = 0;
+          for (int32_t i = X.first[c]; i < X.first[c + 1]; ++i)
+            l += static_cast<int64_t>((X.piece[i] >> 40) & 0xffffffu) - static_cast<int64_t>((X.piece[i] >> 16) & 0xffffffu);
+          m = std::max(m, l);
+        }
+        return m;
+      };
+      const int64_t l1 = max_load(S), l2 = max_load(S2);
+      if (l2 * 100 <= l1 * 101 && S2.n_slots <= 2 * S.n_slots + 8) S = S2;
+    }
+  }
+  return true;
 }
 
 cudaEvent_t take_event(csr_ctx *c) {
@@ -628,9 +722,9 @@ csr_status run_block(csr_ctx *c, int slot, int ws, const void *q, const void *k,
 
   // Foreground: one cooperative launch of the fused kernel when the call is
   // long enough for its fixed costs (query preparation and append before the
-  // first tile, merges by the last pieces: tens of microseconds) to vanish,
-  // else three chained launches (the rebuild's path with a persistent grid).
-  // Flags force either.
+  // first tile, merges by the last pieces: tens of microseconds) to vanish
+  // and has at most two units per CTA, else three chained launches (the
+  // rebuild's path with a persistent grid).  Flags force either.
   bool fused = false;
   if (fg) {
     if (cf.flags & CSR_FLAG_FUSED_ALWAYS) {
@@ -640,12 +734,17 @@ csr_status run_block(csr_ctx *c, int slot, int ws, const void *q, const void *k,
       const int64_t pairs = ceil_div(ap.n_tiles, 2);
       for (int64_t pr = 0; pr < pairs; ++pr) tiles += unit_iters(L, n, T, static_cast<int32_t>(2 * pr + 1));
       tiles *= cf.num_kv_heads;
-      fused = tiles >= static_cast<int64_t>(kFusedMinTilesPerCta) * c->fg_grid;
+      // and at most two units per CTA: with more, the fused schedule's units
+      // drift apart in key position and read the cache through L2 less often
+      // than the chunk-major items of the three launches
+      fused = tiles >= static_cast<int64_t>(kFusedMinTilesPerCta) * c->fg_grid &&
+              pairs * cf.num_kv_heads <= 2ll * c->fg_grid;
     }
     if (n_ids > kMaxStepIds) fused = false;   // more new pages than one fused launch names
   }
   StepParams &sp = c->step;
-  if (fused && !build_step_schedule(L, n, T, cf.num_kv_heads, ap.n_tiles, c->fg_grid, cf.fg_chunk_tiles, sp.s)) {
+  if (fused && !build_step_schedule(L, n, T, cf.num_kv_heads, ap.n_tiles, c->fg_grid, cf.fg_chunk_tiles,
+                                    step_quantum(cf), sp.s)) {
     if (cf.flags & CSR_FLAG_FUSED_ALWAYS)
       return fail(c, CSR_EINVAL, "block cannot be scheduled as one fused launch");
     fused = false;
@@ -1724,7 +1823,7 @@ csr_status csr_foreground_schedule(const csr_config *cfg, int64_t L, int32_t n, 
   const int T = kBM / group;
   const int32_t n_tiles = static_cast<int32_t>(ceil_div(static_cast<int64_t>(n) * group, kBM));
   StepSchedule S;
-  if (!build_step_schedule(L, n, T, cfg->num_kv_heads, n_tiles, grid, cfg->fg_chunk_tiles, S))
+  if (!build_step_schedule(L, n, T, cfg->num_kv_heads, n_tiles, grid, cfg->fg_chunk_tiles, step_quantum(*cfg), S))
     return CSR_EINVAL;
   // What each CTA's walker yields, in order.
   std::vector<csr_piece> out;

@@ -15,9 +15,9 @@ C1 = dict(hq=8, hkv=2, d=64, P=16)
 C2 = dict(hq=64, hkv=4, d=128, P=64)
 
 
-def _cfg(libcsr, shape, chunk=0, max_new=8192):
+def _cfg(libcsr, shape, chunk=0, max_new=8192, flags=0):
     return libcsr.make_config(shape["hq"], shape["hkv"], shape["d"], shape["P"], 1e6, max_new, 4096,
-                              1 << 20, flags=libcsr.FLAG_PLAN_ONLY, fg_chunk_tiles=chunk)
+                              1 << 20, flags=libcsr.FLAG_PLAN_ONLY | flags, fg_chunk_tiles=chunk)
 
 
 def _unit_tiles(shape, L, n):
@@ -128,8 +128,14 @@ def test_pieces_cover_balance_and_finish(libcsr, shape, L, n, grid):
     K = _unit_tiles(shape, L, n)
     load = _check(pieces, n_slots, K, grid)
     W = sum(K.values())
-    assert max(load.values()) <= max(-(-W // grid), 1)     # the optimum, to the tile
+    opt = max(-(-W // grid), 1)
+    assert max(load.values()) <= opt             # the idle-interval construction: the optimum
     assert _run(pieces)
+    local, n_local = libcsr.foreground_schedule(_cfg(libcsr, shape, flags=libcsr.FLAG_SCHEDULE_LOCAL), L, n, grid)
+    load_l = _check(local, n_local, K, grid)
+    # least-advanced-first steps only where they stay within 1 % of the optimum
+    assert max(load_l.values()) <= opt * 1.01
+    assert _run(local)
 
 
 def _times(pieces):
@@ -146,24 +152,46 @@ def _times(pieces):
     return out
 
 
+def _spread(pieces):
+    """Largest spread of the key positions the CTAs read at one time, over
+    every tile-time (CTAs run back to back from time 0, one tile per
+    tile-time), per kv head (units u with the same u % 4)."""
+    events = []
+    for t, p in _times(pieces):
+        events.append((t, t + p[4] - p[3], p[2] % 4, p[3]))
+    horizon = max(e[1] for e in events)
+    worst = 0
+    for t in range(0, horizon, 7):
+        pos = {}
+        for a, b, h, j0 in events:
+            if a <= t < b:
+                pos.setdefault(h, []).append(j0 + t - a)
+        worst = max([worst] + [max(v) - min(v) for v in pos.values()])
+    return worst
+
+
 def test_step_120k_cuts_and_locality(libcsr):
-    """The 120K step: 192 units of 960-966 tiles on 152 CTAs.  At most P - 1
-    partial slots (each 256 rows of 512 + 4 bytes, written once and read once:
-    under 15% of the 278.4 MB the step must move), at most three pieces per
-    CTA, and the keys a CTA reads at any time within one idle period (T - K,
-    about 253 tiles: 16 MB of each head's cache) of the schedule time."""
+    """The 120K step: 192 units of 960-966 tiles on 152 CTAs.  The default
+    idle-interval schedule cuts at most P - 1 = 151 units (partials of 256
+    rows of 512 + 4 bytes, written once and read once: under 15 % of the
+    278.4 MB the step must move), runs at most three pieces per CTA and keeps
+    the keys read at any time within one idle period (T - K, ~253 tiles, 16 MB
+    of each head's cache).  With CSR_FLAG_SCHEDULE_LOCAL the least-advanced-
+    first steps of 128 tiles keep them within about one step (8 MB per head)
+    for at most twice the cuts, the load within 1 % of the optimum."""
     pieces, n_slots = libcsr.foreground_schedule(_cfg(libcsr, C2), 122_880, 768, 152)
-    K = _unit_tiles(C2, 122_880, 768)
     assert n_slots <= 151
     assert 2 * n_slots * 256 * (128 * 4 + 4) <= 0.15 * 278.4e6
     per_cta = {}
     for p in pieces:
         per_cta[p[0]] = per_cta.get(p[0], 0) + 1
     assert max(per_cta.values()) <= 3
+    K = _unit_tiles(C2, 122_880, 768)
     T = -(-sum(K.values()) // 152)
-    window = T - min(K.values())
-    for t, p in _times(pieces):
-        assert abs(t - p[3]) <= window + 2, (t, p)
+    assert _spread(pieces) <= T - min(K.values()) + 2
+    local, n_local = libcsr.foreground_schedule(_cfg(libcsr, C2, flags=libcsr.FLAG_SCHEDULE_LOCAL), 122_880, 768, 152)
+    assert 151 < n_local <= 2 * 151 + 8
+    assert _spread(local) <= 128 + 16
 
 
 def test_short_units_run_whole(libcsr):
