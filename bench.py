@@ -498,7 +498,7 @@ def run_ours(args):
                      "traffic": traffic,
                      "kernel": "attn_pair_kernel<128, true>: the whole call in one cooperative "
                                "launch (RoPE + paged append, tcgen05 QK^T and PV over TMA-staged "
-                               "paged K/V, merge of split pieces after a grid barrier)",
+                               "paged K/V, cut units merged by their last pieces)",
                      "launches": att_n, "avg_launch_us": att_ms / max(1, att_n) * 1e3,
                      "peak_source": f"bf16_tflops ({peak_kind}, burst)",
                      "frac_of_sustained": (achieved / peak_sust) if achieved else None},

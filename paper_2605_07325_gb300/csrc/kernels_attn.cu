@@ -28,18 +28,17 @@
 //
 // Two instantiations of attn_pair_kernel:
 //   kStep = true: the foreground block in ONE cooperative launch of one CTA
-//     per SM.  The softmax warps first append the new tokens' rotated keys and
-//     values to the cache (each CTA a share; a device counter tells the
-//     producers when key tiles past position L may be read), then rotate each
-//     unit's queries straight into the shared-memory Q tiles (no packed-query
-//     buffer).  The schedule (StepSchedule) runs whole units in rounds --
-//     every CTA sweeps its unit's keys from the start, so the CTAs of a head
-//     read the same key tiles through L2 at the same time -- and cuts only
-//     the units left over after the last full round into pieces, level by
-//     level, so that each level fills the grid; pieces of one level cover the
-//     same key section of different units.  Pieces write normalised partial
-//     outputs; after a grid barrier (all CTAs are resident: cooperative
-//     launch) every CTA merges a share of the split rows.
+//     per SM.  Every CTA appends a share of the new tokens' rotated keys and
+//     values to the cache (a device counter tells the producers when key
+//     tiles past position L may be read) and rotates each unit's queries
+//     straight into the shared-memory Q tiles (no packed-query buffer).  The
+//     CTAs walk a host-built table of pieces (unit, key tiles [j0, j1)):
+//     pieces of a cut unit write normalised partial outputs and raise per-warp
+//     flags; the unit's last piece waits for those flags and merges the
+//     partials into its own rows (or, when several last pieces run at the
+//     same time, each merges a share of the rows after its CTA's last piece).
+//     No grid barrier: a piece only waits for pieces that end earlier in the
+//     schedule, and every CTA is resident (cooperative launch).
 //   kStep = false: one item (key chunk, head, pair) per CTA or a persistent
 //     round-robin over items, queries read by TMA from the packed buffer that
 //     K1 (rope_append_kernel) wrote; split items are merged by K3
