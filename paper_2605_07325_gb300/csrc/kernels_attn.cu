@@ -343,33 +343,26 @@ __device__ __forceinline__ int32_t step_page(const StepParams &p, const int32_t 
   return (phys < 0 || phys >= A.pool_pages) ? -1 : phys;
 }
 
-// Part of this CTA's share of the append (nthreads threads, tid
-// 0..nthreads-1): rotated keys and values of the new tokens into their cache
-// slots, and (CTA 0, first call) the new pages' ids into the device table.
-// Work items of 16 bytes out: 8 key pairs (two stores) or 8 values.  `cursor`
-// (-1 before the first call) is the thread's next item; at most `rounds`
-// batches of kBatch items are done per call.  Returns true once the thread
-// has no items left.
+// This CTA's share of the append (nthreads threads, tid 0..nthreads-1):
+// rotated keys and values of the new tokens into their cache slots, and
+// (CTA 0) the new pages' ids into the device table.  Work items of 16 bytes
+// out: 8 key pairs (two stores) or 8 values.
 template <int HD>
-__device__ __noinline__ bool step_append(const StepParams &p, const TurnSplit *turns, const int32_t *ids_s, int tid,
-                                         int nthreads, int64_t &cursor, int rounds) {
+__device__ __noinline__ void step_append(const StepParams &p, const TurnSplit *turns, const int32_t *ids_s, int tid,
+                                         int nthreads) {
   const AttnParams &A = p.a;
   constexpr int half = HD / 2, c16 = HD / 16, c8 = HD / 8;
   constexpr int kBatch = 4;   // items whose input loads are in flight together
+  if (blockIdx.x == 0) {
+    int32_t *table = const_cast<int32_t *>(A.page_table);
+    for (int i = tid; i < p.n_ids; i += nthreads) table[p.first_lp + i] = p.ids[i];
+  }
   const int64_t nk = static_cast<int64_t>(A.n) * A.hkv * c16;
   const int64_t nv = static_cast<int64_t>(A.n) * A.hkv * c8;
   // items interleaved over the CTAs (item g = tid * grid + CTA), so a small
   // block spreads over every CTA instead of filling the first ones
   const int64_t stride = static_cast<int64_t>(gridDim.x) * nthreads;
-  if (cursor < 0) {
-    if (blockIdx.x == 0) {
-      int32_t *table = const_cast<int32_t *>(A.page_table);
-      for (int i = tid; i < p.n_ids; i += nthreads) table[p.first_lp + i] = p.ids[i];
-    }
-    cursor = static_cast<int64_t>(tid) * gridDim.x + blockIdx.x;
-  }
-  int64_t w0 = cursor;
-  for (int r = 0; r < rounds && w0 < nk + nv; ++r, w0 += kBatch * stride) {
+  for (int64_t w0 = static_cast<int64_t>(tid) * gridDim.x + blockIdx.x; w0 < nk + nv; w0 += kBatch * stride) {
     uint4 a[kBatch], b[kBatch];
 #pragma unroll
     for (int u = 0; u < kBatch; ++u) {   // the inputs of up to four items
@@ -423,10 +416,7 @@ __device__ __noinline__ bool step_append(const StepParams &p, const TurnSplit *t
       }
     }
   }
-  cursor = w0;
-  if (w0 < nk + nv) return false;
   fence_proxy_async_global();   // the other CTAs read these slots by TMA
-  return true;
 }
 
 // The raw queries of a unit's two query tiles, brought by the producer: one
@@ -699,31 +689,6 @@ __global__ void __launch_bounds__(kPairThreads, 1)
     bool ok = true;
     bool appended = false;   // fused form: the launch's new keys are in the cache
     bool pending = false;
-    // fused form: this warp appends the CTA's share of the new keys and values
-    // a batch at a time between its first tile copies (the other warps start
-    // on the queries at once) and arrives once for the CTA when done.  It
-    // finishes before its first wait that can block -- for a free stage or Q
-    // buffer, which needs this CTA's MMA and softmax warps to progress, and
-    // they may wait for another CTA's piece, whose producer may wait for this
-    // CTA's arrival -- so every CTA's append completes unconditionally.
-    int64_t app_cursor = -1;
-    bool app_done = !kStep;
-    auto append_some = [&](int rounds) {
-      if constexpr (kStep) {
-        if (app_done) return;
-        app_done = __all_sync(0xffffffffu, step_append<HD>(p, turns, ids_s, lane, 32, app_cursor, rounds));
-        if (app_done) {
-          // every lane's stores before the one arrival (a vote does not
-          // order memory; the warp barrier does)
-          __threadfence();
-          __syncwarp();
-          if (lane == 0) red_release_gpu_add(p.sync, 1u);
-        }
-      }
-    };
-    auto finish_append = [&]() {
-      while (!app_done) append_some(1 << 20);
-    };
     if constexpr (kStep) {
       // the first piece's raw queries before waiting for the previous kernel
       // (they are inputs of this call); then every cache access waits
@@ -737,7 +702,6 @@ __global__ void __launch_bounds__(kPairThreads, 1)
     while (ok && (pending || walk.next(p, T, seg))) {
       if constexpr (kStep) {
         if (!pending) {
-          finish_append();
           ok = __all_sync(0xffffffffu, mbar_wait(&bars->q_empty, (q_round - 1) & 1, abort, A.err,
                                                  CSR_DEVERR_WAIT_TIMEOUT));
           if (!ok) break;
@@ -800,7 +764,6 @@ __global__ void __launch_bounds__(kPairThreads, 1)
           if constexpr (kStep) {
             // key tiles at or past the page holding position L hold the new keys
             if (!appended && (j + 1) * ppt > p.new_lp) {
-              finish_append();
               if (lane == 0) ok = wait_counter(p.sync, p.append_target, A.err, abort);
               ok = __shfl_sync(0xffffffffu, ok, 0);
               if (!ok) break;
@@ -810,7 +773,6 @@ __global__ void __launch_bounds__(kPairThreads, 1)
           }
           const int32_t *phys = stage + static_cast<int>(j - jb) * ppt;
           const int ks = k_it % C::kStages;
-          if (k_it >= C::kStages) finish_append();   // the wait below can block
           ok = __all_sync(0xffffffffu, mbar_wait(&bars->k_empty[ks], ((k_it / C::kStages) & 1) ^ 1,
                                                  abort, A.err, CSR_DEVERR_WAIT_TIMEOUT));
           if (!ok) break;
@@ -826,22 +788,9 @@ __global__ void __launch_bounds__(kPairThreads, 1)
           load_kv_tile_if<HD>(leader, A, &A.tm_v, smem + C::kVOff + vs * C::kTileBytes,
                               &bars->v_full[vs], seg.head, phys);
           ++v_it;
-          append_some(1);
-          if constexpr (kStep) {
-            // a unit's last piece merges the other pieces' partials in its
-            // epilogue: have them in L2 by then (eight key tiles ahead)
-            if (seg.merges > 0 && (seg.share >> 8) <= 1 && j == max(seg.j0, seg.j1 - 8) && leader) {
-              for (int k = 0; k < seg.merges; ++k) {
-                const int64_t slot = static_cast<int64_t>(seg.slot) + k;
-                bulk_prefetch_l2(A.part_o + slot * kPairRows * HD, kPairRows * HD * 4);
-                bulk_prefetch_l2(A.part_lse + slot * kPairRows, kPairRows * 4);
-              }
-            }
-          }
         }
       }
     }
-    if (ok) finish_append();
     if (!ok && lane == 0) {
       if (q_round > 0) drain_wait(kStep ? &bars->qraw_full : &bars->q_full, (q_round - 1) & 1);
       for (uint32_t i = (k_it > C::kStages ? k_it - C::kStages : 0); i < k_it; ++i)
@@ -861,7 +810,19 @@ __global__ void __launch_bounds__(kPairThreads, 1)
     uint32_t q_round = 0, k_it = 0, v_it = 0, seg_n = 0;
     uint32_t pv_n[2] = {0, 0};
     bool ok = true;
-    if constexpr (kStep) pdl_wait();
+    if constexpr (kStep) {
+      pdl_wait();
+      if (p.append_by_mma) {
+        // few new tokens: this warp appends the CTA's share while the softmax
+        // warps rotate the first queries, then arrives once for the CTA
+        step_append<HD>(p, turns, ids_s, lane, 32);
+        __syncwarp();
+        if (lane == 0) {
+          __threadfence();
+          red_release_gpu_add(p.sync, 1u);
+        }
+      }
+    }
     auto wait = [&](uint64_t *bar, uint32_t parity) {
       if (ok)
         ok = __all_sync(0xffffffffu, mbar_wait(bar, parity, abort, A.err, CSR_DEVERR_WAIT_TIMEOUT));
@@ -960,6 +921,16 @@ __global__ void __launch_bounds__(kPairThreads, 1)
                                       seg.pair, wg, row, lane, T))
         ok = false;
       pdl_wait();
+      if (!p.append_by_mma) {
+        // this CTA's share of the new keys/values, then one arrival per CTA
+        // (every softmax thread gets here exactly once)
+        step_append<HD>(p, turns, ids_s, threadIdx.x, 256);
+        named_sync(3, 256);
+        if (threadIdx.x == 0) {
+          __threadfence();
+          red_release_gpu_add(p.sync, 1u);
+        }
+      }
     }
     while (ok && (pending || walk.next(p, T, seg))) {
       pending = false;

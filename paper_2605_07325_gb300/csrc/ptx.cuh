@@ -100,12 +100,6 @@ __device__ __forceinline__ void tma_load_2d(void *dst, const CUtensorMap *map, u
       : "memory");
 }
 
-// Bring `bytes` (a multiple of 16, from a 16-byte aligned address) of global
-// memory into L2 without waiting for it.
-__device__ __forceinline__ void bulk_prefetch_l2(const void *src, uint32_t bytes) {
-  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(src), "r"(bytes) : "memory");
-}
-
 // 1-D bulk copy of `bytes` (a multiple of 16; both addresses 16-byte aligned)
 // from global to this CTA's shared memory, completing on `bar`.
 __device__ __forceinline__ void bulk_load_1d(void *dst, const void *src, uint32_t bytes, uint64_t *bar) {
