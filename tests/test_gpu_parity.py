@@ -274,3 +274,25 @@ def test_merge_many_chunks_per_row(libcsr, shape, chunk_tiles, path):
     p.suffix(p.blk(74, 100))
     p.truncate()
     p.device_clean()
+
+
+@pytest.mark.parametrize("num_ctas", [7, 19])
+def test_local_schedule_matches_oracle(libcsr, num_ctas):
+    """CSR_FLAG_SCHEDULE_LOCAL: the least-advanced-first pieces (taken on
+    these shapes: 300-token suffixes over 2,000-8,000 cached tokens on 7 or 19
+    CTAs, where they stay within 1 % of the optimum load) merge back to the
+    oracle like the default idle-interval pieces."""
+    csr = csr_mod()
+    p = Pair(C2, pool_pages=256, max_seq=12000, max_new=4096, num_ctas=num_ctas,
+             flags=PATHS["fused"] | csr.FLAG_SCHEDULE_LOCAL)
+    p.init_static(p.blk(80, 2000), compare=False)
+    p.suffix(p.blk(81, 300))
+    p.truncate()
+    p.append(p.blk(82, 2000), compare=False)
+    p.suffix(p.blk(83, 300))
+    p.truncate()
+    p.append(p.blk(84, 4000), compare=False)
+    p.suffix(p.blk(85, 300))
+    p.truncate()
+    p.check_layout()
+    p.device_clean()

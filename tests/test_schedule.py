@@ -3,12 +3,14 @@
 For every block shape the pieces must cover each unit's key tiles [0, K(u))
 exactly once -- K(u) from the causal rule, key range [0, L + last token of the
 pair).  A unit run as one piece is written directly; of a cut unit, every
-piece but one writes its own partial slot and the remaining piece merges all
-of them.  Every CTA's load must be within the optimum ceil(W / P) tiles, the
-merge waits must not be able to deadlock (checked by running the schedule as
-the kernel would: a CTA takes its pieces in order and the merging piece
-finishes only once the others have), and the keys in use at any time must
-stay within a narrow window (the cache is then read through L2 about once)."""
+piece but its last writes its own partial slot and the last merges them (or,
+when several last pieces run at the same time, all write slots and each
+merges a share of the rows).  Every CTA's load must be the optimum ceil(W / P)
+tiles (within 1 % for the least-advanced-first steps), the merge waits must
+not be able to deadlock (checked by running the schedule as the kernel would:
+a CTA takes its pieces in order and a merging piece finishes only once the
+others have raised their flags), and the keys in use at any time must stay
+within the schedule's window."""
 import pytest
 
 C1 = dict(hq=8, hkv=2, d=64, P=16)
