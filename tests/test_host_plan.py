@@ -173,7 +173,8 @@ def test_error_codes_and_no_state_change(libcsr):
 @pytest.mark.parametrize("bad", [dict(head_dim=96), dict(page_size=48), dict(num_q_heads=12),
                                  dict(num_kv_heads=3), dict(max_new_tokens=0),
                                  dict(pool_pages=0), dict(pool_pages=70000),
-                                 dict(cap_tokens=10, evict_tokens=0)])
+                                 dict(cap_tokens=10, evict_tokens=0), dict(rebuild_duty=-0.5),
+                                 dict(rebuild_duty=float("nan")), dict(fg_chunk_tiles=-1)])
 def test_invalid_configs_rejected(libcsr, bad):
     kw = dict(num_q_heads=8, num_kv_heads=2, head_dim=64, page_size=16, rope_base=1e4,
               max_new_tokens=64, pool_pages=16, max_seq_tokens=256,
