@@ -522,24 +522,24 @@ __device__ __noinline__ bool step_q_prep(const StepParams &p, uint8_t *qtile, fl
 
 // Merge share of a member of a unit's last group (fused form, group of g > 1
 // pieces that run at the same time): rows [k * 256 / g, (k + 1) * 256 / g) of
-// the unit's 256, those of this warpgroup's tile, over the unit's cnt partial
-// slots (every piece's normalised rows and log2-sum-exps, the group's own
+// the unit's 256, spread over the CTA's eight softmax warps, over the unit's
+// cnt partial slots (every piece's normalised rows and log2-sum-exps, the group's own
 // included): lse = log2 sum_k 2^lse_k, out = sum_k 2^(lse_k - lse) O_k.  One
 // row per warp at a time, HD / 32 columns per lane; the flags of the warp
 // that wrote the row in every piece are awaited first.  False after a failed
 // wait.
 template <int HD>
-__device__ __noinline__ bool step_merge_share(const StepParams &p, const Seg &seg, int T, int wg, int wq,
-                                              int lane, volatile int *abort) {
+__device__ __noinline__ bool step_merge_share(const StepParams &p, const Seg &seg, int T, int w8, int lane,
+                                              volatile int *abort) {
   const AttnParams &A = p.a;
   constexpr int kPer = HD / 32;
   const int32_t g = seg.share >> 8, k = seg.share & 0xff, cnt = seg.merges;
   const int64_t s0 = static_cast<int64_t>(seg.slot) - (cnt - g) - k;
-  const int r_a = max(k * kPairRows / g, wg * kBM), r_b = min((k + 1) * kPairRows / g, wg * kBM + kBM);
-  const int tile = seg.pair * 2 + wg;
+  const int r_a = k * kPairRows / g, r_b = (k + 1) * kPairRows / g;
   int last_fw = -1;
-  for (int r = r_a + wq; r < r_b; r += 4) {
-    const int rr = r - wg * kBM;
+  for (int r = r_a + w8; r < r_b; r += 8) {   // rows over all eight softmax warps
+    const int tile = seg.pair * 2 + r / kBM;
+    const int rr = r % kBM;
     const int64_t t = static_cast<int64_t>(tile) * T + rr / A.group;
     if (tile >= A.n_tiles || t >= A.n) continue;
     const int fw = r / 32;   // the softmax warp that wrote row r in every piece
@@ -551,16 +551,29 @@ __device__ __noinline__ bool step_merge_share(const StepParams &p, const Seg &se
       last_fw = fw;
     }
     const float *lse_r = A.part_lse + s0 * kPairRows + r;
-    float mx = -CUDART_INF_F;
-    for (int kk = lane; kk < cnt; kk += 32) mx = fmaxf(mx, ld_cg_f(lse_r + static_cast<int64_t>(kk) * kPairRows));
+    // lse = log2 sum_k 2^lse_k in one pass: a running (max, sum) per lane,
+    // then combined over the warp
+    float mx = -CUDART_INF_F, sum = 0.f;
+    for (int kk = lane; kk < cnt; kk += 32) {
+      const float x = ld_cg_f(lse_r + static_cast<int64_t>(kk) * kPairRows);
+      if (x > mx) {
+        sum = (mx == -CUDART_INF_F ? 0.f : sum * ex2_approx(mx - x)) + 1.f;
+        mx = x;
+      } else if (x != -CUDART_INF_F) {
+        sum += ex2_approx(x - mx);
+      }
+    }
 #pragma unroll
-    for (int off = 16; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
-    const float m_use = mx == -CUDART_INF_F ? 0.f : mx;
-    float sum = 0.f;
-    for (int kk = lane; kk < cnt; kk += 32) sum += ex2_approx(ld_cg_f(lse_r + static_cast<int64_t>(kk) * kPairRows) - m_use);
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, off);
-    const float lse = sum > 0.f ? m_use + log2f(sum) : -CUDART_INF_F;
+    for (int off = 16; off > 0; off >>= 1) {
+      const float m2 = __shfl_xor_sync(0xffffffffu, mx, off);
+      const float s2 = __shfl_xor_sync(0xffffffffu, sum, off);
+      const float m = fmaxf(mx, m2);
+      if (m != -CUDART_INF_F)
+        sum = (mx == -CUDART_INF_F ? 0.f : sum * ex2_approx(mx - m)) +
+              (m2 == -CUDART_INF_F ? 0.f : s2 * ex2_approx(m2 - m));
+      mx = m;
+    }
+    const float lse = sum > 0.f ? mx + log2f(sum) : -CUDART_INF_F;
     float acc[kPer];
 #pragma unroll
     for (int c = 0; c < kPer; ++c) acc[c] = 0.f;
@@ -602,13 +615,12 @@ __device__ __noinline__ bool step_merge_share(const StepParams &p, const Seg &se
 }
 
 template <int HD>
-__device__ __noinline__ void step_merge_shares(const StepParams &p, int T, int wg, int wq, int lane,
-                                               volatile int *abort) {
+__device__ __noinline__ void step_merge_shares(const StepParams &p, int T, int w8, int lane, volatile int *abort) {
   StepWalker walk = make_walker(p);
   Seg seg;
   while (walk.next(p, T, seg))
     if (seg.merges > 0 && (seg.share >> 8) > 1)
-      if (!step_merge_share<HD>(p, seg, T, wg, wq, lane, abort)) return;
+      if (!step_merge_share<HD>(p, seg, T, w8, lane, abort)) return;
 }
 
 // ============================================================ the kernel
@@ -1131,7 +1143,7 @@ __global__ void __launch_bounds__(kPairThreads, 1)
     if constexpr (kStep) {
       // The merge shares of this CTA's pieces in larger last groups (every
       // flag of this CTA is raised by now, so these waits hold up no one).
-      if (ok) step_merge_shares<HD>(p, T, wg, warp & 3, lane, abort);
+      if (ok) step_merge_shares<HD>(p, T, warp, lane, abort);
     }
   }
 
