@@ -766,12 +766,6 @@ csr_status run_block(csr_ctx *c, int slot, int ws, const void *q, const void *k,
     sp.first_lp = first_lp;
     sp.n_ids = n_ids;
     sp.new_lp = static_cast<int32_t>(L / cf.page_size);
-    // The append's 16-byte work items: up to two per lane of one warp per CTA
-    // go to the MMA warp (idle until the first queries and keys are in
-    // place); more go to the eight softmax warps, after their first queries
-    // (one warp alone takes tens of microseconds over a few hundred tokens).
-    const int64_t append_items = static_cast<int64_t>(n) * cf.num_kv_heads * (cf.head_dim / 16 + cf.head_dim / 8);
-    sp.append_by_mma = append_items <= 2ll * 32 * sp.s.grid ? 1 : 0;
     std::memcpy(sp.inv_turns, c->turns, sizeof(sp.inv_turns));
     for (int i = 0; i < n_ids; ++i) sp.ids[i] = ids[i];
     cudaError_t e =

@@ -110,7 +110,6 @@ struct StepParams {
   uint32_t gen;            // this launch's generation (never 0; stale flags hold older ones)
   int32_t first_lp, n_ids; // logical pages first_lp.. get ids[] (written to the table by CTA 0)
   int32_t new_lp;          // logical page holding position L: key tiles reaching it wait for the append
-  int32_t append_by_mma;   // 1: the MMA warp appends (few tokens); 0: the softmax warps
   TurnSplit inv_turns[kMaxHalfDim];
   int32_t ids[kMaxStepIds];
   StepSchedule s;

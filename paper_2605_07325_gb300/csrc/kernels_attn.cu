@@ -822,19 +822,7 @@ __global__ void __launch_bounds__(kPairThreads, 1)
     uint32_t q_round = 0, k_it = 0, v_it = 0, seg_n = 0;
     uint32_t pv_n[2] = {0, 0};
     bool ok = true;
-    if constexpr (kStep) {
-      pdl_wait();
-      if (p.append_by_mma) {
-        // few new tokens: this warp appends the CTA's share while the softmax
-        // warps rotate the first queries, then arrives once for the CTA
-        step_append<HD>(p, turns, ids_s, lane, 32);
-        __syncwarp();
-        if (lane == 0) {
-          __threadfence();
-          red_release_gpu_add(p.sync, 1u);
-        }
-      }
-    }
+    if constexpr (kStep) pdl_wait();
     auto wait = [&](uint64_t *bar, uint32_t parity) {
       if (ok)
         ok = __all_sync(0xffffffffu, mbar_wait(bar, parity, abort, A.err, CSR_DEVERR_WAIT_TIMEOUT));
@@ -933,15 +921,13 @@ __global__ void __launch_bounds__(kPairThreads, 1)
                                       seg.pair, wg, row, lane, T))
         ok = false;
       pdl_wait();
-      if (!p.append_by_mma) {
-        // this CTA's share of the new keys/values, then one arrival per CTA
-        // (every softmax thread gets here exactly once)
-        step_append<HD>(p, turns, ids_s, threadIdx.x, 256);
-        named_sync(3, 256);
-        if (threadIdx.x == 0) {
-          __threadfence();
-          red_release_gpu_add(p.sync, 1u);
-        }
+      // this CTA's share of the new keys/values, then one arrival per CTA
+      // (every softmax thread gets here exactly once)
+      step_append<HD>(p, turns, ids_s, threadIdx.x, 256);
+      named_sync(3, 256);
+      if (threadIdx.x == 0) {
+        __threadfence();
+        red_release_gpu_add(p.sync, 1u);
       }
     }
     while (ok && (pending || walk.next(p, T, seg))) {
