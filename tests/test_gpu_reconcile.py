@@ -112,12 +112,17 @@ def test_automatic_eviction_and_repeated_cycles(libcsr):
     p.device_clean()
 
 
-def test_fused_steps_through_eviction_cycles(libcsr):
+@pytest.mark.parametrize("pacing", ["paced", "unpaced", "duty"])
+def test_fused_steps_through_eviction_cycles(libcsr, pacing):
     """Fused chunk + suffix steps: tau_mem reached by a fused step starts the
     eviction at its truncation; fused steps during the reconciliation fork
-    only their chunk; two cycles against the oracle."""
+    only their chunk; two cycles against the oracle -- with the rebuild paced
+    (one task in flight after the foreground work, the default), unpaced
+    (CSR_FLAG_UNPACED_REBUILD) and held to half of the wall time."""
     csr = csr_mod()
-    p = Pair(C1, pool_pages=256, max_seq=4096, max_new=256, cap_tokens=400, evict_tokens=128)
+    kw = {"paced": {}, "unpaced": {"flags": csr.FLAG_UNPACED_REBUILD},
+          "duty": {"rebuild_duty": 0.5}}[pacing]
+    p = Pair(C1, pool_pages=256, max_seq=4096, max_new=256, cap_tokens=400, evict_tokens=128, **kw)
     lo = torch.cuda.Stream(priority=0)
     outs = {}
     p.ctx.set_reconciler(_provider(p, outs), lo)
