@@ -131,7 +131,7 @@ struct MergeParams {
 // with at most kMergeChunksPerSlot partial rows in flight; rows of more
 // chunks are spread over 2, 4, ... slots (up to a whole block of
 // 256 / (head_dim / 8) slots, which then loops over its chunks).
-constexpr int kMergeChunksPerSlot = 4;
+constexpr int kMergeChunksPerSlot = 5;
 inline int32_t merge_slots_per_row(int64_t max_chunks, int head_dim) {
   const int32_t block_slots = 256 / (head_dim / 8);
   int32_t spr = 1;

@@ -255,6 +255,21 @@ struct PairBars {
 
 constexpr int kPairThreads = 320;
 
+// Item form: the packed queries of an item's two tiles into the Q slots.
+template <int HD>
+__device__ __forceinline__ void item_q_issue(uint32_t leader, const AttnParams &A, uint8_t *smem, uint64_t *q_full,
+                                             const Seg &seg) {
+  using C = PairCfg<HD>;
+  mbar_arrive_expect_tx_if(leader, q_full, 2 * C::kQBytes);
+  const int32_t qrow = seg.head * A.rows_cap + seg.pair * 2 * kBM;
+#pragma unroll
+  for (int h = 0; h < 2; ++h)
+#pragma unroll
+    for (int b = 0; b < C::kBoxes; ++b)
+      tma_load_2d_if(leader, smem + C::kQOff + h * C::kQBytes + b * (kBM * 128), &A.tm_q, q_full, b * 64,
+                     qrow + h * kBM);
+}
+
 // ============================================================ work walkers
 // Items of the non-fused form: (chunk, head, pair); the pair's key range is
 // that of its second tile.
@@ -679,11 +694,17 @@ __global__ void __launch_bounds__(kPairThreads, 1)
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
-  // The cache, the page table and the partial buffers may still be read or
-  // written by the previous kernel: every role waits for it before its first
-  // access to them.  The fused form's softmax warps first rotate their first
-  // queries (inputs of this call, not written by the previous kernel).
-  if constexpr (!kStep) pdl_wait();
+  // Fused form: the cache, the page table and the partial buffers may still
+  // be read or written by the previous kernel, so every role waits for it
+  // before its first access to them (the softmax warps first rotate their
+  // first queries, inputs of this call).  Item form: the previous kernel is
+  // K1, which lets this grid start only once every earlier kernel of the
+  // stream has completed; K1 itself writes the packed queries, the keys and
+  // values at positions >= L and the page-table entries of the new pages.
+  // The MMA warp waits for K1 and issues the first item's queries; the
+  // producer stages page ids and loads cached K/V tiles meanwhile, and waits
+  // for K1 only before a block that reaches position L.  The partial and
+  // output buffers were last read by kernels that completed before K1 started.
   const uint32_t tmem = bars->tmem_base;
   volatile int *abort = &bars->abort;
   auto walk = make_walker(p);
@@ -701,6 +722,13 @@ __global__ void __launch_bounds__(kPairThreads, 1)
     bool ok = true;
     bool appended = false;   // fused form: the launch's new keys are in the cache
     bool pending = false;
+    bool waited = kStep;     // item form: K1 has completed (griddepcontrol.wait passed)
+    auto await_k1 = [&] {
+      if (!waited) {
+        pdl_wait();
+        waited = true;
+      }
+    };
     if constexpr (kStep) {
       // the first piece's raw queries before waiting for the previous kernel
       // (they are inputs of this call); then every cache access waits
@@ -722,23 +750,22 @@ __global__ void __launch_bounds__(kPairThreads, 1)
         }
         pending = false;
       } else {
-        if (q_round > 0)
+        // the first item's queries are issued by the MMA warp once K1 is done
+        if (q_round > 0) {
           ok = __all_sync(0xffffffffu, mbar_wait(&bars->q_empty, (q_round - 1) & 1, abort, A.err,
                                                  CSR_DEVERR_WAIT_TIMEOUT));
-        if (!ok) break;
-        mbar_arrive_expect_tx_if(leader, &bars->q_full, 2 * C::kQBytes);
-        const int32_t qrow = seg.head * A.rows_cap + seg.pair * 2 * kBM;
-#pragma unroll
-        for (int h = 0; h < 2; ++h)
-#pragma unroll
-          for (int b = 0; b < C::kBoxes; ++b)
-            tma_load_2d_if(leader, smem + C::kQOff + h * C::kQBytes + b * (kBM * 128), &A.tm_q,
-                           &bars->q_full, b * 64, qrow + h * kBM);
+          if (!ok) break;
+          await_k1();
+          item_q_issue<HD>(leader, A, smem, &bars->q_full, seg);
+        }
         ++q_round;
       }
       for (int64_t jb = seg.j0; ok && jb < seg.j1; jb += tiles_per_block) {
         const int64_t je = min(jb + tiles_per_block, seg.j1);
         const int npages = static_cast<int>(je - jb) * ppt;
+        // item form: a block reaching position L stages page ids K1 may write
+        if constexpr (!kStep)
+          if (je * kBN > A.L) await_k1();
         __syncwarp();
         // every lane's page-table loads are issued before any is used (one
         // memory round trip per block instead of one per 32 pages)
@@ -803,6 +830,9 @@ __global__ void __launch_bounds__(kPairThreads, 1)
         }
       }
     }
+    // every CTA of the item form waits for K1 before it completes, so that a
+    // kernel after this one that waits for it also waits for K1
+    if constexpr (!kStep) await_k1();
     if (!ok && lane == 0) {
       if (q_round > 0) drain_wait(kStep ? &bars->qraw_full : &bars->q_full, (q_round - 1) & 1);
       for (uint32_t i = (k_it > C::kStages ? k_it - C::kStages : 0); i < k_it; ++i)
@@ -822,7 +852,19 @@ __global__ void __launch_bounds__(kPairThreads, 1)
     uint32_t q_round = 0, k_it = 0, v_it = 0, seg_n = 0;
     uint32_t pv_n[2] = {0, 0};
     bool ok = true;
-    if constexpr (kStep) pdl_wait();
+    if constexpr (kStep) {
+      pdl_wait();
+    } else {
+      // Item form: the first item's queries as soon as K1 is done (they are
+      // K1's output); the producer meanwhile stages page ids and the first
+      // cached K/V tiles.
+      PairWalker first{static_cast<int32_t>(blockIdx.x)};
+      Seg s0;
+      if (first.next(A, T, s0)) {
+        pdl_wait();
+        item_q_issue<HD>(elect_lane(), A, smem, &bars->q_full, s0);
+      }
+    }
     auto wait = [&](uint64_t *bar, uint32_t parity) {
       if (ok)
         ok = __all_sync(0xffffffffu, mbar_wait(bar, parity, abort, A.err, CSR_DEVERR_WAIT_TIMEOUT));

@@ -22,10 +22,6 @@ namespace csr {
 // sincospi, so positions past 10^5 keep full fp32 angle accuracy).
 __global__ void __launch_bounds__(256) rope_append_kernel(const __grid_constant__ RopeAppendParams p) {
   __shared__ float cs[kMaxHalfDim], sn[kMaxHalfDim];
-  // The attention kernel may launch now: its setup (barriers, TMEM, tensor
-  // maps) overlaps this kernel, and it waits for this grid's writes before
-  // touching queries, keys or the page table.
-  pdl_launch_dependents();
   const int t = blockIdx.x;
   const int64_t pos = p.pos0 + t;
   const int half = p.d / 2;
@@ -33,6 +29,12 @@ __global__ void __launch_bounds__(256) rope_append_kernel(const __grid_constant_
   // The previous kernel of the stream may still read the packed queries and
   // cache pages this block overwrites.
   pdl_wait();
+  // The attention kernel may launch now (its setup overlaps this kernel).
+  // Triggering only after the wait means that when it starts, every earlier
+  // kernel of the stream has completed: it may read the cached keys before
+  // position pos0 and their page-table entries at once, and waits for this
+  // grid only before the queries, the new keys and the new pages.
+  pdl_launch_dependents();
   if (blockIdx.x == 0 && blockIdx.y == 0 && p.n_ids > 0) {
     for (int i = threadIdx.x; i < p.n_ids; i += blockDim.x) p.page_table[p.first_lp + i] = p.ids[i];
   }
