@@ -158,7 +158,7 @@ bool encode_queries(CUtensorMap *m, const void *q, uint64_t n, uint64_t hq, uint
 }
 
 struct Layout {  // workspace carve-out (byte offsets)
-  size_t qpack[2], rb_out, part_o[2], part_lse[2], pt[2], ids_out, err, sync, flags, total;
+  size_t qpack[2], rb_out, part_o[2], part_scale[2], part_lse[2], pt[2], ids_out, err, sync, flags, total;
   int32_t rows_cap, max_pages;
 };
 
@@ -209,7 +209,8 @@ Layout make_layout(const csr_config *c) {
   for (int i = 0; i < 2; ++i) L.qpack[i] = take(static_cast<size_t>(c->num_kv_heads) * L.rows_cap * d * 2);
   L.rb_out = take(static_cast<size_t>(c->max_new_tokens) * c->num_q_heads * d * 2);
   for (int i = 0; i < 2; ++i) {
-    L.part_o[i] = take(static_cast<size_t>(kPartialItems) * kBM * d * 4);
+    L.part_o[i] = take(static_cast<size_t>(kPartialItems) * kBM * d * 2);   // fp16
+    L.part_scale[i] = take(static_cast<size_t>(kPartialItems) * kBM * 4);
     L.part_lse[i] = take(static_cast<size_t>(kPartialItems) * kBM * 4);
   }
   for (int i = 0; i < 2; ++i) L.pt[i] = take(static_cast<size_t>(L.max_pages) * 4);
@@ -704,7 +705,8 @@ csr_status run_block(csr_ctx *c, int slot, int ws, const void *q, const void *k,
   ap.page_table = c->d_pt(slot);
   ap.out = static_cast<uint16_t *>(out);
   ap.lse = lse;
-  ap.part_o = c->wsp<float>(c->lay.part_o[ws]);
+  ap.part_o = c->wsp<uint16_t>(c->lay.part_o[ws]);
+  ap.part_scale = c->wsp<float>(c->lay.part_scale[ws]);
   ap.part_lse = c->wsp<float>(c->lay.part_lse[ws]);
   ap.err = c->wsp<uint32_t>(c->lay.err);
   ap.L = L;
@@ -830,6 +832,7 @@ csr_status run_block(csr_ctx *c, int slot, int ws, const void *q, const void *k,
   if (n_chunks > 1) {
     MergeParams mp{};
     mp.part_o = ap.part_o;
+    mp.part_scale = ap.part_scale;
     mp.part_lse = ap.part_lse;
     mp.out = ap.out;
     mp.lse = lse;

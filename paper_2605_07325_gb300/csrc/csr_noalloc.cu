@@ -19,7 +19,7 @@ namespace {
 using namespace csr;
 
 constexpr size_t kQBytes = 8ull << 20;     // packed rotated queries
-constexpr size_t kPartOBytes = 24ull << 20; // split partial outputs (fp32)
+constexpr size_t kPartOBytes = 24ull << 20; // split partials: fp16 rows, then (from the middle) their scales
 constexpr size_t kPartLseBytes = 512ull << 10;
 constexpr size_t kErrBytes = 256;
 constexpr size_t kScratchBytes = kQBytes + kPartOBytes + kPartLseBytes + kErrBytes;
@@ -151,7 +151,10 @@ extern "C" csr_status csr_attend_block_noalloc(const csr_block_args *a, csr_stre
   csr_status st = setup_device(dev, &ds);
   if (st != CSR_OK) return st;
   uint16_t *q_pack = reinterpret_cast<uint16_t *>(ds->scratch);
-  float *part_o = reinterpret_cast<float *>(ds->scratch + kQBytes);
+  // the item cap below counts 4 bytes per value, so the fp16 rows fit the
+  // first half and their scales (4 bytes per row) the second
+  uint16_t *part_o = reinterpret_cast<uint16_t *>(ds->scratch + kQBytes);
+  float *part_scale = reinterpret_cast<float *>(ds->scratch + kQBytes + kPartOBytes / 2);
   float *part_lse = reinterpret_cast<float *>(ds->scratch + kQBytes + kPartOBytes);
   uint32_t *err = reinterpret_cast<uint32_t *>(ds->scratch + kQBytes + kPartOBytes + kPartLseBytes);
   const cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
@@ -199,6 +202,7 @@ extern "C" csr_status csr_attend_block_noalloc(const csr_block_args *a, csr_stre
   ap.out = static_cast<uint16_t *>(a->out);
   ap.lse = a->lse;
   ap.part_o = part_o;
+  ap.part_scale = part_scale;
   ap.part_lse = part_lse;
   ap.err = err;
   ap.L = a->L;
@@ -241,6 +245,7 @@ extern "C" csr_status csr_attend_block_noalloc(const csr_block_args *a, csr_stre
   if (n_chunks > 1) {
     MergeParams mp{};
     mp.part_o = part_o;
+    mp.part_scale = part_scale;
     mp.part_lse = part_lse;
     mp.out = ap.out;
     mp.lse = a->lse;

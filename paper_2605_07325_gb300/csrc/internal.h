@@ -51,8 +51,13 @@ struct AttnParams {
   const int32_t *page_table;
   uint16_t *out;           // [n][hq][d] bf16
   float *lse;              // [hq][n] natural log, or null
-  float *part_o;           // [n_items][kBM][d] fp32 (normalised partial outputs)
-  float *part_lse;         // [n_items][kBM] fp32 (log2 domain)
+  // Split partials, one row per query row of an item (pair: 2 x kBM rows):
+  // the normalised output O / l scaled by its row's largest magnitude s and
+  // rounded to fp16 (|value| <= 1: 2^-12 of s at most), s itself, and the
+  // log2-sum-exp.  A row of zeros has s = 0.
+  uint16_t *part_o;        // [rows][d] fp16 bits
+  float *part_scale;       // [rows] s
+  float *part_lse;         // [rows] fp32 (log2 domain)
   uint32_t *err;
   int64_t L;               // cached tokens before this call
   int32_t n, hq, hkv, group, page_size, rows_cap, n_tiles, n_pages_valid, pool_pages;
@@ -118,7 +123,8 @@ static_assert(sizeof(StepParams) <= 32000, "kernel parameters of the fused launc
 
 // K3: merge of split partials (rebuild launches and the no-allocation block path).
 struct MergeParams {
-  const float *part_o;
+  const uint16_t *part_o;  // as AttnParams
+  const float *part_scale;
   const float *part_lse;
   uint16_t *out;
   float *lse;

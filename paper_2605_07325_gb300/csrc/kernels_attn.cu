@@ -50,6 +50,7 @@
 // first global access.  Every wait (mbarriers, device counters) is bounded
 // and reports CSR_DEVERR_WAIT_TIMEOUT.
 #include <cuda_bf16.h>
+#include <cuda_fp16.h>
 #include <math_constants.h>
 
 #include "../../include/csr.h"
@@ -215,6 +216,35 @@ __device__ __forceinline__ float2 ld_cg_f2(const float *ptr) {
   float2 v;
   asm volatile("ld.global.cg.v2.f32 {%0, %1}, [%2];" : "=f"(v.x), "=f"(v.y) : "l"(ptr));
   return v;
+}
+// fp16 partial rows: 8, 4 or 2 values per load, converted in pairs
+__device__ __forceinline__ uint4 ld_cg_u4(const void *ptr) {
+  uint4 v;
+  asm volatile("ld.global.cg.v4.u32 {%0, %1, %2, %3}, [%4];"
+               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+               : "l"(ptr));
+  return v;
+}
+__device__ __forceinline__ uint2 ld_cg_u2(const void *ptr) {
+  uint2 v;
+  asm volatile("ld.global.cg.v2.u32 {%0, %1}, [%2];" : "=r"(v.x), "=r"(v.y) : "l"(ptr));
+  return v;
+}
+__device__ __forceinline__ uint32_t ld_cg_u1(const void *ptr) {
+  uint32_t v;
+  asm volatile("ld.global.cg.u32 %0, [%1];" : "=r"(v) : "l"(ptr));
+  return v;
+}
+__device__ __forceinline__ float2 half2_to_f2(uint32_t u) {
+  __half2 h;
+  memcpy(&h, &u, 4);
+  return __half22float2(h);
+}
+__device__ __forceinline__ uint32_t f2_to_half2(float lo, float hi) {
+  const __half2 h = __floats2half2_rn(lo, hi);
+  uint32_t u;
+  memcpy(&u, &h, 4);
+  return u;
 }
 
 // ============================================================ configuration
@@ -592,27 +622,30 @@ __device__ __noinline__ bool step_merge_share(const StepParams &p, const Seg &se
     float acc[kPer];
 #pragma unroll
     for (int c = 0; c < kPer; ++c) acc[c] = 0.f;
-    const float *o_r = A.part_o + (s0 * kPairRows + r) * HD + lane * kPer;
+    const float *sc_r = A.part_scale + s0 * kPairRows + r;
+    const uint16_t *o_r = A.part_o + (s0 * kPairRows + r) * HD + lane * kPer;
     for (int k0 = 0; k0 < cnt; k0 += 8) {
-      float lk[8], v[8][kPer];
+      float lk[8], sk[8], v[8][kPer];
 #pragma unroll
       for (int e = 0; e < 8; ++e) {
         if (k0 + e < cnt) {
           const int64_t off = static_cast<int64_t>(k0 + e) * kPairRows;
           lk[e] = ld_cg_f(lse_r + off);
+          sk[e] = ld_cg_f(sc_r + off);
           if constexpr (kPer == 4) {
-            const float4 x = ld_cg_f4(o_r + off * HD);
-            v[e][0] = x.x; v[e][1] = x.y; v[e][2] = x.z; v[e][3] = x.w;
+            const uint2 x = ld_cg_u2(o_r + off * HD);
+            const float2 a = half2_to_f2(x.x), b = half2_to_f2(x.y);
+            v[e][0] = a.x; v[e][1] = a.y; v[e][2] = b.x; v[e][3] = b.y;
           } else {
-            const float2 x = ld_cg_f2(o_r + off * HD);
-            v[e][0] = x.x; v[e][1] = x.y;
+            const float2 a = half2_to_f2(ld_cg_u1(o_r + off * HD));
+            v[e][0] = a.x; v[e][1] = a.y;
           }
         }
       }
 #pragma unroll
       for (int e = 0; e < 8; ++e) {
         if (k0 + e < cnt) {
-          const float w = lse == -CUDART_INF_F ? 0.f : ex2_approx(lk[e] - lse);
+          const float w = lse == -CUDART_INF_F ? 0.f : ex2_approx(lk[e] - lse) * sk[e];
 #pragma unroll
           for (int c = 0; c < kPer; ++c) acc[c] = fmaf(w, v[e][c], acc[c]);
         }
@@ -1108,19 +1141,23 @@ __global__ void __launch_bounds__(kPairThreads, 1)
           for (int k = 0; k < seg.merges; ++k) {
             const int64_t rk = r0 + k * kPairRows;
             const float lk = ld_cg_f(A.part_lse + rk);
-            const float wk = lse_t == -CUDART_INF_F ? 0.f : ex2_approx(lk - lse_t);
-            const float *src = A.part_o + rk * HD;
+            const float wk = lse_t == -CUDART_INF_F ? 0.f : ex2_approx(lk - lse_t) * ld_cg_f(A.part_scale + rk);
+            const uint16_t *src = A.part_o + rk * HD;
 #pragma unroll
-            for (int c0 = 0; c0 < HD; c0 += 16) {
-              float4 v[4];
+            for (int c0 = 0; c0 < HD; c0 += 32) {
+              uint4 v[4];
 #pragma unroll
-              for (int e = 0; e < 4; ++e) v[e] = ld_cg_f4(src + c0 + 4 * e);
+              for (int e = 0; e < 4; ++e) v[e] = ld_cg_u4(src + c0 + 8 * e);
 #pragma unroll
               for (int e = 0; e < 4; ++e) {
-                o[c0 + 4 * e + 0] = __float_as_uint(fmaf(wk, v[e].x, __uint_as_float(o[c0 + 4 * e + 0])));
-                o[c0 + 4 * e + 1] = __float_as_uint(fmaf(wk, v[e].y, __uint_as_float(o[c0 + 4 * e + 1])));
-                o[c0 + 4 * e + 2] = __float_as_uint(fmaf(wk, v[e].z, __uint_as_float(o[c0 + 4 * e + 2])));
-                o[c0 + 4 * e + 3] = __float_as_uint(fmaf(wk, v[e].w, __uint_as_float(o[c0 + 4 * e + 3])));
+                const uint32_t q[4] = {v[e].x, v[e].y, v[e].z, v[e].w};
+#pragma unroll
+                for (int h = 0; h < 4; ++h) {
+                  const float2 f = half2_to_f2(q[h]);
+                  const int c = c0 + 8 * e + 2 * h;
+                  o[c] = __float_as_uint(fmaf(wk, f.x, __uint_as_float(o[c])));
+                  o[c + 1] = __float_as_uint(fmaf(wk, f.y, __uint_as_float(o[c + 1])));
+                }
               }
             }
           }
@@ -1146,15 +1183,22 @@ __global__ void __launch_bounds__(kPairThreads, 1)
         }
       } else {
         const int64_t base = static_cast<int64_t>(seg.slot) * kPairRows + wg * kBM + row;
-        // the partial buffer is 256-byte aligned and rows are HD floats: 32-byte stores
-        float *dst = A.part_o + base * HD;
+        // the row scaled by its largest magnitude, in fp16 (the partial
+        // buffer is 256-byte aligned and rows are HD halves: 32-byte stores)
+        float mx = 0.f;
 #pragma unroll
-        for (int c = 0; c < HD / 8; ++c) {
+        for (int c = 0; c < HD; ++c) mx = fmaxf(mx, fabsf(__uint_as_float(o[c])));
+        const float inv_s = mx > 0.f ? 1.0f / mx : 0.f;
+        uint16_t *dst = A.part_o + base * HD;
+#pragma unroll
+        for (int c = 0; c < HD / 16; ++c) {
           uint32_t w[8];
 #pragma unroll
-          for (int e = 0; e < 8; ++e) w[e] = __float_as_uint(__uint_as_float(o[8 * c + e]) * inv_l);
-          st_global_v8(dst + 8 * c, w);
+          for (int e = 0; e < 8; ++e)
+            w[e] = f2_to_half2(__uint_as_float(o[16 * c + 2 * e]) * inv_s, __uint_as_float(o[16 * c + 2 * e + 1]) * inv_s);
+          st_global_v8(dst + 16 * c, w);
         }
+        A.part_scale[base] = mx * inv_l;
         A.part_lse[base] = lse2;
         if constexpr (kStep) {
           // this warp's 32 rows are written: raise the slot's flag for the
@@ -1186,19 +1230,32 @@ __global__ void __launch_bounds__(kPairThreads, 1)
 }
 
 // ------------------------------------------------------------------ K3 merge
-// 32-byte global loads (the partial buffer is 256-byte aligned and its rows
-// are HD floats, so every lane's eight floats start on a 32-byte boundary).
-__device__ __forceinline__ void ld_global_v8f(const float *ptr, float (&v)[8]) {
-  asm volatile("ld.global.v8.f32 {%0, %1, %2, %3, %4, %5, %6, %7}, [%8];"
-               : "=f"(v[0]), "=f"(v[1]), "=f"(v[2]), "=f"(v[3]), "=f"(v[4]), "=f"(v[5]), "=f"(v[6]),
-                 "=f"(v[7])
+// 16-byte global loads of eight fp16 values (the partial buffer is 256-byte
+// aligned and its rows are HD halves, so every lane's eight start on a
+// 16-byte boundary), converted when used.
+__device__ __forceinline__ uint4 ld_global_u4(const void *ptr) {
+  uint4 v;
+  asm volatile("ld.global.v4.u32 {%0, %1, %2, %3}, [%4];"
+               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
                : "l"(ptr));
+  return v;
+}
+// acc += w * (the eight fp16 values in q)
+__device__ __forceinline__ void fma_half8(float (&acc)[8], float w, const uint4 &q) {
+  const uint32_t h[4] = {q.x, q.y, q.z, q.w};
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const float2 f = half2_to_f2(h[i]);
+    acc[2 * i] = fmaf(w, f.x, acc[2 * i]);
+    acc[2 * i + 1] = fmaf(w, f.y, acc[2 * i + 1]);
+  }
 }
 
 // K3: combine the split-KV partials of every row: lse = log2(sum_k 2^lse_k),
-// out = sum_k 2^(lse_k - lse) * O_k (each O_k already normalised by its own
-// row sum).  A row is read by a group of HD / 8 lanes (eight floats, one
-// 32-byte load per lane per chunk); a block of 256 threads holds 256 / (HD/8)
+// out = sum_k 2^(lse_k - lse) * s_k * O'_k (O_k = s_k O'_k, normalised by its
+// own row sum, stored as fp16 O'_k with its scale s_k).  A row is read by a
+// group of HD / 8 lanes (eight values, one 16-byte load per lane per chunk);
+// a block of 256 threads holds 256 / (HD/8)
 // such slots.  The merge is bound by how many bytes are in flight, so every
 // load of a slot -- the LSEs of all chunks and up to kMergeChunksPerSlot
 // partial rows -- is issued before any is used; rows with more chunks are
@@ -1260,17 +1317,19 @@ __global__ void __launch_bounds__(256, 4) merge_kernel(const __grid_constant__ M
     }
     // this slot's chunks: their partial rows and (the same address on every
     // lane of the slot) their LSEs
-    float v[kC][8], lk[kC];
+    uint4 v[kC];
+    float lk[kC], sk[kC];
 #pragma unroll
     for (int u = 0; u < kC; ++u) {
       const int k = sub + u * spr;
       if (valid && k < nk) {
         lk[u] = p.part_lse[prow(k)];
-        ld_global_v8f(p.part_o + prow(k) * HD + sl * 8, v[u]);
+        sk[u] = p.part_scale[prow(k)];
+        v[u] = ld_global_u4(p.part_o + prow(k) * HD + sl * 8);
       } else {
         lk[u] = -CUDART_INF_F;
-#pragma unroll
-        for (int e = 0; e < 8; ++e) v[u][e] = 0.f;
+        sk[u] = 0.f;
+        v[u] = make_uint4(0u, 0u, 0u, 0u);
       }
     }
     float mx = l[0];
@@ -1285,11 +1344,7 @@ __global__ void __launch_bounds__(256, 4) merge_kernel(const __grid_constant__ M
     lse2 = sum > 0.f ? m_use + log2f(sum) : -CUDART_INF_F;
     if (sum > 0.f) {
 #pragma unroll
-      for (int u = 0; u < kC; ++u) {
-        const float w = ex2_approx(lk[u] - lse2);
-#pragma unroll
-        for (int x = 0; x < 8; ++x) acc[x] = fmaf(w, v[u][x], acc[x]);
-      }
+      for (int u = 0; u < kC; ++u) fma_half8(acc, ex2_approx(lk[u] - lse2) * sk[u], v[u]);
     }
   } else {
     float mx = -CUDART_INF_F;
@@ -1303,11 +1358,8 @@ __global__ void __launch_bounds__(256, 4) merge_kernel(const __grid_constant__ M
     if (valid && sum > 0.f) {
       for (int k = sub; k < nk; k += spr) {
         const int64_t base = prow(k);
-        const float w = ex2_approx(p.part_lse[base] - lse2);
-        float v[8];
-        ld_global_v8f(p.part_o + base * HD + sl * 8, v);
-#pragma unroll
-        for (int x = 0; x < 8; ++x) acc[x] = fmaf(w, v[x], acc[x]);
+        const float w = ex2_approx(p.part_lse[base] - lse2) * p.part_scale[base];
+        fma_half8(acc, w, ld_global_u4(p.part_o + base * HD + sl * 8));
       }
     }
   }

@@ -296,3 +296,36 @@ def test_local_schedule_matches_oracle(libcsr, num_ctas):
     p.truncate()
     p.check_layout()
     p.device_clean()
+
+
+def _scale_v(b, shift):
+    """The block with V multiplied by 2^shift, exactly (bf16 exponent field)."""
+    v = b.v.copy()
+    nz = (v & 0x7FFF) != 0
+    v[nz] = v[nz] + np.uint16(shift << 7)
+    return synth.Block(b.q, b.k, v)
+
+
+@pytest.mark.parametrize("path", ["fused", "three"])
+def test_split_partials_scale_exactly(libcsr, path):
+    """Split partials are stored as fp16 rows scaled by their largest
+    magnitude.  Values 2^15 times larger (|V| well past 65,504, the largest
+    fp16 value) must give exactly 2^15 times the outputs: every step of the
+    path, the partials and their merge included, scales exactly by a power of
+    two.  Short key chunks make every unit split on both paths."""
+    outs = []
+    for shift in (0, 15):
+        p = Pair(C2, pool_pages=128, max_seq=8192, max_new=1024, fg_chunk_tiles=2, flags=PATHS[path])
+        b0, b1 = p.blk(90, 1500), p.blk(91, 300)
+        if shift:
+            b0, b1 = _scale_v(b0, shift), _scale_v(b1, shift)
+        p.init_static(b0, compare=False)
+        q, k, v = p._dev(b1)
+        out, _ = p.ctx.attend_suffix(q, k, v)
+        torch.cuda.synchronize()
+        outs.append(to_f64(out))
+        p.ctx.truncate_suffix()
+        p.device_clean()
+    assert np.max(np.abs(outs[0])) > 0.1
+    assert np.max(np.abs(outs[1])) > 65504.0
+    assert np.array_equal(outs[1], outs[0] * 2.0 ** 15)
