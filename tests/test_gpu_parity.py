@@ -309,14 +309,15 @@ def _scale_v(b, shift):
 @pytest.mark.parametrize("path", ["fused", "three"])
 def test_split_partials_scale_exactly(libcsr, path):
     """Split partials are stored as fp16 rows scaled by their largest
-    magnitude.  Values 2^15 times larger (|V| well past 65,504, the largest
-    fp16 value) must give exactly 2^15 times the outputs: every step of the
-    path, the partials and their merge included, scales exactly by a power of
-    two.  Short key chunks make every unit split on both paths."""
+    magnitude.  Values 2^20 times larger (outputs, averages of V, and the
+    partial rows well past 65,504, the largest fp16 value) must give exactly
+    2^20 times the outputs: every step of the path, the partials and their
+    merge included, scales exactly by a power of two.  Short key chunks make
+    every unit split on both paths."""
     outs = []
-    for shift in (0, 15):
+    for shift in (0, 20):
         p = Pair(C2, pool_pages=128, max_seq=8192, max_new=1024, fg_chunk_tiles=2, flags=PATHS[path])
-        b0, b1 = p.blk(90, 1500), p.blk(91, 300)
+        b0, b1 = p.blk(90, 1000), p.blk(91, 300)
         if shift:
             b0, b1 = _scale_v(b0, shift), _scale_v(b1, shift)
         p.init_static(b0, compare=False)
@@ -328,4 +329,4 @@ def test_split_partials_scale_exactly(libcsr, path):
         p.device_clean()
     assert np.max(np.abs(outs[0])) > 0.1
     assert np.max(np.abs(outs[1])) > 65504.0
-    assert np.array_equal(outs[1], outs[0] * 2.0 ** 15)
+    assert np.array_equal(outs[1], outs[0] * 2.0 ** 20)
